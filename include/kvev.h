@@ -1,0 +1,185 @@
+/*
+ * kvev.h -- C ABI of the GB300 layer-wise KV-cache eviction library (libkvev.so).
+ *
+ * The library executes a static layer-wise eviction plan (Sec. 3.1, Eq. 1 of
+ * "Exploring a Layer-Wise Design Space for KV Cache Eviction"): every layer l
+ * has, per inference phase, an operator r_l (a retention rule, or FULL = no
+ * eviction in that phase) and a nominal retained-token capacity b_l.  At the
+ * prefill eviction point it scores the prompt keys of every layer with the
+ * rule that layer is routed to, selects the positions to keep per
+ * (sequence, KV head) and gather-compacts K/V into a packed smaller cache.
+ * The per-layer capacities can be produced by the allocator of Sec. 3.3
+ * (Eq. 3 and its b_min clamping and largest-remainder rounding).
+ *
+ * Conventions shared by every entry point
+ *   - Return value: KVEV_OK (0) or one of the KVEV_E* codes below.  Arguments
+ *     are validated before any device work is enqueued; on a non-zero return
+ *     nothing was enqueued.
+ *   - Device buffers are caller-owned raw device pointers (16-byte aligned
+ *     where noted); host arrays are plain host pointers read during the call
+ *     and not retained.  The library never frees caller memory.
+ *   - Device work is enqueued asynchronously on the caller's stream, passed as
+ *     a `void *` holding a cudaStream_t (NULL = legacy default stream).
+ *     Faults the kernels detect themselves (a bounded wait that ran out, a
+ *     layout check) are recorded in a device status word read by kvev_status().
+ *   - bf16 tensors are raw 16-bit patterns; layouts are row-major C order.
+ *   - Threading: a plan may be used by one host thread at a time.
+ */
+#ifndef KVEV_H
+#define KVEV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define KVEV_OK 0
+#define KVEV_EINVAL 1   /* bad argument: shape, pointer, alignment or rule parameter */
+#define KVEV_ENOMEM 2   /* host or device allocation failed, or workspace too small */
+#define KVEV_ECUDA 3    /* a CUDA runtime/driver call failed (e.g. no device) */
+#define KVEV_ETIMEOUT 4 /* device: a bounded wait ran out (see kvev_status) */
+#define KVEV_EDEVICE 5  /* device: an in-kernel consistency check failed */
+#define KVEV_ENOTSUP 6  /* valid request outside what this build supports */
+
+/* ---- operators (the retention rules a layer can be routed to) ----------- */
+#define KVEV_FULL 0      /* no eviction in this phase (Sec. 3.1) */
+#define KVEV_SNAPKV 1    /* observation-window attention + 1-D pooling, top-k (prefill) */
+#define KVEV_H2O 2       /* accumulated attention heavy hitters + recent window (both phases) */
+#define KVEV_STREAMING 3 /* attention sinks + most recent tokens (both phases) */
+#define KVEV_TOVA 4      /* evict the token the current query attends to least (decode only) */
+
+#define KVEV_POOL_MAX 0
+#define KVEV_POOL_AVG 1
+
+#define KVEV_T_IDENTITY 0 /* allocation transform for entropy scores (Sec. 3.3) */
+#define KVEV_T_CAP_Q95 1  /* cap at the across-layer 95th percentile (PPL scores, Sec. 3.3) */
+
+typedef struct kvev_plan kvev_plan;
+
+/* ---- capacity allocation (host only; no GPU needed) ---------------------- */
+
+/* Sec. 3.3, Eq. 3: per-layer capacities from layer scores s[0..L).
+ *   t_l = T(s_l) (identity, or min(s_l, Q_0.95(s)) with type-7 interpolation);
+ *   if min t <= 0 every t is shifted by -min t + 1e-6;
+ *   w_l = t_l / sum t;  b~_l = B_total * w_l;
+ *   layers with b~_l < b_min are fixed at b_min and the remaining capacity is
+ *   re-split over the other layers in proportion to w, until none drops below;
+ *   the result is rounded by largest remainder (ties to the lower layer).
+ * Output: budget_out[0..L) with sum == B_total and every entry >= b_min.
+ * EINVAL if L <= 0, b_min < 0, L*b_min > B_total, or any s is not finite. */
+int kvev_alloc_from_scores(int32_t *budget_out, const double *s, int L, int64_t B_total,
+                           int b_min, int transform);
+
+/* Sec. 3.3 (budget sweep): scale a completed vector budget_in[0..L) to the
+ * total B_target (b_l * B_target / sum budget_in) and round by largest
+ * remainder; no b_min is re-applied.  EINVAL if the input sum is <= 0. */
+int kvev_alloc_rescale(int32_t *budget_out, const int32_t *budget_in, int L, int64_t B_target);
+
+/* ---- plan ---------------------------------------------------------------- */
+
+/* Create the static plan of Eq. 1 (host memory only; no device work).
+ *   L, H_q, H_kv, d      model geometry; H_q must be a multiple of H_kv.
+ *   route_prefill[L]     operator per layer at the prefill eviction point:
+ *                        KVEV_FULL, KVEV_SNAPKV, KVEV_H2O or KVEV_STREAMING.
+ *   route_decode[L]      operator per layer in the decode phase (KVEV_FULL,
+ *                        KVEV_H2O, KVEV_TOVA, KVEV_STREAMING); NULL = all FULL.
+ *   budget[L]            nominal capacity b_l (ignored for FULL layers).
+ *   window               observation window W of the scoring rules (SnapKV, H2O).
+ *   pool_kernel          SnapKV pooling width (odd, >= 1); pool_type KVEV_POOL_*.
+ *   sink                 StreamingLLM attention-sink tokens.
+ *   recent               StreamingLLM recent tokens; -1 = b_l - sink per layer,
+ *                        otherwise min(recent, b_l - sink).
+ *   h2o_recent           H2O protected recent window; -1 = floor(b_l / 2).
+ * EINVAL: a SnapKV layer with b_l <= window, a StreamingLLM layer with
+ * b_l <= sink, an H2O layer with b_l < 1 or h2o_recent > b_l, an even or
+ * non-positive pool_kernel with a SnapKV layer, window < 1 with a scoring
+ * layer, or a decode route that is not FULL/H2O/TOVA/STREAMING.
+ * ENOTSUP: d not 64 or 128, G*window > 256 (G = H_q/H_kv) with a scoring
+ * layer, or more than 64 scoring layers. */
+int kvev_plan_create(kvev_plan **out, int L, int H_q, int H_kv, int d,
+                     const int32_t *route_prefill, const int32_t *route_decode,
+                     const int32_t *budget, int window, int pool_kernel, int pool_type,
+                     int sink, int recent, int h2o_recent);
+
+/* Release the plan and the small device status buffer it may hold. */
+void kvev_plan_destroy(kvev_plan *plan);
+
+/* Sizes of the buffers kvev_evict_prefill() needs for a batch of B sequences
+ * stored in caches of S_cap positions (any pointer may be NULL):
+ *   out_kv_bytes    bytes of out_K (and, separately, of out_V): sum over
+ *                   non-FULL layers of B*H_kv*b_l rows of d bf16;
+ *   out_idx_bytes   bytes of out_idx (int32 per output row; also the size of
+ *                   h2o_state in floats * 4);
+ *   count_bytes     bytes of out_count (int32 [L][B][H_kv]);
+ *   workspace_bytes device scratch for one call.
+ * Worked example (App. E): L=32, b=512, B=1, H_kv=8, d=128 gives
+ * 16,384 layer-token positions and 2*out_kv_bytes = 64.00 MiB of K+V. */
+int kvev_plan_query(const kvev_plan *plan, int B, int S_cap, size_t *out_kv_bytes,
+                    size_t *out_idx_bytes, size_t *count_bytes, size_t *workspace_bytes);
+
+/* First packed output row of `layer` for a batch of B sequences; the row of
+ * (layer, seq s, kv head h, slot j) is row_offset + (s*H_kv + h)*b_l + j.
+ * FULL layers own no rows (the caller keeps their cache as it is). */
+int kvev_plan_layer_offset(const kvev_plan *plan, int B, int layer, int64_t *row_offset);
+
+/* Prefill eviction of every layer of the plan in grouped launches.
+ *   K[L], V[L]     host arrays of device pointers; layer l's cache is bf16
+ *                  [B][H_kv][S_cap][d] (16-byte aligned).  Entries of FULL
+ *                  layers may be NULL.
+ *   Q_win[L]       host array of device pointers to the observation-window
+ *                  queries, bf16 [B][H_q][W][d] (16-byte aligned); query i of
+ *                  the window sits at position lens[s] - W + i.  Needed for
+ *                  SnapKV and H2O layers, may be NULL elsewhere.
+ *   lens_dev       device int32 [B]: valid length of each sequence, 0..S_cap.
+ *   out_K, out_V   device bf16, packed rows (see kvev_plan_layer_offset): row
+ *                  j of (l, s, h) is K[l][s][h][out_idx[row]]; slots past the
+ *                  kept count hold zeros.  16-byte aligned.
+ *   out_idx        device int32 per output row: kept positions in ascending
+ *                  order, -1 in unused slots.
+ *   out_count      device int32 [L][B][H_kv]: kept count (= min(b_l, lens[s])
+ *                  for capacity-controlled layers; lens[s] for FULL layers).
+ *   h2o_state      device fp32 per output row (nullable): for H2O layers the
+ *                  window attention score of each kept token, the initial
+ *                  accumulated-attention state of the decode phase.
+ *   workspace      device scratch of at least the queried size (256-byte
+ *                  aligned); contents need no initialisation.
+ * The rules are the ones Sec. 2.1 cites, at the layer's capacity b_l:
+ *   SnapKV: score[k] = (1/G) sum over the G query heads of the group and the
+ *     W window rows of softmax(q K^T / sqrt(d))[k] (causal inside the window,
+ *     normalised over every visible key); pooled over [0, n-W) with width
+ *     pool_kernel (max, or average with zero padding divided by the width);
+ *     keep the last W positions plus the top (b_l - W) pooled prefix scores.
+ *   H2O: the same window score without pooling; keep the last h2o_recent
+ *     positions plus the top (b_l - h2o_recent) scores before them.
+ *   StreamingLLM: keep positions [0, sink) and the last `recent` positions.
+ *   Any rule with b_l >= lens[s] keeps every position.
+ * Top-k ties keep the lower position.
+ * EINVAL on null/misaligned pointers or B < 0, S_cap < 1; ENOMEM if the
+ * workspace is smaller than kvev_plan_query() reports. */
+int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const *V,
+                       const void *const *Q_win, const int32_t *lens_dev, int B, int S_cap,
+                       void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
+                       float *h2o_state, void *workspace, size_t workspace_bytes, void *stream);
+
+/* Synchronise the plan's last stream and read-and-clear the device status
+ * word: *device_status receives KVEV_OK, KVEV_ETIMEOUT or KVEV_EDEVICE.
+ * Returns ECUDA if the readback itself failed. */
+int kvev_status(kvev_plan *plan, int *device_status);
+
+/* Bound (in nanoseconds) of every in-kernel wait; a wait that runs out
+ * records KVEV_ETIMEOUT and the kernel finishes without producing valid
+ * scores for the affected units.  Default 2e9 (2 s). */
+int kvev_plan_set_wait_limit(kvev_plan *plan, int64_t ns);
+
+/* Test hook: when `unit` >= 0 the score kernel never marks that scoring unit
+ * as ready, so every wait on it runs out after the wait limit.  Used only to
+ * exercise the timeout path; -1 disables it. */
+int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVEV_H */
