@@ -35,6 +35,12 @@
 extern "C" {
 #endif
 
+#if defined(__GNUC__)
+#define KVEV_API __attribute__((visibility("default")))
+#else
+#define KVEV_API
+#endif
+
 /* ---- status codes ------------------------------------------------------ */
 #define KVEV_OK 0
 #define KVEV_EINVAL 1   /* bad argument: shape, pointer, alignment or rule parameter */
@@ -70,13 +76,13 @@ typedef struct kvev_plan kvev_plan;
  *   the result is rounded by largest remainder (ties to the lower layer).
  * Output: budget_out[0..L) with sum == B_total and every entry >= b_min.
  * EINVAL if L <= 0, b_min < 0, L*b_min > B_total, or any s is not finite. */
-int kvev_alloc_from_scores(int32_t *budget_out, const double *s, int L, int64_t B_total,
+KVEV_API int kvev_alloc_from_scores(int32_t *budget_out, const double *s, int L, int64_t B_total,
                            int b_min, int transform);
 
 /* Sec. 3.3 (budget sweep): scale a completed vector budget_in[0..L) to the
  * total B_target (b_l * B_target / sum budget_in) and round by largest
  * remainder; no b_min is re-applied.  EINVAL if the input sum is <= 0. */
-int kvev_alloc_rescale(int32_t *budget_out, const int32_t *budget_in, int L, int64_t B_target);
+KVEV_API int kvev_alloc_rescale(int32_t *budget_out, const int32_t *budget_in, int L, int64_t B_target);
 
 /* ---- plan ---------------------------------------------------------------- */
 
@@ -99,13 +105,13 @@ int kvev_alloc_rescale(int32_t *budget_out, const int32_t *budget_in, int L, int
  * layer, or a decode route that is not FULL/H2O/TOVA/STREAMING.
  * ENOTSUP: d not 64 or 128, G*window > 256 (G = H_q/H_kv) with a scoring
  * layer, or more than 64 scoring layers. */
-int kvev_plan_create(kvev_plan **out, int L, int H_q, int H_kv, int d,
+KVEV_API int kvev_plan_create(kvev_plan **out, int L, int H_q, int H_kv, int d,
                      const int32_t *route_prefill, const int32_t *route_decode,
                      const int32_t *budget, int window, int pool_kernel, int pool_type,
                      int sink, int recent, int h2o_recent);
 
 /* Release the plan and the small device status buffer it may hold. */
-void kvev_plan_destroy(kvev_plan *plan);
+KVEV_API void kvev_plan_destroy(kvev_plan *plan);
 
 /* Sizes of the buffers kvev_evict_prefill() needs for a batch of B sequences
  * stored in caches of S_cap positions (any pointer may be NULL):
@@ -117,13 +123,21 @@ void kvev_plan_destroy(kvev_plan *plan);
  *   workspace_bytes device scratch for one call.
  * Worked example (App. E): L=32, b=512, B=1, H_kv=8, d=128 gives
  * 16,384 layer-token positions and 2*out_kv_bytes = 64.00 MiB of K+V. */
-int kvev_plan_query(const kvev_plan *plan, int B, int S_cap, size_t *out_kv_bytes,
+KVEV_API int kvev_plan_query(const kvev_plan *plan, int B, int S_cap, size_t *out_kv_bytes,
                     size_t *out_idx_bytes, size_t *count_bytes, size_t *workspace_bytes);
 
 /* First packed output row of `layer` for a batch of B sequences; the row of
  * (layer, seq s, kv head h, slot j) is row_offset + (s*H_kv + h)*b_l + j.
  * FULL layers own no rows (the caller keeps their cache as it is). */
-int kvev_plan_layer_offset(const kvev_plan *plan, int B, int layer, int64_t *row_offset);
+KVEV_API int kvev_plan_layer_offset(const kvev_plan *plan, int B, int layer, int64_t *row_offset);
+
+/* Where a call leaves the window scores of a SnapKV/H2O layer: after
+ * kvev_evict_prefill() returns (and its stream is synchronised), the bytes at
+ * workspace + *byte_offset hold fp32 [B][H_kv][S_cap] scores of `layer`
+ * (entry k of (s, h) valid for k < lens[s]; see the rule description below),
+ * until the workspace is reused.  EINVAL if the layer has no scores. */
+KVEV_API int kvev_plan_scores_offset(const kvev_plan *plan, int B, int S_cap, int layer,
+                                     size_t *byte_offset);
 
 /* Prefill eviction of every layer of the plan in grouped launches.
  *   K[L], V[L]     host arrays of device pointers; layer l's cache is bf16
@@ -159,7 +173,7 @@ int kvev_plan_layer_offset(const kvev_plan *plan, int B, int layer, int64_t *row
  * Top-k ties keep the lower position.
  * EINVAL on null/misaligned pointers or B < 0, S_cap < 1; ENOMEM if the
  * workspace is smaller than kvev_plan_query() reports. */
-int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const *V,
+KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const *V,
                        const void *const *Q_win, const int32_t *lens_dev, int B, int S_cap,
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
                        float *h2o_state, void *workspace, size_t workspace_bytes, void *stream);
@@ -167,17 +181,17 @@ int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const 
 /* Synchronise the plan's last stream and read-and-clear the device status
  * word: *device_status receives KVEV_OK, KVEV_ETIMEOUT or KVEV_EDEVICE.
  * Returns ECUDA if the readback itself failed. */
-int kvev_status(kvev_plan *plan, int *device_status);
+KVEV_API int kvev_status(kvev_plan *plan, int *device_status);
 
 /* Bound (in nanoseconds) of every in-kernel wait; a wait that runs out
  * records KVEV_ETIMEOUT and the kernel finishes without producing valid
  * scores for the affected units.  Default 2e9 (2 s). */
-int kvev_plan_set_wait_limit(kvev_plan *plan, int64_t ns);
+KVEV_API int kvev_plan_set_wait_limit(kvev_plan *plan, int64_t ns);
 
 /* Test hook: when `unit` >= 0 the score kernel never marks that scoring unit
  * as ready, so every wait on it runs out after the wait limit.  Used only to
  * exercise the timeout path; -1 disables it. */
-int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
+KVEV_API int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
 
 #ifdef __cplusplus
 }

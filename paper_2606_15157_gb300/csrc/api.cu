@@ -1,0 +1,538 @@
+// api.cu -- host side of libkvev.so: the static plan (Sec. 3.1, Eq. 1), the
+// capacity allocator (Sec. 3.3, Eq. 3), workspace layout, TMA descriptor
+// encoding and the grouped launch sequence of the prefill eviction:
+//   prologue (lengths, work items)  ->  window scores (tcgen05)  ->
+//   selection (radix top-k)          ->  gather-compaction.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <numeric>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "kvev_internal.cuh"
+
+using namespace kvev;
+
+struct kvev_plan {
+  int L = 0, H_q = 0, H_kv = 0, d = 0, G = 0;
+  int W = 0, pool_kernel = 1, pool_type = 0, sink = 0, recent = -1, h2o_recent = -1;
+  std::vector<int> route_pre, route_dec, budget;
+  std::vector<int> slots;       // output slots per (seq, head), 0 for FULL
+  std::vector<int> recent_eff;  // StreamingLLM recent kept
+  std::vector<int> h2o_r;       // H2O protected window
+  std::vector<int> score_slot;  // index among scoring layers, -1 if none
+  std::vector<int> score_layers;
+  int64_t wait_ns = 2000000000LL;
+  int stall_unit = -1;
+  // device-side state, created on first use
+  int device = -1;
+  int num_sms = 0;
+  int smem_optin = 0;
+  int* d_status = nullptr;
+  cudaStream_t last_stream = nullptr;
+  bool attrs_set = false;
+  size_t score_smem_set = 0, select_smem_set = 0;
+};
+
+namespace {
+
+constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
+
+struct WsLayout {
+  int n_units = 0, R = 0, R_pad = 0, max_items = 0;
+  size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item_unit = 0, part = 0,
+         lam = 0, raw = 0, total = 0;
+};
+
+WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
+  WsLayout w;
+  w.n_units = static_cast<int>(p.score_layers.size()) * B * p.H_kv;
+  w.R = p.G * p.W;
+  w.R_pad = (w.R + 15) / 16 * 16;
+  const int chunk_min = kTileKeys * kMinChunkTiles;
+  w.max_items = w.n_units * ((S_cap + chunk_min - 1) / chunk_min);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, kWsAlign);
+    return o;
+  };
+  w.lens = take(sizeof(int) * std::max(B, 1));
+  w.abort_flag = take(sizeof(int));
+  w.cnt = take(sizeof(int) * std::max(w.n_units, 1));
+  w.ready = take(sizeof(int) * std::max(w.n_units, 1));
+  w.chunk_start = take(sizeof(int) * (w.n_units + 1));
+  w.item_unit = take(sizeof(int) * std::max(w.max_items, 1));
+  w.part = take(sizeof(float2) * 2 * static_cast<size_t>(w.max_items) * w.R_pad);
+  w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
+  w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
+  w.total = off;
+  return w;
+}
+
+int64_t rows_per_layer(const kvev_plan& p, int B, int l) {
+  return static_cast<int64_t>(B) * p.H_kv * p.slots[l];
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 2-D bf16 map {d, rows} with a {64, box_rows} box and the 128-byte swizzle.
+bool encode_map(CUtensorMap* m, const void* base, int d, uint64_t rows, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), rows};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int ensure_device(kvev_plan* p) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return KVEV_ECUDA;
+  if (p->device == dev && p->d_status) return KVEV_OK;
+  if (p->d_status) {
+    cudaFree(p->d_status);
+    p->d_status = nullptr;
+  }
+  int major = 0;
+  if (cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&p->smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
+    return KVEV_ECUDA;
+  if (major < 10) return KVEV_ENOTSUP;
+  if (cudaMalloc(&p->d_status, sizeof(int)) != cudaSuccess) return KVEV_ENOMEM;
+  if (cudaMemset(p->d_status, 0, sizeof(int)) != cudaSuccess) return KVEV_ECUDA;
+  p->device = dev;
+  p->score_smem_set = p->select_smem_set = 0;
+  return KVEV_OK;
+}
+
+// Largest-remainder rounding of x (non-negative, sum == total): floor, then one
+// extra unit to each of the largest fractional parts, lower index first on ties.
+void round_largest_remainder(const std::vector<double>& x, int64_t total, int32_t* out) {
+  const int L = static_cast<int>(x.size());
+  std::vector<double> frac(L);
+  int64_t sum = 0;
+  for (int l = 0; l < L; ++l) {
+    const double f = std::floor(x[l]);
+    out[l] = static_cast<int32_t>(f);
+    frac[l] = x[l] - f;
+    sum += out[l];
+  }
+  std::vector<int> order(L);
+  std::iota(order.begin(), order.end(), 0);
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int a, int b) { return frac[a] > frac[b]; });
+  int64_t left = total - sum;
+  for (int i = 0; i < L && left > 0; ++i, --left) out[order[i]] += 1;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Allocation (Sec. 3.3)
+// ---------------------------------------------------------------------------
+
+extern "C" int kvev_alloc_from_scores(int32_t* budget_out, const double* s, int L,
+                                      int64_t B_total, int b_min, int transform) {
+  if (!budget_out || !s || L <= 0 || b_min < 0 || static_cast<int64_t>(L) * b_min > B_total)
+    return KVEV_EINVAL;
+  if (transform != KVEV_T_IDENTITY && transform != KVEV_T_CAP_Q95) return KVEV_EINVAL;
+  for (int l = 0; l < L; ++l)
+    if (!std::isfinite(s[l])) return KVEV_EINVAL;
+  std::vector<double> t(s, s + L);
+  if (transform == KVEV_T_CAP_Q95) {
+    std::vector<double> sorted(t);
+    std::sort(sorted.begin(), sorted.end());
+    const double h = 0.95 * (L - 1);
+    const int lo = static_cast<int>(std::floor(h));
+    double q = sorted[lo];
+    if (lo + 1 < L) q += (h - lo) * (sorted[lo + 1] - sorted[lo]);
+    for (double& v : t) v = std::min(v, q);
+  }
+  const double mn = *std::min_element(t.begin(), t.end());
+  if (mn <= 0.0)
+    for (double& v : t) v += -mn + 1e-6;
+  double tsum = 0.0;
+  for (double v : t) tsum += v;
+  std::vector<double> w(L), bt(L);
+  for (int l = 0; l < L; ++l) w[l] = t[l] / tsum;
+  std::vector<char> fixed(L, 0);
+  bool changed = true;
+  while (changed) {
+    changed = false;
+    int nfixed = 0;
+    double wfree = 0.0;
+    for (int l = 0; l < L; ++l) {
+      if (fixed[l]) ++nfixed;
+      else wfree += w[l];
+    }
+    const double rest = static_cast<double>(B_total) - static_cast<double>(nfixed) * b_min;
+    for (int l = 0; l < L; ++l)
+      bt[l] = fixed[l] ? static_cast<double>(b_min) : (wfree > 0.0 ? rest * w[l] / wfree : 0.0);
+    for (int l = 0; l < L; ++l)
+      if (!fixed[l] && bt[l] < static_cast<double>(b_min)) fixed[l] = 1, changed = true;
+  }
+  round_largest_remainder(bt, B_total, budget_out);
+  return KVEV_OK;
+}
+
+extern "C" int kvev_alloc_rescale(int32_t* budget_out, const int32_t* budget_in, int L,
+                                  int64_t B_target) {
+  if (!budget_out || !budget_in || L <= 0 || B_target < 0) return KVEV_EINVAL;
+  int64_t sum = 0;
+  for (int l = 0; l < L; ++l) {
+    if (budget_in[l] < 0) return KVEV_EINVAL;
+    sum += budget_in[l];
+  }
+  if (sum <= 0) return KVEV_EINVAL;
+  std::vector<double> x(L);
+  for (int l = 0; l < L; ++l)
+    x[l] = static_cast<double>(budget_in[l]) * (static_cast<double>(B_target) / sum);
+  round_largest_remainder(x, B_target, budget_out);
+  return KVEV_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Plan
+// ---------------------------------------------------------------------------
+
+extern "C" int kvev_plan_create(kvev_plan** out, int L, int H_q, int H_kv, int d,
+                                const int32_t* route_prefill, const int32_t* route_decode,
+                                const int32_t* budget, int window, int pool_kernel,
+                                int pool_type, int sink, int recent, int h2o_recent) {
+  if (!out) return KVEV_EINVAL;
+  *out = nullptr;
+  if (L <= 0 || H_q <= 0 || H_kv <= 0 || H_q % H_kv != 0 || d <= 0 || !route_prefill || !budget)
+    return KVEV_EINVAL;
+  if (L > kMaxLayers) return KVEV_ENOTSUP;
+  if (pool_type != KVEV_POOL_MAX && pool_type != KVEV_POOL_AVG) return KVEV_EINVAL;
+  std::unique_ptr<kvev_plan> p(new (std::nothrow) kvev_plan);
+  if (!p) return KVEV_ENOMEM;
+  p->L = L;
+  p->H_q = H_q;
+  p->H_kv = H_kv;
+  p->d = d;
+  p->G = H_q / H_kv;
+  p->W = window;
+  p->pool_kernel = pool_kernel;
+  p->pool_type = pool_type;
+  p->sink = sink;
+  p->recent = recent;
+  p->h2o_recent = h2o_recent;
+  p->route_pre.assign(route_prefill, route_prefill + L);
+  p->budget.assign(budget, budget + L);
+  p->route_dec.assign(L, KVEV_FULL);
+  if (route_decode) p->route_dec.assign(route_decode, route_decode + L);
+  p->slots.assign(L, 0);
+  p->recent_eff.assign(L, 0);
+  p->h2o_r.assign(L, 0);
+  p->score_slot.assign(L, -1);
+  bool any_scoring = false, any_snap = false;
+  for (int l = 0; l < L; ++l) {
+    const int m = p->route_pre[l], b = p->budget[l];
+    switch (m) {
+      case KVEV_FULL:
+        break;
+      case KVEV_SNAPKV:
+        if (b <= window) return KVEV_EINVAL;
+        any_snap = any_scoring = true;
+        break;
+      case KVEV_H2O: {
+        const int r = h2o_recent < 0 ? b / 2 : h2o_recent;
+        if (b < 1 || r > b) return KVEV_EINVAL;
+        p->h2o_r[l] = r;
+        any_scoring = true;
+        break;
+      }
+      case KVEV_STREAMING:
+        if (sink < 0 || b <= sink) return KVEV_EINVAL;
+        p->recent_eff[l] = recent < 0 ? b - sink : std::min(recent, b - sink);
+        break;
+      default:
+        return KVEV_EINVAL;
+    }
+    if (m != KVEV_FULL) p->slots[l] = b;
+    if (is_scoring(m)) {
+      p->score_slot[l] = static_cast<int>(p->score_layers.size());
+      p->score_layers.push_back(l);
+    }
+    const int md = p->route_dec[l];
+    if (md != KVEV_FULL && md != KVEV_H2O && md != KVEV_TOVA && md != KVEV_STREAMING)
+      return KVEV_EINVAL;
+  }
+  if (any_snap && (pool_kernel < 1 || (pool_kernel & 1) == 0)) return KVEV_EINVAL;
+  if (any_scoring) {
+    if (window < 1) return KVEV_EINVAL;
+    if (d != 64 && d != 128) return KVEV_ENOTSUP;
+    if (p->G * window > 256) return KVEV_ENOTSUP;
+    if (static_cast<int>(p->score_layers.size()) > kMaxScoreLayers) return KVEV_ENOTSUP;
+  }
+  if (d % 8 != 0) return KVEV_ENOTSUP;  // 16-byte row vectors in the gather
+  *out = p.release();
+  return KVEV_OK;
+}
+
+extern "C" void kvev_plan_destroy(kvev_plan* plan) {
+  if (!plan) return;
+  if (plan->d_status) cudaFree(plan->d_status);
+  delete plan;
+}
+
+extern "C" int kvev_plan_query(const kvev_plan* plan, int B, int S_cap, size_t* out_kv_bytes,
+                               size_t* out_idx_bytes, size_t* count_bytes,
+                               size_t* workspace_bytes) {
+  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
+  int64_t rows = 0;
+  for (int l = 0; l < plan->L; ++l) rows += rows_per_layer(*plan, B, l);
+  if (out_kv_bytes) *out_kv_bytes = static_cast<size_t>(rows) * plan->d * 2;
+  if (out_idx_bytes) *out_idx_bytes = static_cast<size_t>(rows) * sizeof(int32_t);
+  if (count_bytes) *count_bytes = static_cast<size_t>(plan->L) * B * plan->H_kv * sizeof(int32_t);
+  if (workspace_bytes) *workspace_bytes = ws_layout(*plan, B, S_cap).total;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_layer_offset(const kvev_plan* plan, int B, int layer,
+                                      int64_t* row_offset) {
+  if (!plan || !row_offset || B < 0 || layer < 0 || layer >= plan->L) return KVEV_EINVAL;
+  int64_t off = 0;
+  for (int l = 0; l < layer; ++l) off += rows_per_layer(*plan, B, l);
+  *row_offset = off;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_scores_offset(const kvev_plan* plan, int B, int S_cap, int layer,
+                                       size_t* byte_offset) {
+  if (!plan || !byte_offset || B < 0 || S_cap < 1 || layer < 0 || layer >= plan->L ||
+      plan->score_slot[layer] < 0)
+    return KVEV_EINVAL;
+  const WsLayout ws = ws_layout(*plan, B, S_cap);
+  *byte_offset = ws.raw + sizeof(float) * static_cast<size_t>(plan->score_slot[layer]) * B *
+                              plan->H_kv * S_cap;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_set_wait_limit(kvev_plan* plan, int64_t ns) {
+  if (!plan || ns <= 0) return KVEV_EINVAL;
+  plan->wait_ns = ns;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_debug_stall_unit(kvev_plan* plan, int unit) {
+  if (!plan) return KVEV_EINVAL;
+  plan->stall_unit = unit;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_status(kvev_plan* plan, int* device_status) {
+  if (!plan || !device_status) return KVEV_EINVAL;
+  *device_status = KVEV_OK;
+  if (!plan->d_status) return KVEV_OK;
+  if (cudaStreamSynchronize(plan->last_stream) != cudaSuccess) return KVEV_ECUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, plan->d_status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemset(plan->d_status, 0, sizeof(int)) != cudaSuccess)
+    return KVEV_ECUDA;
+  *device_status = (v & kStatusTimeout) ? KVEV_ETIMEOUT : (v & kStatusDevice) ? KVEV_EDEVICE : 0;
+  return KVEV_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Prefill eviction
+// ---------------------------------------------------------------------------
+
+extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const void* const* V,
+                                  const void* const* Q_win, const int32_t* lens_dev, int B,
+                                  int S_cap, void* out_K, void* out_V, int32_t* out_idx,
+                                  int32_t* out_count, float* h2o_state, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
+  kvev_plan& P = *plan;
+  if (B == 0) return KVEV_OK;
+  if (!K || !V || !lens_dev || !out_count || !workspace) return KVEV_EINVAL;
+  if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
+  int64_t total_rows = 0;
+  for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
+  if (total_rows > 0 && (!out_K || !out_V || !out_idx)) return KVEV_EINVAL;
+  if (!aligned16(out_K) || !aligned16(out_V) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return KVEV_EINVAL;
+  for (int l = 0; l < P.L; ++l) {
+    if (P.route_pre[l] == KVEV_FULL) continue;
+    if (!K[l] || !V[l] || !aligned16(K[l]) || !aligned16(V[l])) return KVEV_EINVAL;
+    if (is_scoring(P.route_pre[l]) && (!Q_win || !Q_win[l] || !aligned16(Q_win[l])))
+      return KVEV_EINVAL;
+  }
+  const WsLayout ws = ws_layout(P, B, S_cap);
+  if (workspace_bytes < ws.total) return KVEV_ENOMEM;
+  int rc = ensure_device(plan);
+  if (rc != KVEV_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P.last_stream = s;
+  uint8_t* wsb = static_cast<uint8_t*>(workspace);
+  int* lens_ok = reinterpret_cast<int*>(wsb + ws.lens);
+
+  // ---- prologue: validated lengths, work items, flag reset -------------
+  const int n_slayers = static_cast<int>(P.score_layers.size());
+  // chunk size: at least kMinChunkTiles tiles, and few enough chunks per unit
+  // that a unit never spans more than two rounds of the persistent grid
+  const int grid = P.num_sms;
+  const int tiles_max = (S_cap + kTileKeys - 1) / kTileKeys;
+  const int chunk_tiles = std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid);
+  PrologueParams pp = {};
+  pp.n_units = ws.n_units;
+  pp.B = B;
+  pp.H_kv = P.H_kv;
+  pp.chunk_keys = chunk_tiles * kTileKeys;
+  for (int i = 0; i < n_slayers; ++i) {
+    pp.slayer_method[i] = P.route_pre[P.score_layers[i]];
+    pp.slayer_budget[i] = P.budget[P.score_layers[i]];
+  }
+  pp.lens_in = lens_dev;
+  pp.lens = lens_ok;
+  pp.S_cap = S_cap;
+  pp.status = P.d_status;
+  pp.cnt = reinterpret_cast<int*>(wsb + ws.cnt);
+  pp.ready = reinterpret_cast<int*>(wsb + ws.ready);
+  pp.abort_flag = reinterpret_cast<int*>(wsb + ws.abort_flag);
+  pp.chunk_start = reinterpret_cast<int*>(wsb + ws.chunk_start);
+  pp.item_unit = reinterpret_cast<int*>(wsb + ws.item_unit);
+  if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+
+  // ---- window scores ----------------------------------------------------
+  if (ws.n_units > 0) {
+    ScoreParams sp;
+    std::memset(&sp, 0, sizeof(sp));
+    const int q_rows = ws.R_pad > 128 ? 256 : 128;
+    for (int i = 0; i < n_slayers; ++i) {
+      const int l = P.score_layers[i];
+      if (!encode_map(&sp.kmap[i], K[l], P.d, static_cast<uint64_t>(B) * P.H_kv * S_cap,
+                      kTileKeys) ||
+          !encode_map(&sp.qmap[i], Q_win[l], P.d, static_cast<uint64_t>(B) * P.H_q * P.W,
+                      ws.R_pad))
+        return KVEV_ECUDA;
+    }
+    int stages = 6;
+    while (stages >= 2 && score_smem_bytes(P.d, q_rows, ws.R_pad, stages) + 1024 > P.smem_optin)
+      --stages;
+    if (stages < 2) return KVEV_ENOTSUP;
+    // Request more than half of the SM's shared memory so exactly one CTA is
+    // resident per SM: its TMEM allocation then never waits on another CTA.
+    const size_t smem = std::max<size_t>(score_smem_bytes(P.d, q_rows, ws.R_pad, stages),
+                                         static_cast<size_t>(P.smem_optin) / 2 + 1024);
+    if (P.score_smem_set != smem) {
+      if (score_set_smem(P.d, smem) != cudaSuccess) return KVEV_ECUDA;
+      P.score_smem_set = smem;
+    }
+    sp.n_units = ws.n_units;
+    sp.B = B;
+    sp.H_kv = P.H_kv;
+    sp.H_q = P.H_q;
+    sp.G = P.G;
+    sp.W = P.W;
+    sp.R = ws.R;
+    sp.R_pad = ws.R_pad;
+    sp.S_cap = S_cap;
+    sp.chunk_keys = pp.chunk_keys;
+    sp.q_rows = q_rows;
+    sp.stages = stages;
+    sp.tmem_buf_cols = (ws.R_pad > 128) ? 256 : 128;
+    sp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));
+    sp.inv_G = 1.0f / static_cast<float>(P.G);
+    sp.lens = lens_ok;
+    sp.chunk_start = pp.chunk_start;
+    sp.item_unit = pp.item_unit;
+    sp.cnt = pp.cnt;
+    sp.ready = pp.ready;
+    sp.abort_flag = pp.abort_flag;
+    sp.status = P.d_status;
+    sp.part = reinterpret_cast<float2*>(wsb + ws.part);
+    sp.lam = reinterpret_cast<float*>(wsb + ws.lam);
+    sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
+    sp.wait_ns = P.wait_ns;
+    sp.stall_unit = P.stall_unit;
+    if (launch_score(sp, P.d, grid, smem, s) != cudaSuccess) return KVEV_ECUDA;
+  }
+
+  // ---- selection --------------------------------------------------------
+  SelectParams sel;
+  std::memset(&sel, 0, sizeof(sel));
+  GatherParams ga;
+  std::memset(&ga, 0, sizeof(ga));
+  int64_t off = 0;
+  for (int l = 0; l < P.L; ++l) {
+    LayerDesc ld;
+    ld.method = P.route_pre[l];
+    ld.slots = P.slots[l];
+    ld.recent = P.recent_eff[l];
+    ld.h2o_recent = P.h2o_r[l];
+    ld.score_slot = P.score_slot[l];
+    ld.row_off = off;
+    off += rows_per_layer(P, B, l);
+    sel.layer[l] = ld;
+    ga.layer[l] = ld;
+    ga.K[l] = K[l];
+    ga.V[l] = V[l];
+  }
+  sel.L = P.L;
+  sel.B = B;
+  sel.H_kv = P.H_kv;
+  sel.S_cap = S_cap;
+  sel.W = P.W;
+  sel.pool_kernel = P.pool_kernel;
+  sel.pool_type = P.pool_type;
+  sel.sink = P.sink;
+  sel.lens = lens_ok;
+  sel.raw = reinterpret_cast<const float*>(wsb + ws.raw);
+  sel.out_idx = out_idx;
+  sel.out_count = out_count;
+  const size_t sel_smem = ws.n_units > 0 ? sizeof(uint32_t) * static_cast<size_t>(S_cap) : 0;
+  if (sel_smem + 4096 > static_cast<size_t>(P.smem_optin)) return KVEV_ENOTSUP;
+  if (sel_smem > 48 * 1024 && P.select_smem_set < sel_smem) {
+    if (select_set_smem(sel_smem) != cudaSuccess) return KVEV_ECUDA;
+    P.select_smem_set = sel_smem;
+  }
+  if (launch_select(sel, P.L * B * P.H_kv, sel_smem, s) != cudaSuccess) return KVEV_ECUDA;
+
+  // ---- gather-compaction ---------------------------------------------------
+  ga.L = P.L;
+  ga.B = B;
+  ga.H_kv = P.H_kv;
+  ga.S_cap = S_cap;
+  ga.d = P.d;
+  ga.total_rows = total_rows;
+  ga.out_idx = out_idx;
+  ga.raw = sel.raw;
+  ga.out_K = out_K;
+  ga.out_V = out_V;
+  ga.h2o_state = h2o_state;
+  ga.status = P.d_status;
+  if (launch_gather(ga, s, P.num_sms) != cudaSuccess) return KVEV_ECUDA;
+  return KVEV_OK;
+}

@@ -1,0 +1,305 @@
+// kvev_internal.cuh -- device helpers and launch parameter blocks shared by the
+// kernels of libkvev.so (GB300 / sm_103a).  Inline PTX for mbarrier, TMA and
+// the 5th-generation tensor core (tcgen05 + tensor memory).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/kvev.h"
+
+namespace kvev {
+
+constexpr int kMaxLayers = 128;       // layers in one plan
+constexpr int kMaxScoreLayers = 64;   // SnapKV/H2O layers (tensor maps travel as kernel params)
+constexpr int kTileKeys = 128;        // keys per tensor-core tile (MMA M or N)
+constexpr int kMinChunkTiles = 8;     // tiles per scoring work item (chunk), at least
+constexpr int kScoreThreads = 320;    // 1 TMA warp, 1 MMA warp, 2 softmax warpgroups
+constexpr int kSelectThreads = 512;
+constexpr int kWsAlign = 256;
+
+// Bits of the device status word.
+constexpr int kStatusTimeout = 1;
+constexpr int kStatusDevice = 2;
+
+// Per-layer description used by the selection and gather kernels.
+struct LayerDesc {
+  int method;         // prefill operator (KVEV_*)
+  int slots;          // output slots per (seq, kv head): b_l, 0 for FULL
+  int recent;         // StreamingLLM recent tokens kept (<= b - sink)
+  int h2o_recent;     // H2O protected recent window
+  int score_slot;     // index among scoring layers, -1 if none
+  long long row_off;  // first packed output row of the layer
+};
+
+struct PrologueParams {
+  int n_units;        // scoring units = n_slayers * B * H_kv
+  int B, H_kv, S_cap;
+  int chunk_keys;
+  int slayer_method[kMaxScoreLayers];
+  int slayer_budget[kMaxScoreLayers];
+  const int* lens_in; // caller's lengths
+  int* lens;          // validated copy (out-of-range lengths become 0, flagged)
+  int* status;
+  int* cnt;
+  int* ready;
+  int* abort_flag;
+  int* chunk_start;   // [n_units + 1]
+  int* item_unit;     // [items]
+};
+
+struct ScoreParams {
+  CUtensorMap kmap[kMaxScoreLayers];  // K of each scoring layer, 2-D {d, B*H_kv*S_cap}
+  CUtensorMap qmap[kMaxScoreLayers];  // Q_win of each scoring layer, 2-D {d, B*H_q*W}
+  int n_units, B, H_kv, H_q, G, W, R, R_pad, S_cap;
+  int chunk_keys;     // keys per work item (multiple of 128)
+  int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
+  int stages;         // K tile ring depth
+  int tmem_buf_cols;  // TMEM columns per accumulator buffer (128 or 256)
+  float scale_log2;   // log2(e) / sqrt(d)
+  float inv_G;
+  const int* lens;
+  const int* chunk_start;
+  const int* item_unit;
+  int* cnt;
+  int* ready;
+  int* abort_flag;
+  int* status;
+  float2* part;       // [items][2][R_pad] per-row (max, sum) partials, base-2 units
+  float* lam;         // [n_units][R_pad] per-row log2-sum-exp
+  float* raw;         // [n_units][S_cap] window scores
+  long long wait_ns;
+  int stall_unit;
+};
+
+struct SelectParams {
+  LayerDesc layer[kMaxLayers];
+  int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink;
+  const int* lens;
+  const float* raw;   // [n_units][S_cap]
+  int* out_idx;
+  int* out_count;     // [L][B][H_kv]
+};
+
+struct GatherParams {
+  LayerDesc layer[kMaxLayers];
+  const void* K[kMaxLayers];
+  const void* V[kMaxLayers];
+  int L, B, H_kv, S_cap, d;
+  long long total_rows;
+  const int* out_idx;
+  const float* raw;
+  void* out_K;
+  void* out_V;
+  float* h2o_state;
+  int* status;
+};
+
+// ---------------------------------------------------------------------------
+// Small PTX wrappers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// 2-D tiled TMA load into shared memory, completion counted on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// ---- tcgen05 -----------------------------------------------------------------
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D(tmem) (+)= A(smem) * B(smem)^T, bf16 inputs, fp32 accumulate, one CTA.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on `bar` once every tcgen05 operation issued so far by this thread completes.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  tmem_wait_ld();
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  tmem_wait_ld();
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor of a K-major bf16 operand stored with the
+// 128-byte swizzle: rows of 128 B (64 elements), 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // start address
+  d |= static_cast<uint64_t>(16u >> 4) << 16;           // leading-dim byte offset (unused)
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;         // stride between 8-row groups
+  d |= static_cast<uint64_t>(1) << 46;                  // descriptor version
+  d |= static_cast<uint64_t>(2) << 61;                  // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: kind::f16 with bf16 A/B, fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_volatile(const int* p) {
+  return *reinterpret_cast<const volatile int*>(p);
+}
+
+// Order-preserving map of an fp32 to uint32 (larger float -> larger key).
+__device__ __forceinline__ uint32_t float_key(float f) {
+  uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+}  // namespace kvev
+
+// Launchers implemented by the kernel translation units.
+namespace kvev {
+cudaError_t launch_prologue(const PrologueParams& p, cudaStream_t s);
+cudaError_t launch_score(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
+int score_smem_bytes(int d, int q_rows, int R_pad, int stages);
+cudaError_t score_set_smem(int d, size_t smem);
+cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s);
+cudaError_t select_set_smem(size_t smem);
+cudaError_t launch_gather(const GatherParams& p, cudaStream_t s, int num_sms);
+}  // namespace kvev

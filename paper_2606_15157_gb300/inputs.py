@@ -348,3 +348,90 @@ def decode_token(wl: Workload, step: int, layer: int, s: int, h: int):
     qidx = (qrow[:, None] * d + np.arange(d)[None, :]).astype(np.uint64)
     q = gauss_bf16(stream_key(wl.seed, T_QNEW, layer), qidx.ravel()).reshape(wl.G, d)
     return k, v, q
+
+
+# --------------------------------------------------------------------------
+# Device tensor generation (full-size workloads), bit-identical to the above
+# --------------------------------------------------------------------------
+
+_synth = None
+
+
+def synth_lib():
+    """ctypes handle of libkvev_synth.so (raises if it was not built)."""
+    global _synth
+    if _synth is None:
+        import ctypes as C
+        import os
+        path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libkvev_synth.so")
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build()")
+        lib = C.CDLL(path)
+        vp, i, u64, f = C.c_void_p, C.c_int, C.c_uint64, C.c_float
+        lib.kvev_synth_k.argtypes = [vp, i, i, i, i, u64, i, f, i, i, f, vp, vp]
+        lib.kvev_synth_q.argtypes = [vp, i, i, i, i, i, u64, f, vp, vp]
+        lib.kvev_synth_gauss.argtypes = [vp, u64, u64, u64, vp]
+        lib.kvev_synth_bits.argtypes = [vp, u64, u64, u64, vp]
+        for fn in ("kvev_synth_k", "kvev_synth_q", "kvev_synth_gauss", "kvev_synth_bits"):
+            getattr(lib, fn).restype = C.c_int
+        _synth = lib
+    return _synth
+
+
+def _stream_ptr(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def device_layer(wl: Workload, layer: int, stream=None, need_q: bool = True):
+    """(K, V, Q) CUDA tensors of one layer, bf16; Q is None when need_q is False."""
+    import torch
+    lib = synth_lib()
+    sp = _stream_ptr(stream)
+    K = torch.empty((wl.B, wl.H_kv, wl.S_cap, wl.d), dtype=torch.bfloat16, device="cuda")
+    V = torch.empty_like(K)
+    u_dev, lo, hi, gamma = None, 0, 0, 0.0
+    if wl.plant is not None:
+        u = np.stack([_unit_u(wl, layer, h) for h in range(wl.H_kv)]).astype(np.float32)
+        u_dev = torch.from_numpy(u).cuda()
+        lo = int(wl.plant["start"][layer])
+        hi = lo + int(wl.plant["size"][layer])
+        gamma = float(wl.plant["gamma"][layer])
+    rc = lib.kvev_synth_k(K.data_ptr(), wl.B, wl.H_kv, wl.S_cap, wl.d,
+                          stream_key(wl.seed, T_K, layer), wl.sink_tokens, float(wl.sink_scale),
+                          lo, hi, gamma, None if u_dev is None else u_dev.data_ptr(), sp)
+    assert rc == 0, rc
+    rc = lib.kvev_synth_bits(V.data_ptr(), V.numel(), stream_key(wl.seed, T_V, layer), 0, sp)
+    assert rc == 0, rc
+    Q = None
+    if need_q:
+        Q = torch.empty((wl.B, wl.H_q, wl.W, wl.d), dtype=torch.bfloat16, device="cuda")
+        rc = lib.kvev_synth_q(Q.data_ptr(), wl.B, wl.H_q, wl.W, wl.d, wl.G,
+                              stream_key(wl.seed, T_Q, layer),
+                              float(wl.plant["alpha"]) if wl.plant is not None else 0.0,
+                              None if u_dev is None else u_dev.data_ptr(), sp)
+        assert rc == 0, rc
+    if u_dev is not None:
+        torch.cuda.current_stream().synchronize()
+    return K, V, Q
+
+
+def device_decode_tokens(wl: Workload, step: int, layer: int, stream=None):
+    """New-token k, v [B][H_kv][d] and q [B][H_q][d] of one decode step (CUDA, bf16)."""
+    import torch
+    lib = synth_lib()
+    sp = _stream_ptr(stream)
+    d = wl.d
+    k = torch.empty((wl.B, wl.H_kv, d), dtype=torch.bfloat16, device="cuda")
+    v = torch.empty_like(k)
+    q = torch.empty((wl.B, wl.H_q, d), dtype=torch.bfloat16, device="cuda")
+    base_kv = step * wl.B * wl.H_kv * d
+    base_q = step * wl.B * wl.H_q * d
+    assert lib.kvev_synth_gauss(k.data_ptr(), k.numel(), stream_key(wl.seed, T_KNEW, layer),
+                                base_kv, sp) == 0
+    assert lib.kvev_synth_bits(v.data_ptr(), v.numel(), stream_key(wl.seed, T_VNEW, layer),
+                               base_kv, sp) == 0
+    assert lib.kvev_synth_gauss(q.data_ptr(), q.numel(), stream_key(wl.seed, T_QNEW, layer),
+                                base_q, sp) == 0
+    return k, v, q

@@ -1,0 +1,249 @@
+"""ctypes binding of ``libkvev.so`` (C ABI in ``include/kvev.h``).
+
+Argument marshalling only: every step of the eviction runs in the library's
+kernels.  Functions keep the C names; :class:`Plan` is a small convenience
+wrapper that owns a plan handle and sizes the buffers.  If the library has not
+been built, loading raises -- there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "lib", "libkvev.so")
+
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE, ENOTSUP = range(7)
+FULL, SNAPKV, H2O, STREAMING, TOVA = 0, 1, 2, 3, 4
+POOL_MAX, POOL_AVG = 0, 1
+T_IDENTITY, T_CAP_Q95 = 0, 1
+
+STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA",
+                ETIMEOUT: "ETIMEOUT", EDEVICE: "EDEVICE", ENOTSUP: "ENOTSUP"}
+
+EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
+           "kvev_plan_destroy", "kvev_plan_query", "kvev_plan_layer_offset",
+           "kvev_evict_prefill", "kvev_status", "kvev_plan_set_wait_limit",
+           "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset"]
+
+
+class KvevError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{what}: {STATUS_NAMES.get(code, code)}")
+        self.code = code
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load the library (once).  Raises if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build()")
+        L = C.CDLL(path)
+        vp, i32, i64, sz = C.c_void_p, C.c_int32, C.c_int64, C.c_size_t
+        P = C.POINTER
+        L.kvev_alloc_from_scores.argtypes = [vp, vp, C.c_int, i64, C.c_int, C.c_int]
+        L.kvev_alloc_rescale.argtypes = [vp, vp, C.c_int, i64]
+        L.kvev_plan_create.argtypes = [P(vp), C.c_int, C.c_int, C.c_int, C.c_int, vp, vp, vp,
+                                       C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]
+        L.kvev_plan_destroy.argtypes = [vp]
+        L.kvev_plan_destroy.restype = None
+        L.kvev_plan_query.argtypes = [vp, C.c_int, C.c_int, P(sz), P(sz), P(sz), P(sz)]
+        L.kvev_plan_layer_offset.argtypes = [vp, C.c_int, C.c_int, P(i64)]
+        L.kvev_evict_prefill.argtypes = [vp, vp, vp, vp, vp, C.c_int, C.c_int, vp, vp, vp, vp, vp,
+                                         vp, sz, vp]
+        L.kvev_status.argtypes = [vp, P(C.c_int)]
+        L.kvev_plan_set_wait_limit.argtypes = [vp, i64]
+        L.kvev_plan_debug_stall_unit.argtypes = [vp, C.c_int]
+        L.kvev_plan_scores_offset.argtypes = [vp, C.c_int, C.c_int, C.c_int, P(sz)]
+        for name in EXPORTS:
+            if name != "kvev_plan_destroy":
+                getattr(L, name).restype = C.c_int
+        _lib = L
+    return _lib
+
+
+def _check(rc: int, what: str):
+    if rc != OK:
+        raise KvevError(rc, what)
+
+
+# ---------------------------------------------------------------------------
+# C-named wrappers
+# ---------------------------------------------------------------------------
+
+def kvev_alloc_from_scores(s, B_total: int, b_min: int, transform: int = T_IDENTITY) -> np.ndarray:
+    s = np.ascontiguousarray(s, dtype=np.float64)
+    out = np.zeros(len(s), np.int32)
+    _check(load().kvev_alloc_from_scores(out.ctypes.data, s.ctypes.data, len(s), int(B_total),
+                                         int(b_min), int(transform)), "kvev_alloc_from_scores")
+    return out
+
+
+def kvev_alloc_rescale(b_in, B_target: int) -> np.ndarray:
+    b_in = np.ascontiguousarray(b_in, dtype=np.int32)
+    out = np.zeros(len(b_in), np.int32)
+    _check(load().kvev_alloc_rescale(out.ctypes.data, b_in.ctypes.data, len(b_in), int(B_target)),
+           "kvev_alloc_rescale")
+    return out
+
+
+alloc_from_scores = kvev_alloc_from_scores
+alloc_rescale = kvev_alloc_rescale
+
+
+def kvev_plan_create(L, H_q, H_kv, d, route_prefill, route_decode, budget, window, pool_kernel,
+                     pool_type, sink, recent=-1, h2o_recent=-1) -> int:
+    rp = np.ascontiguousarray(route_prefill, np.int32)
+    rd = None if route_decode is None else np.ascontiguousarray(route_decode, np.int32)
+    b = np.ascontiguousarray(budget, np.int32)
+    h = C.c_void_p()
+    rc = load().kvev_plan_create(C.byref(h), L, H_q, H_kv, d, rp.ctypes.data,
+                                 None if rd is None else rd.ctypes.data, b.ctypes.data, window,
+                                 pool_kernel, pool_type, sink, recent, h2o_recent)
+    _check(rc, "kvev_plan_create")
+    return h.value
+
+
+def kvev_plan_destroy(handle: int):
+    load().kvev_plan_destroy(handle)
+
+
+def kvev_plan_query(handle: int, B: int, S_cap: int):
+    vals = [C.c_size_t() for _ in range(4)]
+    _check(load().kvev_plan_query(handle, B, S_cap, *[C.byref(v) for v in vals]),
+           "kvev_plan_query")
+    return tuple(v.value for v in vals)
+
+
+def kvev_plan_layer_offset(handle: int, B: int, layer: int) -> int:
+    v = C.c_int64()
+    _check(load().kvev_plan_layer_offset(handle, B, layer, C.byref(v)), "kvev_plan_layer_offset")
+    return v.value
+
+
+def kvev_evict_prefill(handle, K_ptrs, V_ptrs, Q_ptrs, lens_ptr, B, S_cap, out_K, out_V, out_idx,
+                       out_count, h2o_state, workspace, workspace_bytes, stream) -> int:
+    """Pointer-level call; returns the status code (does not raise)."""
+    Ln = len(K_ptrs)
+    arr = C.c_void_p * Ln
+    Ka, Va = arr(*K_ptrs), arr(*V_ptrs)
+    Qa = arr(*Q_ptrs) if Q_ptrs is not None else None
+    return load().kvev_evict_prefill(handle, Ka, Va, Qa, lens_ptr, B, S_cap, out_K, out_V,
+                                     out_idx, out_count, h2o_state, workspace, workspace_bytes,
+                                     stream)
+
+
+def kvev_status(handle: int) -> int:
+    v = C.c_int()
+    _check(load().kvev_status(handle, C.byref(v)), "kvev_status")
+    return v.value
+
+
+def kvev_plan_scores_offset(handle: int, B: int, S_cap: int, layer: int) -> int:
+    v = C.c_size_t()
+    _check(load().kvev_plan_scores_offset(handle, B, S_cap, layer, C.byref(v)),
+           "kvev_plan_scores_offset")
+    return v.value
+
+
+def kvev_plan_set_wait_limit(handle: int, ns: int):
+    _check(load().kvev_plan_set_wait_limit(handle, int(ns)), "kvev_plan_set_wait_limit")
+
+
+def kvev_plan_debug_stall_unit(handle: int, unit: int):
+    _check(load().kvev_plan_debug_stall_unit(handle, int(unit)), "kvev_plan_debug_stall_unit")
+
+
+def alloc_pyramid(L: int, B_total: int, b_min: int) -> np.ndarray:
+    """Pyramidal schedule: weights decreasing linearly with depth (1.5 -> 0.5) fed to Eq. 3."""
+    w = np.ones(1) if L == 1 else 1.5 - np.arange(L) / (L - 1)
+    return kvev_alloc_from_scores(w, B_total, b_min, T_IDENTITY)
+
+
+# ---------------------------------------------------------------------------
+# Convenience: a plan plus its buffers, with torch tensors as device memory
+# ---------------------------------------------------------------------------
+
+class Plan:
+    """Owns a kvev plan; allocates outputs/workspace as torch CUDA tensors."""
+
+    def __init__(self, L, H_q, H_kv, d, route, budget, window, pool_kernel=7, pool_type=POOL_AVG,
+                 sink=4, recent=-1, h2o_recent=-1, route_decode=None):
+        self.L, self.H_q, self.H_kv, self.d = L, H_q, H_kv, d
+        self.route = np.asarray(route, np.int32)
+        self.budget = np.asarray(budget, np.int32)
+        self.window = window
+        self.handle = kvev_plan_create(L, H_q, H_kv, d, self.route, route_decode, self.budget,
+                                       window, pool_kernel, pool_type, sink, recent, h2o_recent)
+
+    @classmethod
+    def from_workload(cls, wl):
+        return cls(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel,
+                   wl.pool_type, wl.sink, wl.recent, wl.h2o_recent, wl.route_decode)
+
+    def close(self):
+        if self.handle:
+            kvev_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def query(self, B, S_cap):
+        return kvev_plan_query(self.handle, B, S_cap)
+
+    def layer_offset(self, B, layer):
+        return kvev_plan_layer_offset(self.handle, B, layer)
+
+    def buffers(self, B, S_cap, device="cuda"):
+        import torch
+        kv_bytes, idx_bytes, cnt_bytes, ws_bytes = self.query(B, S_cap)
+        rows = idx_bytes // 4
+        return {
+            "out_K": torch.empty((max(rows, 1), self.d), dtype=torch.bfloat16, device=device),
+            "out_V": torch.empty((max(rows, 1), self.d), dtype=torch.bfloat16, device=device),
+            "out_idx": torch.empty(max(rows, 1), dtype=torch.int32, device=device),
+            "out_count": torch.empty((self.L, B, self.H_kv), dtype=torch.int32, device=device),
+            "h2o_state": torch.empty(max(rows, 1), dtype=torch.float32, device=device),
+            "workspace": torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=device),
+            "rows": rows,
+        }
+
+    def evict_prefill(self, K, V, Q, lens, B, S_cap, bufs, stream=None, check=True) -> int:
+        """K, V, Q: lists (per layer) of CUDA tensors or None; lens: int32 CUDA tensor."""
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        ptr = lambda t: None if t is None else t.data_ptr()
+        rc = kvev_evict_prefill(
+            self.handle, [ptr(k) for k in K], [ptr(v) for v in V],
+            [ptr(q) for q in Q] if Q is not None else None, lens.data_ptr(), B, S_cap,
+            bufs["out_K"].data_ptr(), bufs["out_V"].data_ptr(), bufs["out_idx"].data_ptr(),
+            bufs["out_count"].data_ptr(), bufs["h2o_state"].data_ptr(),
+            bufs["workspace"].data_ptr(), bufs["workspace"].numel(), stream.cuda_stream)
+        if check:
+            _check(rc, "kvev_evict_prefill")
+        return rc
+
+    def status(self) -> int:
+        return kvev_status(self.handle)
+
+    def scores(self, bufs, B, S_cap, layer):
+        """fp32 window scores [B][H_kv][S_cap] of a SnapKV/H2O layer (a view of the workspace)."""
+        import torch
+        off = kvev_plan_scores_offset(self.handle, B, S_cap, layer)
+        n = B * self.H_kv * S_cap
+        return bufs["workspace"][off: off + 4 * n].view(torch.float32).view(B, self.H_kv, S_cap)

@@ -1,0 +1,172 @@
+"""Host-side checks of the C ABI (no GPU needed, no kernel launched).
+
+* the shared libraries load and export every symbol include/*.h declares;
+* the library's allocator equals the oracle's bit for bit;
+* plan validation, byte accounting (App. E worked example) and layer offsets;
+* argument errors are reported before any device work.
+"""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2606_15157_gb300 import inputs as gen
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def kv():
+    from paper_2606_15157_gb300 import build, kvev
+    build.build()
+    kvev.load()
+    return kvev
+
+
+def declared(header, macro):
+    txt = open(os.path.join(ROOT, "include", header)).read()
+    return re.findall(macro + r"\s+[\w\s\*]*?\b(kvev_\w+)\s*\(", txt)
+
+
+def test_libraries_export_every_declared_symbol(kv):
+    names = declared("kvev.h", "KVEV_API")
+    assert len(names) >= 10
+    lib = C.CDLL(kv.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(kv.EXPORTS)
+    synth = declared("kvev_synth.h", "KVEV_SYNTH_API")
+    slib = C.CDLL(os.path.join(os.path.dirname(kv.LIB_PATH), "libkvev_synth.so"))
+    assert len(synth) == 4
+    for n in synth:
+        assert hasattr(slib, n), n
+
+
+def test_operator_ids_match_header(kv):
+    txt = open(os.path.join(ROOT, "include", "kvev.h")).read()
+    ids = dict(re.findall(r"#define KVEV_(FULL|SNAPKV|H2O|STREAMING|TOVA)\s+(\d+)", txt))
+    assert {k: int(v) for k, v in ids.items()} == {
+        "FULL": kv.FULL, "SNAPKV": kv.SNAPKV, "H2O": kv.H2O, "STREAMING": kv.STREAMING, "TOVA": kv.TOVA}
+    assert (gen.FULL, gen.SNAPKV, gen.H2O, gen.STREAMING) == (kv.FULL, kv.SNAPKV, kv.H2O, kv.STREAMING)
+
+
+def test_allocator_matches_oracle_bit_exact(kv, orc):
+    rng = np.random.default_rng(11)
+    for trial in range(500):
+        L = int(rng.integers(1, 80))
+        b_min = int(rng.integers(0, 100))
+        B = L * b_min + int(rng.integers(0, 100000))
+        kind = trial % 4
+        if kind == 0:
+            s = rng.gamma(0.3, size=L)
+        elif kind == 1:
+            s = rng.standard_normal(L)            # non-positive values: shift rule
+        elif kind == 2:
+            s = np.round(rng.random(L) * 4) / 4    # many exact ties
+        else:
+            s = np.exp(rng.standard_normal(L) * 3)  # outliers for the Q95 cap
+        for T in (kv.T_IDENTITY, kv.T_CAP_Q95):
+            a = kv.alloc_from_scores(s, B, b_min, T)
+            b = orc.alloc_from_scores(s, B, b_min, T)
+            assert a.tolist() == b.tolist(), (trial, T)
+    for trial in range(200):
+        b_in = rng.integers(1, 4000, size=int(rng.integers(1, 64))).astype(np.int32)
+        T = int(rng.integers(0, 200000))
+        assert kv.alloc_rescale(b_in, T).tolist() == orc.alloc_rescale(b_in, T).tolist()
+
+
+def test_workload_budgets(kv, orc):
+    # Pyramidal (decreasing with depth) and Dirichlet allocations of the
+    # synthetic workloads: exact totals, b_min respected, same on both sides.
+    al = lambda f: (lambda s, B, m, t: f(s, B, m, t))
+    for bbar in (128, 256, 512, 1024, 2048):
+        wk = gen.config_hetero8k(kv.alloc_from_scores, bbar=bbar)
+        wo = gen.config_hetero8k(orc.alloc_from_scores, bbar=bbar)
+        assert wk.budget.tolist() == wo.budget.tolist()
+        assert wk.budget.sum() == 32 * bbar and wk.budget.min() >= 48
+        assert np.all(np.diff(wk.budget) <= 0)
+        assert (wk.route == gen.SNAPKV).sum() == 18 and (wk.route == gen.H2O).sum() == 7
+    wk = gen.config_long(kv.alloc_from_scores)
+    wo = gen.config_long(orc.alloc_from_scores)
+    assert wk.budget.tolist() == wo.budget.tolist()
+    assert wk.budget.sum() == 32 * 1024 and wk.budget.min() >= 80
+    assert np.all((wk.lens >= 16384) & (wk.lens <= 32768))
+
+
+def test_plan_validation(kv):
+    ok = dict(L=2, H_q=8, H_kv=2, d=128, route_prefill=[kv.SNAPKV, kv.STREAMING],
+              route_decode=None, budget=[64, 64], window=32, pool_kernel=7, pool_type=kv.POOL_AVG,
+              sink=4, recent=-1, h2o_recent=-1)
+    h = kv.kvev_plan_create(**ok)
+    kv.kvev_plan_destroy(h)
+
+    def bad(code, **kw):
+        args = dict(ok)
+        args.update(kw)
+        with pytest.raises(kv.KvevError) as e:
+            kv.kvev_plan_create(**args)
+        assert e.value.code == code
+
+    bad(kv.EINVAL, budget=[32, 64])                       # SnapKV b <= W
+    bad(kv.EINVAL, budget=[64, 4])                        # StreamingLLM b <= sink
+    bad(kv.EINVAL, pool_kernel=4)                         # even pooling width
+    bad(kv.EINVAL, H_q=7)                                 # H_q not a multiple of H_kv
+    bad(kv.EINVAL, route_prefill=[kv.H2O, 9])             # unknown operator
+    bad(kv.EINVAL, route_prefill=[kv.H2O, kv.STREAMING], h2o_recent=100)  # r > b
+    bad(kv.EINVAL, route_decode=[kv.SNAPKV, kv.FULL])     # SnapKV is not a decode operator
+    bad(kv.ENOTSUP, d=96)                                 # scoring needs d in {64, 128}
+    bad(kv.ENOTSUP, window=128, budget=[200, 64])         # G*W = 512 > 256
+    # FULL layers ignore their budget; StreamingLLM needs no window
+    h = kv.kvev_plan_create(**dict(ok, route_prefill=[kv.FULL, kv.STREAMING], budget=[0, 64],
+                                   window=0))
+    kv.kvev_plan_destroy(h)
+
+
+def test_app_e_byte_accounting(kv):
+    # App. E: 32 layers x 512 retained tokens, 8 KV heads, d=128, bf16 K and V
+    # -> 16,384 layer-token positions, 64.00 MiB of exact KV state.
+    h = kv.kvev_plan_create(32, 32, 8, 128, [kv.H2O] * 32, None, [512] * 32, 32, 7, kv.POOL_AVG, 4)
+    kv_bytes, idx_bytes, cnt_bytes, ws = kv.kvev_plan_query(h, 1, 32768)
+    assert idx_bytes // 4 == 16384 * 8
+    assert 2 * kv_bytes == 64 * 2 ** 20
+    assert cnt_bytes == 32 * 8 * 4
+    assert kv.kvev_plan_layer_offset(h, 1, 0) == 0
+    assert kv.kvev_plan_layer_offset(h, 1, 5) == 5 * 512 * 8
+    assert kv.kvev_plan_layer_offset(h, 3, 5) == 5 * 512 * 8 * 3
+    kv.kvev_plan_destroy(h)
+
+
+def test_layer_offsets_skip_full_layers(kv):
+    routes = [kv.FULL, kv.SNAPKV, kv.FULL, kv.STREAMING, kv.H2O, kv.FULL]
+    budget = [999, 100, 999, 50, 70, 999]
+    h = kv.kvev_plan_create(6, 4, 2, 64, routes, None, budget, 16, 5, kv.POOL_MAX, 4)
+    B, H = 3, 2
+    exp = [0, 0, 100 * B * H, 100 * B * H, 150 * B * H, 220 * B * H]
+    assert [kv.kvev_plan_layer_offset(h, B, l) for l in range(6)] == exp
+    kv_bytes, idx_bytes, _, _ = kv.kvev_plan_query(h, B, 4096)
+    assert idx_bytes // 4 == 220 * B * H and kv_bytes == 220 * B * H * 64 * 2
+    with pytest.raises(kv.KvevError):
+        kv.kvev_plan_scores_offset(h, B, 4096, 3)   # StreamingLLM layer has no scores
+    o1 = kv.kvev_plan_scores_offset(h, B, 4096, 1)
+    o4 = kv.kvev_plan_scores_offset(h, B, 4096, 4)
+    assert o4 - o1 == 4 * B * H * 4096
+    kv.kvev_plan_destroy(h)
+
+
+def test_evict_argument_errors_before_device_work(kv):
+    h = kv.kvev_plan_create(2, 4, 2, 64, [kv.SNAPKV, kv.STREAMING], None, [64, 64], 8, 5,
+                            kv.POOL_MAX, 4)
+    fake = 1 << 20
+    args = dict(handle=h, K_ptrs=[fake, fake], V_ptrs=[fake, fake], Q_ptrs=[fake, fake],
+                lens_ptr=fake, B=1, S_cap=512, out_K=fake, out_V=fake, out_idx=fake,
+                out_count=fake, h2o_state=None, workspace=fake, workspace_bytes=1 << 30, stream=None)
+    assert kv.kvev_evict_prefill(**dict(args, B=-1)) == kv.EINVAL
+    assert kv.kvev_evict_prefill(**dict(args, S_cap=0)) == kv.EINVAL
+    assert kv.kvev_evict_prefill(**dict(args, K_ptrs=[fake + 8, fake])) == kv.EINVAL   # misaligned
+    assert kv.kvev_evict_prefill(**dict(args, Q_ptrs=[None, fake])) == kv.EINVAL      # SnapKV needs Q
+    assert kv.kvev_evict_prefill(**dict(args, workspace=fake + 16)) == kv.EINVAL      # 256-B alignment
+    assert kv.kvev_evict_prefill(**dict(args, workspace_bytes=64)) == kv.ENOMEM
+    assert kv.kvev_evict_prefill(**dict(args, B=0)) == kv.OK                          # nothing to do
+    kv.kvev_plan_destroy(h)

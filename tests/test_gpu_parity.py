@@ -1,0 +1,250 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle.
+
+Every test runs the library's kernels (libkvev.so) on seeded synthetic inputs
+and compares scores, kept positions, gathered K/V bytes and H2O state with the
+oracle under the match criteria of ``tests/parity.py``.
+"""
+import numpy as np
+import pytest
+
+from paper_2606_15157_gb300 import inputs as gen
+
+from . import parity
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch as t
+    if not t.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_15157_gb300 import kvev
+    kvev.load()
+    return t
+
+
+def host_to_dev(torch, arrays):
+    out = {}
+    for l, (K, V, Q) in arrays.items():
+        f = lambda a: None if a is None else torch.from_numpy(a.view(np.int16)).cuda().view(torch.bfloat16)
+        out[l] = (f(K), f(V), f(Q))
+    return out
+
+
+def device_workload(wl, layers=None):
+    layers = range(wl.L) if layers is None else layers
+    return {l: gen.device_layer(wl, l, need_q=wl.route[l] in (gen.SNAPKV, gen.H2O)) for l in layers}
+
+
+def oracle_alloc(s, B_total, b_min, transform):
+    import oracle
+    return oracle.alloc_from_scores(s, B_total, b_min, transform)
+
+
+def kvev_alloc(s, B_total, b_min, transform):
+    from paper_2606_15157_gb300 import kvev
+    return kvev.alloc_from_scores(s, B_total, b_min, transform)
+
+
+# ---------------------------------------------------------------------------
+
+def test_synth_device_matches_host(torch):
+    # The device generator reproduces the host generator bit for bit.
+    wl = gen.config_tiny(seed=3)
+    host = gen.host_tensors(wl, [0, 2])
+    for l in (0, 2):
+        K, V, Q = gen.device_layer(wl, l)
+        assert np.array_equal(parity.to_host_u16(K), host[l][0])
+        assert np.array_equal(parity.to_host_u16(V), host[l][1])
+        assert np.array_equal(parity.to_host_u16(Q), host[l][2])
+    wl2 = gen.config_homog8k(seed=1)
+    for l in (0, 13, 31):
+        K, V, Q = gen.device_layer(wl2, l)
+        pos = np.array([0, 5, wl2.plant["start"][l], wl2.plant["start"][l] + 1, 8191])
+        for h in (0, 7):
+            assert np.array_equal(parity.to_host_u16(K[0, h])[pos], gen.k_rows(wl2, l, 0, h, pos))
+            assert np.array_equal(parity.to_host_u16(Q[0, h * 4:(h + 1) * 4]), gen.q_group(wl2, l, 0, h))
+    k, v, q = gen.device_decode_tokens(wl2, 5, 3)
+    kh, vh, qh = gen.decode_token(wl2, 5, 3, 0, 6)
+    assert np.array_equal(parity.to_host_u16(k[0, 6]), kh)
+    assert np.array_equal(parity.to_host_u16(v[0, 6]), vh)
+    assert np.array_equal(parity.to_host_u16(q[0, 24:28]), qh)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_tiny_config(torch, orc, seed):
+    wl = gen.config_tiny(seed)
+    dev = host_to_dev(torch, gen.host_tensors(wl))
+    stats = {}
+    parity.check_workload(wl, dev, wl.lens, stats=stats)
+    assert stats["max_rel_err"] < 2e-3
+
+
+def test_homogeneous_snapkv_8k(torch, orc):
+    wl = gen.config_homog8k(seed=0)
+    dev = device_workload(wl)
+    stats = {}
+    parity.check_workload(wl, dev, wl.lens, stats=stats)
+    print("homog8k", stats)
+
+
+@pytest.mark.parametrize("bbar", [128, 256, 512, 1024, 2048])
+def test_heterogeneous_route_8k(torch, orc, bbar):
+    wl = gen.config_hetero8k(kvev_alloc, seed=0, bbar=bbar)
+    wl_o = gen.config_hetero8k(oracle_alloc, seed=0, bbar=bbar)
+    assert np.array_equal(wl.budget, wl_o.budget)
+    assert wl.budget.sum() == 32 * bbar
+    dev = device_workload(wl)
+    stats = {}
+    parity.check_workload(wl_o, dev, wl.lens, stats=stats)
+    print("hetero8k", bbar, stats)
+
+
+def _sample_units(wl, k, seed):
+    rng = np.random.default_rng(seed)
+    units = []
+    for op in (gen.SNAPKV, gen.H2O, gen.STREAMING):
+        layers = np.nonzero(wl.route == op)[0]
+        for _ in range(k):
+            units.append((int(rng.choice(layers)), int(rng.integers(wl.B)), int(rng.integers(wl.H_kv))))
+    return sorted(set(units))
+
+
+def test_long_context_batch_sampled(torch, orc):
+    # Full-size headline workload (batch 8, ragged 16K-32K, W=64) in the launch
+    # configuration the benchmark times; the oracle checks sampled units and
+    # every unit is checked against properties that hold at any size.
+    wl = gen.config_long(kvev_alloc, seed=0)
+    wl_o = gen.config_long(oracle_alloc, seed=0)
+    assert np.array_equal(wl.budget, wl_o.budget)
+    dev = device_workload(wl)
+    stats = {}
+    plan, bufs, gpu = parity.check_workload(wl_o, dev, wl.lens, units=_sample_units(wl, 4, 0),
+                                            stats=stats)
+    print("long sampled", stats)
+    # properties over every unit
+    for l in range(wl.L):
+        b = int(wl.budget[l])
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            assert np.all(gpu.count[l, s] == min(b, n))
+            base0 = plan.layer_offset(wl.B, l)
+            blk = gpu.idx[base0 + s * wl.H_kv * b: base0 + (s + 1) * wl.H_kv * b].reshape(wl.H_kv, b)
+            assert np.all(np.diff(blk, axis=1) > 0)
+            prot = {gen.SNAPKV: wl.W, gen.H2O: b // 2, gen.STREAMING: b - wl.sink}[int(wl.route[l])]
+            assert np.all(blk[:, b - prot:] == np.arange(n - prot, n)[None, :])
+            if wl.route[l] in (gen.SNAPKV, gen.H2O):
+                tot = gpu.scores[l][s, :, :n].astype(np.float64).sum(axis=1)
+                assert np.allclose(tot, wl.W, rtol=1e-3)  # each window row's softmax sums to 1
+    # gathered rows of every unit equal the source rows (device-side check)
+    outK = bufs["out_K"]
+    for l in range(wl.L):
+        b = int(wl.budget[l])
+        base0 = plan.layer_offset(wl.B, l)
+        idx = bufs["out_idx"][base0: base0 + wl.B * wl.H_kv * b].view(wl.B, wl.H_kv, b).long()
+        src = dev[l][0].view(torch.int16)
+        ref = torch.gather(src, 2, idx.unsqueeze(-1).expand(-1, -1, -1, wl.d))
+        got = outK[base0: base0 + wl.B * wl.H_kv * b].view(torch.int16).view(wl.B, wl.H_kv, b, wl.d)
+        assert torch.equal(ref, got)
+
+
+def _custom(L_routes, budgets, lens, W=16, d=128, H_q=8, H_kv=2, S_cap=None, pool=(5, gen.POOL_MAX),
+            seed=7, sink=4, h2o_recent=-1):
+    lens = np.asarray(lens, np.int32)
+    S_cap = S_cap or int(max(lens.max(), 1))
+    return gen.Workload(name="edge", L=len(L_routes), H_q=H_q, H_kv=H_kv, d=d, B=len(lens), lens=lens,
+                        S_cap=S_cap, W=W, pool_kernel=pool[0], pool_type=pool[1],
+                        route=np.asarray(L_routes, np.int32), budget=np.asarray(budgets, np.int32),
+                        sink=sink, seed=seed, sink_tokens=4, h2o_recent=h2o_recent)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_edge_lengths(torch, orc, d):
+    # Ragged batch with empty, shorter-than-window, exactly-budget, budget+1,
+    # non-multiple-of-tile and full-capacity lengths; FULL layers interleaved.
+    b = 40
+    lens = [0, 1, 15, 16, 40, 41, 127, 129, 1000, 1031]
+    routes = [gen.SNAPKV, gen.H2O, gen.STREAMING, gen.FULL, gen.H2O, gen.SNAPKV]
+    wl = _custom(routes, [b, b, b, 0, 7, 130], lens, d=d, S_cap=1031)
+    dev = device_workload(wl)
+    parity.check_workload(wl, dev, wl.lens)
+
+
+def test_edge_window_and_groups(torch, orc):
+    # Different GQA group sizes and windows: R = G*W = 16, 48 (a 16-column tail), 128, 192, 256.
+    for (H_q, H_kv, W) in [(4, 2, 8), (12, 4, 16), (8, 2, 32), (12, 2, 32), (32, 8, 64)]:
+        wl = _custom([gen.SNAPKV, gen.H2O], [W + 37, 100], [700, 3000, 2 * W], W=W, H_q=H_q, H_kv=H_kv,
+                     pool=(7, gen.POOL_AVG))
+        dev = device_workload(wl)
+        parity.check_workload(wl, dev, wl.lens)
+
+
+def test_h2o_recent_override_and_ties(torch, orc):
+    # h2o_recent = 0 (pure heavy hitters) and = b (pure recency); plus all-zero
+    # queries so every score in a row ties and the lower-position rule decides.
+    wl = _custom([gen.H2O, gen.H2O, gen.SNAPKV], [64, 64, 64], [900, 2000], h2o_recent=0)
+    dev = device_workload(wl)
+    for l in dev:
+        if dev[l][2] is not None:
+            dev[l][2].zero_() if l == 2 else None
+    parity.check_workload(wl, dev, wl.lens)
+    wl2 = _custom([gen.H2O], [50], [600], h2o_recent=50)
+    parity.check_workload(wl2, device_workload(wl2), wl2.lens)
+
+
+def test_repeat_calls_identical(torch):
+    wl = gen.config_tiny(1)
+    dev = host_to_dev(torch, gen.host_tensors(wl))
+    plan, bufs = parity.run_gpu(wl, dev, wl.lens)
+    first = {k: v.clone() for k, v in bufs.items() if hasattr(v, "clone")}
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    for _ in range(3):
+        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    for k in ("out_K", "out_V", "out_idx", "out_count"):
+        assert torch.equal(first[k], bufs[k])
+
+
+def test_wait_timeout_reports_status(torch):
+    # A unit whose normaliser is never published: every wait on it runs out
+    # after the (short) limit, the kernel finishes, the status word says
+    # ETIMEOUT, and the context stays usable for the next call.
+    from paper_2606_15157_gb300 import kvev
+    wl = gen.config_tiny(0)
+    dev = host_to_dev(torch, gen.host_tensors(wl))
+    plan = kvev.Plan.from_workload(wl)
+    kvev.kvev_plan_set_wait_limit(plan.handle, 20_000_000)  # 20 ms
+    kvev.kvev_plan_debug_stall_unit(plan.handle, 0)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    assert plan.status() == kvev.ETIMEOUT
+    kvev.kvev_plan_debug_stall_unit(plan.handle, -1)
+    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    assert plan.status() == kvev.OK
+
+
+def test_invalid_lengths_flagged(torch):
+    from paper_2606_15157_gb300 import kvev
+    wl = _custom([gen.SNAPKV, gen.STREAMING], [40, 40], [100, 200], S_cap=200)
+    dev = device_workload(wl)
+    plan = kvev.Plan.from_workload(wl)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.tensor([100, 5000], dtype=torch.int32, device="cuda")  # 5000 > S_cap
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    assert plan.status() == kvev.EDEVICE
+    cnt = bufs["out_count"].cpu().numpy()
+    assert np.all(cnt[:, 1] == 0)  # the invalid sequence is treated as empty
