@@ -1,0 +1,463 @@
+#!/usr/bin/env python
+"""Benchmark of the prefill eviction hot path on GB300.
+
+One step = one kvev_evict_prefill() over the whole synthetic workload: window
+scores of every SnapKV/H2O layer, selection, gather-compaction of every
+layer of the heterogeneous route.  The default workload is the batch-8,
+ragged 16K-32K-token, window-64 route of 32 LLaMA-3.1-8B-shaped layers
+(18 SnapKV / 7 H2O / 7 StreamingLLM, Dirichlet capacity allocation summing to
+1024 tokens per layer on average), whose inputs (about 34 GB of K/V) are far
+larger than L2.
+
+Usage:  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun each rank runs its own batch (different seed): weak scaling,
+no collective on the data path; rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2606_15157_gb300 import inputs as gen  # noqa: E402
+
+METRIC = "KV-eviction GB/s and % of HBM peak (Llama-3.1-8B shape, 32K ctx)"
+NOMINAL_HBM_GBS = 8000.0
+
+
+# ---------------------------------------------------------------------------
+# Workload accounting (algorithmic bytes, evicted tokens)
+# ---------------------------------------------------------------------------
+
+def unit_bytes(wl, l: int, n: int) -> tuple[int, int]:
+    """(algorithmic bytes, score-kernel bytes) of one (sequence, layer, KV head).
+
+    Scoring layer: all K read (n rows) + the group's window queries + kept K
+    and V written; the score kernel's share is K read + window queries + the
+    fp32 scores it writes.  StreamingLLM: kept K and V read and written.
+    """
+    row = wl.d * 2
+    m = int(wl.route[l])
+    b = int(wl.budget[l])
+    if m in (gen.SNAPKV, gen.H2O):
+        if m == gen.SNAPKV and n <= b:      # identity, no scoring
+            return 4 * n * row, 0
+        q = wl.G * wl.W * row
+        return n * row + q + 2 * min(n, b) * row, n * row + q + 4 * n
+    if m == gen.STREAMING:
+        cap = wl.sink + (wl.recent if wl.recent >= 0 else b - wl.sink)
+        return 4 * min(n, cap) * row, 0
+    return 0, 0
+
+
+def workload_bytes(wl):
+    tot = sc = ev = 0
+    for l in range(wl.L):
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            a, c = unit_bytes(wl, l, n)
+            tot += a * wl.H_kv
+            sc += c * wl.H_kv
+            if wl.route[l] != gen.FULL:
+                ev += (n - min(n, int(wl.budget[l]))) * wl.H_kv
+    return tot, sc, ev
+
+
+def make_workload(name: str, seed: int, alloc, batch: int | None = None):
+    if name == "long":
+        wl = gen.config_long(alloc, seed=seed)
+        if batch:  # first `batch` sequences of the same draw (small profiling case)
+            wl.B, wl.lens = batch, wl.lens[:batch].copy()
+            wl.name += f"_first{batch}"
+        return wl
+    if name == "long32k":
+        return gen.config_long(alloc, seed=seed, fixed_len=32768)
+    if name == "homog8k":
+        return gen.config_homog8k(seed=seed)
+    if name == "hetero8k":
+        return gen.config_hetero8k(alloc, seed=seed, bbar=512)
+    raise ValueError(name)
+
+
+def workload_config(wl, extra=None):
+    cfg = {
+        "workload": wl.name,
+        "layers": wl.L, "heads_q": wl.H_q, "heads_kv": wl.H_kv, "head_dim": wl.d,
+        "batch": wl.B, "seq_lens": [int(x) for x in wl.lens], "window": wl.W,
+        "pool": f"{'avg' if wl.pool_type == gen.POOL_AVG else 'max'}{wl.pool_kernel}",
+        "route": {"snapkv": int((wl.route == gen.SNAPKV).sum()), "h2o": int((wl.route == gen.H2O).sum()),
+                  "streaming": int((wl.route == gen.STREAMING).sum())},
+        "budget_mean": float(np.mean(wl.budget)), "budget_total": int(np.sum(wl.budget)),
+        "l2": "inputs larger than L2 (no flush needed)",
+    }
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        mhz, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                mhz.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.path)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a bounded sample (CPU baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+def sample_units(wl, count: int, seed: int = 0):
+    """A sample of (layer, seq, head) units with the route's operator mix."""
+    rng = np.random.default_rng(seed)
+    active = [l for l in range(wl.L) if wl.route[l] != gen.FULL]
+    out = []
+    for i in range(count):
+        l = active[i % len(active)] if i < len(active) else int(rng.choice(active))
+        out.append((l, int(rng.integers(wl.B)), int(rng.integers(wl.H_kv))))
+    return out
+
+
+def oracle_sample(wl, units, nthreads=0):
+    """Time the oracle on `units` (inputs generated on the host); returns (seconds, bytes)."""
+    import oracle
+    oracle.build()
+    specs, nbytes = [], 0
+    for (l, s, h) in units:
+        n = int(wl.lens[s])
+        pos = np.arange(n, dtype=np.int64)
+        K = gen.k_rows(wl, l, s, h, pos)
+        Q = gen.q_group(wl, l, s, h) if wl.route[l] in (gen.SNAPKV, gen.H2O) else None
+        specs.append(dict(method=int(wl.route[l]), n=n, b=int(wl.budget[l]), W=wl.W,
+                          pool_kernel=wl.pool_kernel, pool_type=wl.pool_type, sink=wl.sink,
+                          recent=wl.recent, h2o_recent=wl.h2o_recent, K=K, Q=Q))
+        nbytes += unit_bytes(wl, l, n)[0]
+    t0 = time.perf_counter()
+    oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=nthreads)
+    return time.perf_counter() - t0, nbytes
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ---------------------------------------------------------------------------
+# The two arms
+# ---------------------------------------------------------------------------
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    import oracle
+    wl = make_workload(args.workload, 0, oracle.alloc_from_scores, args.batch)
+    cores = cpu_cores()
+    units = sample_units(wl, args.ref_units)
+    for _ in range(args.warmup):
+        oracle_sample(wl, units[: max(1, len(units) // 4)], cores)
+    tot_s, tot_b = 0.0, 0
+    for k in range(args.steps):
+        s, b = oracle_sample(wl, sample_units(wl, args.ref_units, seed=k), cores)
+        tot_s += s
+        tot_b += b
+    value = tot_b / tot_s / 1e9
+    sample = f"{args.ref_units} (sequence, layer, KV-head) units of the workload per step, route mix kept"
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; shapes of LLaMA-3.1-8B long-context workloads)",
+        "config": workload_config(wl, {"sample": sample}),
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": min(cores, args.ref_units),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("score.cu", "kvev_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2606_15157_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    from paper_2606_15157_gb300 import kvev
+
+    torch.cuda.set_device(local_rank)
+    dist = world > 1
+    if dist:
+        import torch.distributed as td
+
+    wl = make_workload(args.workload, rank, kvev.alloc_from_scores, args.batch)
+    tot_bytes, score_bytes, evicted = workload_bytes(wl)
+    need_q = lambda l: wl.route[l] in (gen.SNAPKV, gen.H2O)
+    dev = {l: gen.device_layer(wl, l, need_q=need_q(l)) for l in range(wl.L)}
+    plan = kvev.Plan.from_workload(wl)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if dist:
+            td.barrier()
+        torch.cuda.synchronize()
+
+    def reduce(x: float, op) -> float:
+        if not dist:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        td.all_reduce(t, op=op)
+        return float(t.item())
+
+    max_over_ranks = lambda x: reduce(x, td.ReduceOp.MAX) if dist else x
+    sum_over_ranks = lambda x: reduce(x, td.ReduceOp.SUM) if dist else x
+
+    # ---- device-resident timed region ----
+    kvev.kvev_plan_enable_timing(plan.handle, True)
+    for _ in range(args.warmup):
+        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
+    barrier()
+    per_kernel = {k: [] for k in kvev.KERNEL_NAMES}
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local_rank) as clk:
+        barrier()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
+            for k, v in kvev.kvev_plan_last_timings(plan.handle).items():
+                if v >= 0:
+                    per_kernel[k].append(v)
+        ev1.record(stream)
+        barrier()
+    ms_total = ev0.elapsed_time(ev1)
+    ms_step = max_over_ranks(ms_total / args.steps)
+    status = plan.status()
+    assert status == kvev.OK, f"device status {status}"
+    clocks = clk.summary()
+    kernels_launched = sum(len(v) for v in per_kernel.values())
+    all_bytes = sum_over_ranks(float(tot_bytes))
+    all_evicted = sum_over_ranks(float(evicted))
+    value = all_bytes / (ms_step / 1e3) / 1e9
+
+    # ---- roofline of the dominant kernel (window scores) ----
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+    score_ms = statistics.mean(per_kernel["score"]) if per_kernel["score"] else float("nan")
+    achieved = score_bytes / (score_ms / 1e3) / 1e9
+    kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
+    traffic = None
+    tf = os.path.join(ROOT, "profiles", "score_traffic.json")
+    if os.path.exists(tf):
+        try:
+            t = json.load(open(tf))
+            if t.get("workload") == wl.name and t.get("kernel_src_hash") == kernel_hash():
+                traffic = t["bytes_per_launch"]
+        except (OSError, ValueError, KeyError):
+            pass
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, wl, plan, dev, lens, stream, tot_bytes, barrier, max_over_ranks,
+                      sum_over_ranks)
+
+    # ---- CPU baseline (rank 0, one GPU only) ----
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = cpu_cores()
+        units, secs, nb, i = [], 0.0, 0, 0
+        while secs < args.cpu_seconds and i < 4096:
+            batch = sample_units(wl, 8, seed=100 + i)
+            s, b = oracle_sample(wl, batch, cores)
+            units += batch
+            secs += s
+            nb += b
+            i += 1
+        cpu = {"value": nb / secs / 1e9, "unit": "GB/s", "cores": min(cores, 8), "kind": "oracle",
+               "sample": f"{len(units)} (sequence, layer, KV-head) units of the workload, "
+                         f"route mix kept, {secs:.1f} s of oracle time"}
+
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; shapes of LLaMA-3.1-8B long-context workloads)",
+            "config": workload_config(wl, {"parallelism": f"independent batch per GPU x{world}"}),
+            "hbm_frac": {"of_measured": value / hbm_peak, "of_nominal_8TBs": value / NOMINAL_HBM_GBS},
+            "evicted_tokens_per_s": all_evicted / (ms_step / 1e3),
+            "kernel_ms": kernel_ms,
+            "roofline": {"kernel": "score_kernel", "bound": "hbm", "achieved": achieved,
+                         "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                         "traffic": traffic, "peak_source": peak_src},
+            "clocks": clocks,
+            "gpu_launches": kernels_launched,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(out), flush=True)
+
+
+def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_ranks,
+            sum_over_ranks):
+    """Same metric through the public API with pinned host inputs copied in and
+    the kept indices / counts read back every step."""
+    import torch
+    from paper_2606_15157_gb300 import kvev
+    host = {}
+    for l, (Kd, Vd, Qd) in dev.items():
+        host[l] = tuple(None if t is None else torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                        for t in (Kd, Vd, Qd))
+        for hsrc, dsrc in zip(host[l], (Kd, Vd, Qd)):
+            if hsrc is not None:
+                hsrc.copy_(dsrc)
+    lens_h = torch.from_numpy(np.asarray(wl.lens, np.int32)).pin_memory()
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    idx_h = torch.empty(bufs["out_idx"].shape, dtype=torch.int32, pin_memory=True)
+    cnt_h = torch.empty(bufs["out_count"].shape, dtype=torch.int32, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for ts in host.values() for t in ts if t is not None)
+    h2d += lens_h.numel() * 4
+    d2h = idx_h.numel() * 4 + cnt_h.numel() * 4
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+
+    def step():
+        for l in range(wl.L):
+            for hsrc, dsrc in zip(host[l], dev[l]):
+                if hsrc is not None:
+                    dsrc.copy_(hsrc, non_blocking=True)
+        lens_dev.copy_(lens_h, non_blocking=True)
+        plan.evict_prefill(K, V, Q, lens_dev, wl.B, wl.S_cap, bufs, stream)
+        idx_h.copy_(bufs["out_idx"], non_blocking=True)
+        cnt_h.copy_(bufs["out_count"], non_blocking=True)
+
+    kvev.kvev_plan_enable_timing(plan.handle, False)
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n = args.e2e_steps
+    e0.record(stream)
+    for _ in range(n):
+        step()
+    e1.record(stream)
+    barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1) / n)
+    return {"value": sum_over_ranks(float(tot_bytes)) / (ms / 1e3) / 1e9, "unit": "GB/s",
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": ms,
+            "steps": n}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="long", choices=["long", "long32k", "homog8k", "hetero8k"])
+    ap.add_argument("--batch", type=int, default=None,
+                    help="use only the first B sequences of the 'long' workload (profiling)")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-units", type=int, default=16)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as td
+        torch.cuda.set_device(local_rank)
+        td.init_process_group("nccl")
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_ours(args, rank, world, local_rank)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as td
+        td.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -193,6 +193,26 @@ KVEV_API int kvev_plan_set_wait_limit(kvev_plan *plan, int64_t ns);
  * exercise the timeout path; -1 disables it. */
 KVEV_API int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
 
+/* ---- measurement ---------------------------------------------------------- */
+
+/* Kernels of one kvev_evict_prefill() call, in launch order. */
+#define KVEV_K_PROLOGUE 0
+#define KVEV_K_SCORE 1
+#define KVEV_K_SELECT 2
+#define KVEV_K_GATHER 3
+#define KVEV_NUM_KERNELS 4
+
+/* When `on` is non-zero, every later kvev_evict_prefill() records a CUDA
+ * event pair on the caller's stream around each of its kernel launches
+ * (creates the events on first use; ECUDA if that fails). */
+KVEV_API int kvev_plan_enable_timing(kvev_plan *plan, int on);
+
+/* Device time in milliseconds of each kernel of the most recent timed call
+ * (synchronises on its last event); ms[k] = -1 for a kernel that call did not
+ * launch.  n = number of entries of ms (up to KVEV_NUM_KERNELS are written).
+ * EINVAL if timing is off or no timed call was made. */
+KVEV_API int kvev_plan_last_timings(kvev_plan *plan, float *ms, int n);
+
 #ifdef __cplusplus
 }
 #endif

@@ -38,6 +38,11 @@ struct kvev_plan {
   cudaStream_t last_stream = nullptr;
   bool attrs_set = false;
   size_t score_smem_set = 0, select_smem_set = 0;
+  // optional per-kernel timing of the last call
+  bool timing = false;
+  bool timed_call = false;
+  cudaEvent_t ev[2 * KVEV_NUM_KERNELS] = {};
+  bool launched[KVEV_NUM_KERNELS] = {};
 };
 
 namespace {
@@ -303,7 +308,35 @@ extern "C" int kvev_plan_create(kvev_plan** out, int L, int H_q, int H_kv, int d
 extern "C" void kvev_plan_destroy(kvev_plan* plan) {
   if (!plan) return;
   if (plan->d_status) cudaFree(plan->d_status);
+  for (cudaEvent_t e : plan->ev)
+    if (e) cudaEventDestroy(e);
   delete plan;
+}
+
+extern "C" int kvev_plan_enable_timing(kvev_plan* plan, int on) {
+  if (!plan) return KVEV_EINVAL;
+  if (on && !plan->ev[0]) {
+    for (cudaEvent_t& e : plan->ev)
+      if (cudaEventCreate(&e) != cudaSuccess) return KVEV_ECUDA;
+  }
+  plan->timing = on != 0;
+  plan->timed_call = false;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_last_timings(kvev_plan* plan, float* ms, int n) {
+  if (!plan || !ms || n < 0 || !plan->timing || !plan->timed_call) return KVEV_EINVAL;
+  int last = -1;
+  for (int k = 0; k < KVEV_NUM_KERNELS; ++k)
+    if (plan->launched[k]) last = k;
+  if (last >= 0 && cudaEventSynchronize(plan->ev[2 * last + 1]) != cudaSuccess) return KVEV_ECUDA;
+  for (int k = 0; k < n && k < KVEV_NUM_KERNELS; ++k) {
+    ms[k] = -1.f;
+    if (plan->launched[k] &&
+        cudaEventElapsedTime(&ms[k], plan->ev[2 * k], plan->ev[2 * k + 1]) != cudaSuccess)
+      return KVEV_ECUDA;
+  }
+  return KVEV_OK;
 }
 
 extern "C" int kvev_plan_query(const kvev_plan* plan, int B, int S_cap, size_t* out_kv_bytes,
@@ -423,7 +456,17 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   pp.abort_flag = reinterpret_cast<int*>(wsb + ws.abort_flag);
   pp.chunk_start = reinterpret_cast<int*>(wsb + ws.chunk_start);
   pp.item_unit = reinterpret_cast<int*>(wsb + ws.item_unit);
+  for (bool& b : P.launched) b = false;
+  P.timed_call = P.timing;
+  auto mark = [&](int k, int which) {
+    if (P.timing) {
+      cudaEventRecord(P.ev[2 * k + which], s);
+      if (which == 1) P.launched[k] = true;
+    }
+  };
+  mark(KVEV_K_PROLOGUE, 0);
   if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+  mark(KVEV_K_PROLOGUE, 1);
 
   // ---- window scores ----------------------------------------------------
   if (ws.n_units > 0) {
@@ -477,7 +520,9 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
     sp.wait_ns = P.wait_ns;
     sp.stall_unit = P.stall_unit;
+    mark(KVEV_K_SCORE, 0);
     if (launch_score(sp, P.d, grid, smem, s) != cudaSuccess) return KVEV_ECUDA;
+    mark(KVEV_K_SCORE, 1);
   }
 
   // ---- selection --------------------------------------------------------
@@ -518,7 +563,9 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
     if (select_set_smem(sel_smem) != cudaSuccess) return KVEV_ECUDA;
     P.select_smem_set = sel_smem;
   }
+  mark(KVEV_K_SELECT, 0);
   if (launch_select(sel, P.L * B * P.H_kv, sel_smem, s) != cudaSuccess) return KVEV_ECUDA;
+  mark(KVEV_K_SELECT, 1);
 
   // ---- gather-compaction ---------------------------------------------------
   ga.L = P.L;
@@ -533,6 +580,8 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   ga.out_V = out_V;
   ga.h2o_state = h2o_state;
   ga.status = P.d_status;
+  mark(KVEV_K_GATHER, 0);
   if (launch_gather(ga, s, P.num_sms) != cudaSuccess) return KVEV_ECUDA;
+  if (total_rows > 0) mark(KVEV_K_GATHER, 1);
   return KVEV_OK;
 }

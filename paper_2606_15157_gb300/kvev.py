@@ -27,7 +27,9 @@ STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA",
 EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_destroy", "kvev_plan_query", "kvev_plan_layer_offset",
            "kvev_evict_prefill", "kvev_status", "kvev_plan_set_wait_limit",
-           "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset"]
+           "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
+           "kvev_plan_last_timings"]
+KERNEL_NAMES = ["prologue", "score", "select", "gather"]
 
 
 class KvevError(RuntimeError):
@@ -65,6 +67,8 @@ def load(path: str = LIB_PATH):
         L.kvev_plan_set_wait_limit.argtypes = [vp, i64]
         L.kvev_plan_debug_stall_unit.argtypes = [vp, C.c_int]
         L.kvev_plan_scores_offset.argtypes = [vp, C.c_int, C.c_int, C.c_int, P(sz)]
+        L.kvev_plan_enable_timing.argtypes = [vp, C.c_int]
+        L.kvev_plan_last_timings.argtypes = [vp, vp, C.c_int]
         for name in EXPORTS:
             if name != "kvev_plan_destroy":
                 getattr(L, name).restype = C.c_int
@@ -154,6 +158,17 @@ def kvev_plan_scores_offset(handle: int, B: int, S_cap: int, layer: int) -> int:
     _check(load().kvev_plan_scores_offset(handle, B, S_cap, layer, C.byref(v)),
            "kvev_plan_scores_offset")
     return v.value
+
+
+def kvev_plan_enable_timing(handle: int, on: bool = True):
+    _check(load().kvev_plan_enable_timing(handle, int(bool(on))), "kvev_plan_enable_timing")
+
+
+def kvev_plan_last_timings(handle: int) -> dict:
+    """Per-kernel device milliseconds of the last timed call ({name: ms}, -1 if not launched)."""
+    ms = np.zeros(len(KERNEL_NAMES), np.float32)
+    _check(load().kvev_plan_last_timings(handle, ms.ctypes.data, len(ms)), "kvev_plan_last_timings")
+    return {k: float(v) for k, v in zip(KERNEL_NAMES, ms)}
 
 
 def kvev_plan_set_wait_limit(handle: int, ns: int):
