@@ -193,6 +193,41 @@ KVEV_API int kvev_plan_set_wait_limit(kvev_plan *plan, int64_t ns);
  * exercise the timeout path; -1 disables it. */
 KVEV_API int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
 
+/* ---- prefill eviction for callers that cannot allocate device memory ------ */
+
+/* Size of the device scratch that kvev_evict_prefill_noalloc() uses instead of
+ * a caller workspace (32 MiB; every GPU that loads the library holds it until
+ * the process exits). */
+#define KVEV_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+/* Same eviction as kvev_evict_prefill(), for callers that must not allocate:
+ * code running where cudaMalloc is forbidden or unavailable (inside a memory
+ * pool whose budget is already committed, in a custom allocator's own hooks,
+ * under a framework that owns all device memory), or that has no workspace to
+ * lend.  No counterpart in the paper: it is a deployment convenience.
+ *   - The scratch is a fixed library-owned device array of
+ *     KVEV_NOALLOC_SCRATCH_BYTES; a request whose kvev_plan_query()
+ *     workspace_bytes exceeds it returns KVEV_ENOMEM before any device work.
+ *   - The call allocates nothing: no cudaMalloc/cudaFree and no allocating
+ *     library routine.  Inputs and outputs are the caller's, as for
+ *     kvev_evict_prefill().
+ *   - device_status: optional device int32 (NULL allowed) that the call zeroes
+ *     on `stream` and in which the kernels record their status bits
+ *     (1 = a bounded wait ran out, 2 = an in-kernel check failed).
+ *     kvev_status() does not see this entry point's calls.
+ *   - The first call on each device looks up the scratch array's device
+ *     address for that device (with that device current); make that first
+ *     call before any stream capture on the device.
+ *   - All calls in the process share the one array per device and each call
+ *     starts by resetting the parts that must start at zero; calls whose GPU
+ *     work overlaps (other streams, other host threads) race on it and must
+ *     be serialised by the caller. */
+KVEV_API int kvev_evict_prefill_noalloc(kvev_plan *plan, const void *const *K,
+                                        const void *const *V, const void *const *Q_win,
+                                        const int32_t *lens_dev, int B, int S_cap, void *out_K,
+                                        void *out_V, int32_t *out_idx, int32_t *out_count,
+                                        float *h2o_state, int32_t *device_status, void *stream);
+
 /* ---- measurement ---------------------------------------------------------- */
 
 /* Kernels of one kvev_evict_prefill() call, in launch order. */

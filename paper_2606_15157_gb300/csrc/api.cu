@@ -19,6 +19,16 @@
 
 using namespace kvev;
 
+// Per-device launch context: device properties, which kernel attributes were
+// set, and the device status word the kernels report to.
+struct DevCtx {
+  int device = -1;
+  int num_sms = 0;
+  int smem_optin = 0;
+  size_t score_smem_set = 0, select_smem_set = 0;
+  int* status = nullptr;
+};
+
 struct kvev_plan {
   int L = 0, H_q = 0, H_kv = 0, d = 0, G = 0;
   int W = 0, pool_kernel = 1, pool_type = 0, sink = 0, recent = -1, h2o_recent = -1;
@@ -30,14 +40,9 @@ struct kvev_plan {
   std::vector<int> score_layers;
   int64_t wait_ns = 2000000000LL;
   int stall_unit = -1;
-  // device-side state, created on first use
-  int device = -1;
-  int num_sms = 0;
-  int smem_optin = 0;
-  int* d_status = nullptr;
+  // device-side state, created on first use (status word allocated lazily)
+  DevCtx ctx;
   cudaStream_t last_stream = nullptr;
-  bool attrs_set = false;
-  size_t score_smem_set = 0, select_smem_set = 0;
   // optional per-kernel timing of the last call
   bool timing = false;
   bool timed_call = false;
@@ -117,25 +122,35 @@ bool encode_map(CUtensorMap* m, const void* base, int d, uint64_t rows, int box_
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-int ensure_device(kvev_plan* p) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return KVEV_ECUDA;
-  if (p->device == dev && p->d_status) return KVEV_OK;
-  if (p->d_status) {
-    cudaFree(p->d_status);
-    p->d_status = nullptr;
-  }
+// Device properties of the current device into `c` (no allocation).
+int query_device(DevCtx& c, int dev) {
   int major = 0;
-  if (cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&p->smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+  if (cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c.smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
           cudaSuccess ||
       cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
     return KVEV_ECUDA;
   if (major < 10) return KVEV_ENOTSUP;
-  if (cudaMalloc(&p->d_status, sizeof(int)) != cudaSuccess) return KVEV_ENOMEM;
-  if (cudaMemset(p->d_status, 0, sizeof(int)) != cudaSuccess) return KVEV_ECUDA;
-  p->device = dev;
-  p->score_smem_set = p->select_smem_set = 0;
+  c.device = dev;
+  c.score_smem_set = c.select_smem_set = 0;
+  return KVEV_OK;
+}
+
+int ensure_device(kvev_plan* p) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return KVEV_ECUDA;
+  DevCtx& c = p->ctx;
+  if (c.device == dev && c.status) return KVEV_OK;
+  if (c.status) {
+    cudaFree(c.status);
+    c.status = nullptr;
+  }
+  int rc = query_device(c, dev);
+  if (rc != KVEV_OK) return rc;
+  c.device = -1;
+  if (cudaMalloc(&c.status, sizeof(int)) != cudaSuccess) return KVEV_ENOMEM;
+  if (cudaMemset(c.status, 0, sizeof(int)) != cudaSuccess) return KVEV_ECUDA;
+  c.device = dev;
   return KVEV_OK;
 }
 
@@ -307,7 +322,7 @@ extern "C" int kvev_plan_create(kvev_plan** out, int L, int H_q, int H_kv, int d
 
 extern "C" void kvev_plan_destroy(kvev_plan* plan) {
   if (!plan) return;
-  if (plan->d_status) cudaFree(plan->d_status);
+  if (plan->ctx.status) cudaFree(plan->ctx.status);
   for (cudaEvent_t e : plan->ev)
     if (e) cudaEventDestroy(e);
   delete plan;
@@ -387,11 +402,11 @@ extern "C" int kvev_plan_debug_stall_unit(kvev_plan* plan, int unit) {
 extern "C" int kvev_status(kvev_plan* plan, int* device_status) {
   if (!plan || !device_status) return KVEV_EINVAL;
   *device_status = KVEV_OK;
-  if (!plan->d_status) return KVEV_OK;
+  if (!plan->ctx.status) return KVEV_OK;
   if (cudaStreamSynchronize(plan->last_stream) != cudaSuccess) return KVEV_ECUDA;
   int v = 0;
-  if (cudaMemcpy(&v, plan->d_status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess ||
-      cudaMemset(plan->d_status, 0, sizeof(int)) != cudaSuccess)
+  if (cudaMemcpy(&v, plan->ctx.status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemset(plan->ctx.status, 0, sizeof(int)) != cudaSuccess)
     return KVEV_ECUDA;
   *device_status = (v & kStatusTimeout) ? KVEV_ETIMEOUT : (v & kStatusDevice) ? KVEV_EDEVICE : 0;
   return KVEV_OK;
@@ -401,6 +416,37 @@ extern "C" int kvev_status(kvev_plan* plan, int* device_status) {
 // Prefill eviction
 // ---------------------------------------------------------------------------
 
+namespace {
+
+// Argument checks shared by the prefill entry points (no device work).
+int check_prefill_args(const kvev_plan& P, const void* const* K, const void* const* V,
+                       const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap,
+                       void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count) {
+  if (!K || !V || !lens_dev || !out_count) return KVEV_EINVAL;
+  if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
+  int64_t total_rows = 0;
+  for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
+  if (total_rows > 0 && (!out_K || !out_V || !out_idx)) return KVEV_EINVAL;
+  if (!aligned16(out_K) || !aligned16(out_V)) return KVEV_EINVAL;
+  for (int l = 0; l < P.L; ++l) {
+    if (P.route_pre[l] == KVEV_FULL) continue;
+    if (!K[l] || !V[l] || !aligned16(K[l]) || !aligned16(V[l])) return KVEV_EINVAL;
+    if (is_scoring(P.route_pre[l]) && (!Q_win || !Q_win[l] || !aligned16(Q_win[l])))
+      return KVEV_EINVAL;
+  }
+  return KVEV_OK;
+}
+
+// The launch sequence of one prefill eviction, given a validated argument set,
+// a device context (properties + status word) and a scratch workspace of at
+// least ws_layout(P, B, S_cap).total bytes (256-byte aligned).
+int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
+               const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
+               void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
+               void* workspace, cudaStream_t s);
+
+}  // namespace
+
 extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const void* const* V,
                                   const void* const* Q_win, const int32_t* lens_dev, int B,
                                   int S_cap, void* out_K, void* out_V, int32_t* out_idx,
@@ -409,25 +455,28 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
   kvev_plan& P = *plan;
   if (B == 0) return KVEV_OK;
-  if (!K || !V || !lens_dev || !out_count || !workspace) return KVEV_EINVAL;
-  if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
-  int64_t total_rows = 0;
-  for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
-  if (total_rows > 0 && (!out_K || !out_V || !out_idx)) return KVEV_EINVAL;
-  if (!aligned16(out_K) || !aligned16(out_V) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
-    return KVEV_EINVAL;
-  for (int l = 0; l < P.L; ++l) {
-    if (P.route_pre[l] == KVEV_FULL) continue;
-    if (!K[l] || !V[l] || !aligned16(K[l]) || !aligned16(V[l])) return KVEV_EINVAL;
-    if (is_scoring(P.route_pre[l]) && (!Q_win || !Q_win[l] || !aligned16(Q_win[l])))
-      return KVEV_EINVAL;
-  }
-  const WsLayout ws = ws_layout(P, B, S_cap);
-  if (workspace_bytes < ws.total) return KVEV_ENOMEM;
-  int rc = ensure_device(plan);
+  int rc = check_prefill_args(P, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count);
+  if (rc != KVEV_OK) return rc;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return KVEV_EINVAL;
+  if (workspace_bytes < ws_layout(P, B, S_cap).total) return KVEV_ENOMEM;
+  rc = ensure_device(plan);
   if (rc != KVEV_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   P.last_stream = s;
+  return evict_impl(P, P.ctx, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count,
+                    h2o_state, workspace, s);
+}
+
+namespace {
+
+int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
+               const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
+               void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
+               void* workspace, cudaStream_t s) {
+  if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
+  int64_t total_rows = 0;
+  for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
+  const WsLayout ws = ws_layout(P, B, S_cap);
   uint8_t* wsb = static_cast<uint8_t*>(workspace);
   int* lens_ok = reinterpret_cast<int*>(wsb + ws.lens);
 
@@ -435,7 +484,7 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   const int n_slayers = static_cast<int>(P.score_layers.size());
   // chunk size: at least kMinChunkTiles tiles, and few enough chunks per unit
   // that a unit never spans more than two rounds of the persistent grid
-  const int grid = P.num_sms;
+  const int grid = D.num_sms;
   const int tiles_max = (S_cap + kTileKeys - 1) / kTileKeys;
   const int chunk_tiles = std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid);
   PrologueParams pp = {};
@@ -450,7 +499,7 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   pp.lens_in = lens_dev;
   pp.lens = lens_ok;
   pp.S_cap = S_cap;
-  pp.status = P.d_status;
+  pp.status = D.status;
   pp.cnt = reinterpret_cast<int*>(wsb + ws.cnt);
   pp.ready = reinterpret_cast<int*>(wsb + ws.ready);
   pp.abort_flag = reinterpret_cast<int*>(wsb + ws.abort_flag);
@@ -482,16 +531,16 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
         return KVEV_ECUDA;
     }
     int stages = 6;
-    while (stages >= 2 && score_smem_bytes(P.d, q_rows, ws.R_pad, stages) + 1024 > P.smem_optin)
+    while (stages >= 2 && score_smem_bytes(P.d, q_rows, ws.R_pad, stages) + 1024 > D.smem_optin)
       --stages;
     if (stages < 2) return KVEV_ENOTSUP;
     // Request more than half of the SM's shared memory so exactly one CTA is
     // resident per SM: its TMEM allocation then never waits on another CTA.
     const size_t smem = std::max<size_t>(score_smem_bytes(P.d, q_rows, ws.R_pad, stages),
-                                         static_cast<size_t>(P.smem_optin) / 2 + 1024);
-    if (P.score_smem_set != smem) {
+                                         static_cast<size_t>(D.smem_optin) / 2 + 1024);
+    if (D.score_smem_set != smem) {
       if (score_set_smem(P.d, smem) != cudaSuccess) return KVEV_ECUDA;
-      P.score_smem_set = smem;
+      D.score_smem_set = smem;
     }
     sp.n_units = ws.n_units;
     sp.B = B;
@@ -514,7 +563,7 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
     sp.cnt = pp.cnt;
     sp.ready = pp.ready;
     sp.abort_flag = pp.abort_flag;
-    sp.status = P.d_status;
+    sp.status = D.status;
     sp.part = reinterpret_cast<float2*>(wsb + ws.part);
     sp.lam = reinterpret_cast<float*>(wsb + ws.lam);
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
@@ -558,10 +607,10 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   sel.out_idx = out_idx;
   sel.out_count = out_count;
   const size_t sel_smem = ws.n_units > 0 ? sizeof(uint32_t) * static_cast<size_t>(S_cap) : 0;
-  if (sel_smem + 4096 > static_cast<size_t>(P.smem_optin)) return KVEV_ENOTSUP;
-  if (sel_smem > 48 * 1024 && P.select_smem_set < sel_smem) {
+  if (sel_smem + 4096 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
+  if (sel_smem > 48 * 1024 && D.select_smem_set < sel_smem) {
     if (select_set_smem(sel_smem) != cudaSuccess) return KVEV_ECUDA;
-    P.select_smem_set = sel_smem;
+    D.select_smem_set = sel_smem;
   }
   mark(KVEV_K_SELECT, 0);
   if (launch_select(sel, P.L * B * P.H_kv, sel_smem, s) != cudaSuccess) return KVEV_ECUDA;
@@ -579,9 +628,71 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
   ga.out_K = out_K;
   ga.out_V = out_V;
   ga.h2o_state = h2o_state;
-  ga.status = P.d_status;
+  ga.status = D.status;
   mark(KVEV_K_GATHER, 0);
-  if (launch_gather(ga, s, P.num_sms) != cudaSuccess) return KVEV_ECUDA;
+  if (launch_gather(ga, s, D.num_sms) != cudaSuccess) return KVEV_ECUDA;
   if (total_rows > 0) mark(KVEV_K_GATHER, 1);
   return KVEV_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Prefill eviction without allocation: the workspace is a file-scope device
+// array instead of caller memory.  Its name is only a host-side stand-in, so
+// host code obtains the array's device address per device with
+// cudaGetSymbolAddress (with that device current) and passes that pointer on.
+// ---------------------------------------------------------------------------
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[KVEV_NOALLOC_SCRATCH_BYTES];
+static __device__ int g_noalloc_status;  // status word used when the caller passes none
+
+constexpr int kMaxDevices = 64;
+
+struct NoallocDevice {
+  bool ready = false;
+  DevCtx ctx;
+  void* scratch = nullptr;  // device address of g_noalloc_scratch on this device
+  int* status = nullptr;    // device address of g_noalloc_status on this device
+};
+
+std::mutex g_noalloc_mu;
+NoallocDevice g_noalloc[kMaxDevices];
+
+}  // namespace
+
+extern "C" int kvev_evict_prefill_noalloc(kvev_plan* plan, const void* const* K,
+                                          const void* const* V, const void* const* Q_win,
+                                          const int32_t* lens_dev, int B, int S_cap, void* out_K,
+                                          void* out_V, int32_t* out_idx, int32_t* out_count,
+                                          float* h2o_state, int32_t* device_status, void* stream) {
+  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
+  kvev_plan& P = *plan;
+  if (B == 0) return KVEV_OK;
+  int rc = check_prefill_args(P, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count);
+  if (rc != KVEV_OK) return rc;
+  if (ws_layout(P, B, S_cap).total > KVEV_NOALLOC_SCRATCH_BYTES) return KVEV_ENOMEM;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return KVEV_ECUDA;
+  if (dev < 0 || dev >= kMaxDevices) return KVEV_ENOTSUP;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  NoallocDevice& nd = g_noalloc[dev];
+  if (!nd.ready) {  // once per device, with that device current
+    rc = query_device(nd.ctx, dev);
+    if (rc != KVEV_OK) return rc;
+    if (cudaGetSymbolAddress(&nd.scratch, g_noalloc_scratch) != cudaSuccess ||
+        cudaGetSymbolAddress(reinterpret_cast<void**>(&nd.status), g_noalloc_status) !=
+            cudaSuccess)
+      return KVEV_ECUDA;
+    nd.ready = true;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  nd.ctx.status = nd.status;
+  if (device_status) {
+    if (cudaMemsetAsync(device_status, 0, sizeof(int32_t), s) != cudaSuccess) return KVEV_ECUDA;
+    nd.ctx.status = reinterpret_cast<int*>(device_status);
+  }
+  return evict_impl(P, nd.ctx, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count,
+                    h2o_state, nd.scratch, s);
 }

@@ -28,7 +28,7 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_destroy", "kvev_plan_query", "kvev_plan_layer_offset",
            "kvev_evict_prefill", "kvev_status", "kvev_plan_set_wait_limit",
            "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
-           "kvev_plan_last_timings"]
+           "kvev_plan_last_timings", "kvev_evict_prefill_noalloc"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
 
 
@@ -68,6 +68,8 @@ def load(path: str = LIB_PATH):
         L.kvev_plan_debug_stall_unit.argtypes = [vp, C.c_int]
         L.kvev_plan_scores_offset.argtypes = [vp, C.c_int, C.c_int, C.c_int, P(sz)]
         L.kvev_plan_enable_timing.argtypes = [vp, C.c_int]
+        L.kvev_evict_prefill_noalloc.argtypes = [vp, vp, vp, vp, vp, C.c_int, C.c_int, vp, vp,
+                                                 vp, vp, vp, vp, vp]
         L.kvev_plan_last_timings.argtypes = [vp, vp, C.c_int]
         for name in EXPORTS:
             if name != "kvev_plan_destroy":
@@ -145,6 +147,20 @@ def kvev_evict_prefill(handle, K_ptrs, V_ptrs, Q_ptrs, lens_ptr, B, S_cap, out_K
     return load().kvev_evict_prefill(handle, Ka, Va, Qa, lens_ptr, B, S_cap, out_K, out_V,
                                      out_idx, out_count, h2o_state, workspace, workspace_bytes,
                                      stream)
+
+
+NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def kvev_evict_prefill_noalloc(handle, K_ptrs, V_ptrs, Q_ptrs, lens_ptr, B, S_cap, out_K, out_V,
+                               out_idx, out_count, h2o_state, device_status, stream) -> int:
+    """Pointer-level call of the entry point that allocates nothing (its scratch is
+    a fixed library-owned device array); returns the status code."""
+    arr = C.c_void_p * len(K_ptrs)
+    Ka, Va = arr(*K_ptrs), arr(*V_ptrs)
+    Qa = arr(*Q_ptrs) if Q_ptrs is not None else None
+    return load().kvev_evict_prefill_noalloc(handle, Ka, Va, Qa, lens_ptr, B, S_cap, out_K, out_V,
+                                             out_idx, out_count, h2o_state, device_status, stream)
 
 
 def kvev_status(handle: int) -> int:
