@@ -14,7 +14,11 @@ namespace kvev {
 constexpr int kMaxLayers = 128;       // layers in one plan
 constexpr int kMaxScoreLayers = 64;   // SnapKV/H2O layers (tensor maps travel as kernel params)
 constexpr int kTileKeys = 128;        // keys per tensor-core tile (MMA M or N)
-constexpr int kMinChunkTiles = 8;     // tiles per scoring work item (chunk), at least
+// Tiles per scoring work item (chunk), at least.  Larger chunks give each CTA
+// more slack before it needs a unit's normaliser and halve the partials to
+// merge; the cost is reuse distance (grid * chunk bytes between a tile's two
+// reads, ~78 MB at 16 tiles on 152 SMs, inside the 126 MB L2).
+constexpr int kMinChunkTiles = 16;
 constexpr int kScoreThreads = 320;    // 1 TMA warp, 1 MMA warp, 2 softmax warpgroups
 constexpr int kSelectThreads = 512;
 constexpr int kWsAlign = 256;
@@ -152,6 +156,28 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Same, with an L2 cache-eviction policy (from createpolicy).
+__device__ __forceinline__ void tma_load_2d_hint(void* dst, const CUtensorMap* map, int x, int y,
+                                                 uint64_t* bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
 }
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {

@@ -35,7 +35,8 @@ namespace kvev {
 namespace {
 
 struct Smem {
-  uint8_t* qbuf[2];
+  uint8_t* qbuf;     // two Q buffers of qbytes each, indexed arithmetically (a dynamically
+  uint32_t qbytes;   // indexed member array would push the whole struct to local memory)
   uint8_t* kbuf;     // stages * tile bytes
   float* lam[2];     // per warpgroup copy of lse2 of the current sweep-2 unit
   uint64_t* kfull;
@@ -54,10 +55,9 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   size_t off = 0;
   const size_t qbytes = static_cast<size_t>(p.q_rows) * D * 2;
   const size_t tbytes = static_cast<size_t>(kTileKeys) * D * 2;
-  s.qbuf[0] = base + off;
-  off += qbytes;
-  s.qbuf[1] = base + off;
-  off += qbytes;
+  s.qbuf = base + off;
+  s.qbytes = static_cast<uint32_t>(qbytes);
+  off += 2 * qbytes;
   s.kbuf = base + off;
   off += tbytes * p.stages;
   s.lam[0] = reinterpret_cast<float*>(base + off);
@@ -134,9 +134,11 @@ template <int D>
 __device__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
   const uint32_t qbytes = static_cast<uint32_t>(p.R_pad) * D * 2;
+  const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
+  const uint64_t drop = policy_evict_first();  // second read: its last use
   uint32_t tile = 0;
   int last_q_item = -1;
-  int issued_q[2] = {0, 0};
+  int issued_q0 = 0, issued_q1 = 0;  // Q loads issued into each buffer
   bool ok = true;
   for (int j = 0; j <= J && ok; ++j) {
     for (int sweep = 0; sweep < 2 && ok; ++sweep) {
@@ -153,9 +155,9 @@ __device__ void producer(const ScoreParams& p, const Smem& sm, int first, int st
         const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
 #pragma unroll
         for (int kc = 0; kc < D / 64; ++kc)
-          tma_load_2d(sm.qbuf[qb] + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
+          tma_load_2d(sm.qbuf + qb * sm.qbytes + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
                       kc * 64, qrow, &sm.qfull[qb]);
-        issued_q[qb] = jj + 1;
+        if (qb == 0) issued_q0 = jj + 1; else issued_q1 = jj + 1;
         last_q_item = jj;
       }
       const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
@@ -167,8 +169,8 @@ __device__ void producer(const ScoreParams& p, const Smem& sm, int first, int st
         mbar_expect_tx(&sm.kfull[st], kTileBytes);
 #pragma unroll
         for (int kc = 0; kc < D / 64; ++kc)
-          tma_load_2d(dst + kc * (kTileKeys * 128), kmap, kc * 64, row0 + i * kTileKeys,
-                      &sm.kfull[st]);
+          tma_load_2d_hint(dst + kc * (kTileKeys * 128), kmap, kc * 64, row0 + i * kTileKeys,
+                           &sm.kfull[st], sweep == 0 ? keep : drop);
       }
     }
   }
@@ -181,9 +183,8 @@ __device__ void producer(const ScoreParams& p, const Smem& sm, int first, int st
       const uint32_t last = ((tile - 1 - st) / S) * S + st;  // last tile issued into st
       wait_bar_drain(&sm.kfull[st], (last / S) & 1, 100000000ull);
     }
-    for (int qb = 0; qb < 2; ++qb)
-      if (issued_q[qb] > 0)
-        wait_bar_drain(&sm.qfull[qb], ((issued_q[qb] - 1) >> 1) & 1, 100000000ull);
+    if (issued_q0 > 0) wait_bar_drain(&sm.qfull[0], ((issued_q0 - 1) >> 1) & 1, 100000000ull);
+    if (issued_q1 > 0) wait_bar_drain(&sm.qfull[1], ((issued_q1 - 1) >> 1) & 1, 100000000ull);
   }
 }
 
@@ -208,7 +209,7 @@ __device__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_b
       const int t = first + jj * stride;
       const ItemInfo it = item_info(p, t);
       const int qb = jj & 1;
-      const uint32_t qaddr = smem_u32(sm.qbuf[qb]);
+      const uint32_t qaddr = smem_u32(sm.qbuf) + qb * sm.qbytes;
       if (sweep == 0) {
         if (!wait_bar(&sm.qfull[qb], (jj >> 1) & 1, p)) { ok = false; break; }
       }
@@ -389,19 +390,33 @@ __device__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_b
       }
       named_bar_sync(bar_id, 128);
       if (sm.flag[wg]) {
-        // last arrival for this unit: combine every chunk's partials into lse2
+        // Last arrival for this unit: merge every chunk's (max, sum) partials
+        // of each row into lse2 = M + log2(Z) in one pass, with eight
+        // independent loads in flight (this runs while the unit's other
+        // chunk-holders wait for it).
         for (int h = 0; h < nh; ++h) {
           const int r = h * 128 + lrow;
           if (r >= p.R_pad) continue;
           const float2* pp = p.part + static_cast<size_t>(it.cs) * 2 * p.R_pad + r;
-          float M = -INFINITY;
-          for (int q = 0; q < 2 * it.nchunks; ++q) M = fmaxf(M, __ldcg(&pp[q * p.R_pad]).x);
-          float Z = 0.f;
-          if (M != -INFINITY)
-            for (int q = 0; q < 2 * it.nchunks; ++q) {
-              const float2 mz = __ldcg(&pp[q * p.R_pad]);
-              if (mz.x != -INFINITY) Z += mz.y * ex2_approx(mz.x - M);
+          const int nq = 2 * it.nchunks;
+          float M = -INFINITY, Z = 0.f;
+          for (int q0 = 0; q0 < nq; q0 += 8) {
+            float2 e[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              e[i] = q0 + i < nq ? __ldcg(&pp[static_cast<size_t>(q0 + i) * p.R_pad])
+                                 : make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              if (e[i].x == -INFINITY) continue;
+              if (e[i].x > M) {
+                Z = Z * ex2_approx(M - e[i].x) + e[i].y;
+                M = e[i].x;
+              } else {
+                Z += e[i].y * ex2_approx(e[i].x - M);
+              }
             }
+          }
           p.lam[static_cast<size_t>(it.u) * p.R_pad + r] =
               (M == -INFINITY || Z <= 0.f) ? INFINITY : M + lg2_approx(Z);
         }
