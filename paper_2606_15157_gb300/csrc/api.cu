@@ -59,14 +59,14 @@ bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 struct WsLayout {
   int n_units = 0, R = 0, R_pad = 0, max_items = 0;
   size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item_unit = 0, part = 0,
-         lam = 0, raw = 0, total = 0;
+         lam = 0, raw = 0, raw1 = 0, total = 0;
 };
 
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   WsLayout w;
   w.n_units = static_cast<int>(p.score_layers.size()) * B * p.H_kv;
   w.R = p.G * p.W;
-  w.R_pad = (w.R + 15) / 16 * 16;
+  w.R_pad = (w.R + 31) / 32 * 32;  // whole 32-column TMEM loads in the second sweep
   const int chunk_min = kTileKeys * kMinChunkTiles;
   w.max_items = w.n_units * ((S_cap + chunk_min - 1) / chunk_min);
   size_t off = 0;
@@ -81,9 +81,15 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.ready = take(sizeof(int) * std::max(w.n_units, 1));
   w.chunk_start = take(sizeof(int) * (w.n_units + 1));
   w.item_unit = take(sizeof(int) * std::max(w.max_items, 1));
-  w.part = take(sizeof(float2) * 2 * static_cast<size_t>(w.max_items) * w.R_pad);
+  // sweep-1 partials: one record per (item, softmax warpgroup), of the rows of
+  // that warpgroup's 128-row group
+  const int part_rows = w.R_pad > 128 ? 128 : w.R_pad;
+  w.part = take(sizeof(float2) * kSoftmaxWGs * static_cast<size_t>(w.max_items) * part_rows);
   w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
   w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
+  // with two row groups the score kernel writes each score as two partial sums
+  // (rows 0-127 into raw, the rest into raw1); the selection kernel adds them
+  w.raw1 = take(w.R_pad > 128 ? sizeof(float) * static_cast<size_t>(w.n_units) * S_cap : 0);
   w.total = off;
   return w;
 }
@@ -469,6 +475,19 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
 
 namespace {
 
+// 1 when the compiled score kernel for head size d is launched with enough
+// registers for its setmaxnreg split, 0 when not, -1 when the query failed.
+int score_regs_ok(int d) {
+  static std::once_flag once[2];
+  static int ok[2] = {-1, -1};
+  const int i = d == 64 ? 0 : 1;
+  std::call_once(once[i], [&] {
+    const int regs = score_kernel_regs(d);
+    ok[i] = regs < 0 ? -1 : (regs * kScoreThreads >= kRegsNeeded ? 1 : 0);
+  });
+  return ok[i];
+}
+
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
                const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
                void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
@@ -534,6 +553,11 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     while (stages >= 2 && score_smem_bytes(P.d, q_rows, ws.R_pad, stages) + 1024 > D.smem_optin)
       --stages;
     if (stages < 2) return KVEV_ENOTSUP;
+    // The softmax warpgroups raise their register count with setmaxnreg,
+    // drawing on the registers the CTA was launched with; refuse to launch a
+    // build whose allocation could not cover that (the raise would never
+    // complete).
+    if (score_regs_ok(P.d) != 1) return KVEV_ENOTSUP;
     // Request more than half of the SM's shared memory so exactly one CTA is
     // resident per SM: its TMEM allocation then never waits on another CTA.
     const size_t smem = std::max<size_t>(score_smem_bytes(P.d, q_rows, ws.R_pad, stages),
@@ -554,7 +578,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.chunk_keys = pp.chunk_keys;
     sp.q_rows = q_rows;
     sp.stages = stages;
-    sp.tmem_buf_cols = (ws.R_pad > 128) ? 256 : 128;
     sp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));
     sp.inv_G = 1.0f / static_cast<float>(P.G);
     sp.lens = lens_ok;
@@ -567,6 +590,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.part = reinterpret_cast<float2*>(wsb + ws.part);
     sp.lam = reinterpret_cast<float*>(wsb + ws.lam);
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
+    sp.raw1 = ws.R_pad > 128 ? reinterpret_cast<float*>(wsb + ws.raw1) : nullptr;
     sp.wait_ns = P.wait_ns;
     sp.stall_unit = P.stall_unit;
     mark(KVEV_K_SCORE, 0);
@@ -603,7 +627,8 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.pool_type = P.pool_type;
   sel.sink = P.sink;
   sel.lens = lens_ok;
-  sel.raw = reinterpret_cast<const float*>(wsb + ws.raw);
+  sel.raw = reinterpret_cast<float*>(wsb + ws.raw);
+  sel.raw1 = ws.R_pad > 128 ? reinterpret_cast<const float*>(wsb + ws.raw1) : nullptr;
   sel.out_idx = out_idx;
   sel.out_count = out_count;
   const size_t sel_smem = ws.n_units > 0 ? sizeof(uint32_t) * static_cast<size_t>(S_cap) : 0;

@@ -19,7 +19,18 @@ constexpr int kTileKeys = 128;        // keys per tensor-core tile (MMA M or N)
 // merge; the cost is reuse distance (grid * chunk bytes between a tile's two
 // reads, ~78 MB at 16 tiles on 152 SMs, inside the 126 MB L2).
 constexpr int kMinChunkTiles = 16;
-constexpr int kScoreThreads = 320;    // 1 TMA warp, 1 MMA warp, 2 softmax warpgroups
+constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel (one per TMEM slot)
+constexpr int kScoreThreads = 128 * (1 + kSoftmaxWGs);  // + warpgroup 0: TMA warp, MMA warp, 2 idle
+constexpr int kSlots = 4;             // TMEM accumulator slots of the score kernel
+constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 512 columns)
+// Register split of the score kernel (setmaxnreg): warpgroup 0 shrinks to 56,
+// the softmax warpgroups grow to 104.  The CTA must be launched with at least
+// 128 * 56 + 512 * 104 = 60416 registers (96 per thread x 640): the host
+// checks the compiled allocation before launching, since an increase that the
+// launch pool cannot cover would never complete.
+constexpr int kRegsControl = 56;
+constexpr int kRegsSoftmax = 104;
+constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
 constexpr int kSelectThreads = 512;
 constexpr int kWsAlign = 256;
 
@@ -60,7 +71,6 @@ struct ScoreParams {
   int chunk_keys;     // keys per work item (multiple of 128)
   int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
   int stages;         // K tile ring depth
-  int tmem_buf_cols;  // TMEM columns per accumulator buffer (128 or 256)
   float scale_log2;   // log2(e) / sqrt(d)
   float inv_G;
   const int* lens;
@@ -70,9 +80,11 @@ struct ScoreParams {
   int* ready;
   int* abort_flag;
   int* status;
-  float2* part;       // [items][2][R_pad] per-row (max, sum) partials, base-2 units
+  float2* part;       // [items][4][PR] per-row (max, sum) partials per softmax warpgroup,
+                      // base-2 units; PR = 128 when R_pad > 128, else R_pad
   float* lam;         // [n_units][R_pad] per-row log2-sum-exp
-  float* raw;         // [n_units][S_cap] window scores
+  float* raw;         // [n_units][S_cap] window scores (rows 0-127 partial when R_pad > 128)
+  float* raw1;        // [n_units][S_cap] rows 128+ partial when R_pad > 128
   long long wait_ns;
   int stall_unit;
 };
@@ -81,7 +93,8 @@ struct SelectParams {
   LayerDesc layer[kMaxLayers];
   int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink;
   const int* lens;
-  const float* raw;   // [n_units][S_cap]
+  float* raw;         // [n_units][S_cap]
+  const float* raw1;  // second partial of each score (R_pad > 128), or nullptr
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
 };
@@ -229,6 +242,69 @@ __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Issue a load of 32 consecutive fp32 columns of this thread's TMEM lane; the
+// registers are valid only after tmem_wait32() on the same array.
+__device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
+
+// Wait for every outstanding TMEM load.  The array is tied to the wait as an
+// in/out operand so no use of its registers can be scheduled before it.
+__device__ __forceinline__ void tmem_wait32(uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+        "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
+        "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]),
+        "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]),
+        "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]),
+        "+r"(r[31])
+      :
+      : "memory");
+}
+
+// Two-lane packed fp32 fused multiply-add (one instruction for two values).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  uint64_t ra, rb, rc, rd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
+  float2 d;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+__device__ __forceinline__ float4 lds4(const float* p) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(smem_u32(p)));
+  return v;
+}
+
+__device__ __forceinline__ float lds1(const float* p) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(smem_u32(p)));
+  return v;
+}
+
 // 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
@@ -293,6 +369,15 @@ __device__ __forceinline__ float lg2_approx(float x) {
   return y;
 }
 
+template <int N>
+__device__ __forceinline__ void regs_dealloc() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void regs_alloc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
@@ -324,6 +409,7 @@ namespace kvev {
 cudaError_t launch_prologue(const PrologueParams& p, cudaStream_t s);
 cudaError_t launch_score(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
 int score_smem_bytes(int d, int q_rows, int R_pad, int stages);
+int score_kernel_regs(int d);
 cudaError_t score_set_smem(int d, size_t smem);
 cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s);
 cudaError_t select_set_smem(size_t smem);

@@ -24,10 +24,15 @@
 // co-resident (cooperative launch) and a unit spans at most two rounds of
 // items, so the wait always ends.
 //
-// Roles per CTA (320 threads): warp 0 issues TMA loads (one thread), warp 1
-// owns TMEM and issues tcgen05.mma (one thread), warps 2-5 and 6-9 are two
-// softmax warpgroups that take alternate tiles, each with its own TMEM
-// accumulator buffer.
+// Roles per CTA (640 threads, five warpgroups): warp 0 issues TMA loads (one
+// thread), warp 1 owns TMEM and issues tcgen05.mma (one thread), warps 2-3
+// idle; warpgroups 1-4 are softmax warpgroups.  TMEM is four 128-column
+// slots, one per 128-row group of a tile's accumulator (a tile uses one or
+// two), and softmax warpgroup w owns slot w: it copies the slot to registers
+// in 64-column pieces and releases it before the last piece's arithmetic, so
+// the tensor core keeps filling the other slots meanwhile.  The softmax
+// warpgroups never wait on each other.  setmaxnreg moves registers from
+// warpgroup 0 to the softmax warpgroups.
 #include "kvev_internal.cuh"
 
 namespace kvev {
@@ -38,7 +43,7 @@ struct Smem {
   uint8_t* qbuf;     // two Q buffers of qbytes each, indexed arithmetically (a dynamically
   uint32_t qbytes;   // indexed member array would push the whole struct to local memory)
   uint8_t* kbuf;     // stages * tile bytes
-  float* lam[2];     // per warpgroup copy of lse2 of the current sweep-2 unit
+  float* lam;        // [4][R_pad]: per-warpgroup copy of -lse2 of the current sweep-2 unit
   uint64_t* kfull;
   uint64_t* kempty;
   uint64_t* qfull;
@@ -47,7 +52,7 @@ struct Smem {
   uint64_t* tempty;
   uint64_t* done;
   uint32_t* tmem_slot;
-  int* flag;         // [4]: [wg] last-arrival of sweep 1, [2+wg] ready of sweep 2
+  int* flag;         // [8]: [wg] last-arrival of sweep 1, [4+wg] ready of sweep 2
 };
 
 __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D) {
@@ -60,10 +65,8 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   off += 2 * qbytes;
   s.kbuf = base + off;
   off += tbytes * p.stages;
-  s.lam[0] = reinterpret_cast<float*>(base + off);
-  off += sizeof(float) * p.R_pad;
-  s.lam[1] = reinterpret_cast<float*>(base + off);
-  off += sizeof(float) * p.R_pad;
+  s.lam = reinterpret_cast<float*>(base + off);
+  off += kSoftmaxWGs * sizeof(float) * p.R_pad;
   off = (off + 7) & ~size_t(7);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + off);
   s.kfull = bars;
@@ -71,8 +74,8 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   s.qfull = bars + 2 * p.stages;
   s.qempty = s.qfull + 2;
   s.tfull = s.qempty + 2;
-  s.tempty = s.tfull + 2;
-  s.done = s.tempty + 2;
+  s.tempty = s.tfull + kSlots;
+  s.done = s.tempty + kSlots;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.done + 1);
   s.flag = reinterpret_cast<int*>(s.tmem_slot + 1);
   return s;
@@ -131,7 +134,7 @@ __device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, u
 // Producer: TMA loads of Q (once per item) and of K tiles (twice per item).
 // ---------------------------------------------------------------------------
 template <int D>
-__device__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
+__device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
   const uint32_t qbytes = static_cast<uint32_t>(p.R_pad) * D * 2;
   const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
@@ -192,14 +195,16 @@ __device__ void producer(const ScoreParams& p, const Smem& sm, int first, int st
 // MMA issuer (one thread): sweep 1 -> S = Q K^T, sweep 2 -> S^T = K Q^T.
 // ---------------------------------------------------------------------------
 template <int D>
-__device__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_base, int first,
+__device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_base, int first,
                            int stride, int J) {
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
   const int nh = p.R_pad > 128 ? 2 : 1;
   const uint32_t idesc1 = idesc_bf16_f32(128, kTileKeys);
-  const uint32_t idesc2 = idesc_bf16_f32(128, p.R_pad);
+  // sweep 2: N = rows of the group (128, or what is left of R_pad in the last group)
+  const uint32_t idesc2a = idesc_bf16_f32(128, p.R_pad > 128 ? 128 : p.R_pad);
+  const uint32_t idesc2b = idesc_bf16_f32(128, p.R_pad > 128 ? p.R_pad - 128 : 128);
   const uint32_t qcol_bytes = static_cast<uint32_t>(p.q_rows) * 128;  // one 64-wide column block
-  uint32_t tile = 0;
+  uint32_t tile = 0, slot = 0;
   bool ok = true;
   for (int j = 0; j <= J && ok; ++j) {
     for (int sweep = 0; sweep < 2 && ok; ++sweep) {
@@ -215,32 +220,35 @@ __device__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_b
       }
       for (int i = 0; i < it.ntiles; ++i, ++tile) {
         const uint32_t st = tile % p.stages;
-        const uint32_t buf = tile & 1;
         if (!wait_bar(&sm.kfull[st], (tile / p.stages) & 1, p)) { ok = false; break; }
-        if (!wait_bar(&sm.tempty[buf], ((tile >> 1) & 1) ^ 1, p)) { ok = false; break; }
-        tc_fence_after();
         const uint32_t kaddr = smem_u32(sm.kbuf) + st * kTileBytes;
-        const uint32_t dcol = tmem_base + buf * p.tmem_buf_cols;
-        if (sweep == 0) {
-          for (int h = 0; h < nh; ++h) {
+        // One 128-column TMEM slot per 128-row group of Q: sweep 1 writes
+        // S[rows of group h][keys], sweep 2 writes S^T[keys][rows of group h].
+        for (int h = 0; h < nh && ok; ++h, ++slot) {
+          const uint32_t sl = slot % kSlots;
+          if (!wait_bar(&sm.tempty[sl], ((slot / kSlots) & 1) ^ 1, p)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t dcol = tmem_base + sl * kSlotCols;
+          if (sweep == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
               const uint32_t koff = (k >> 2) * (kTileKeys * 128) + (k & 3) * 32;
               const uint32_t qoff = (k >> 2) * qcol_bytes + h * (128 * 128) + (k & 3) * 32;
-              umma_bf16(dcol + h * 128, sw128_desc(qaddr + qoff), sw128_desc(kaddr + koff),
-                        idesc1, k > 0);
+              umma_bf16(dcol, sw128_desc(qaddr + qoff), sw128_desc(kaddr + koff), idesc1, k > 0);
+            }
+          } else {
+            const uint32_t idesc2 = h == 0 ? idesc2a : idesc2b;
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+              const uint32_t koff = (k >> 2) * (kTileKeys * 128) + (k & 3) * 32;
+              const uint32_t qoff = (k >> 2) * qcol_bytes + h * (128 * 128) + (k & 3) * 32;
+              umma_bf16(dcol, sw128_desc(kaddr + koff), sw128_desc(qaddr + qoff), idesc2, k > 0);
             }
           }
-        } else {
-#pragma unroll
-          for (int k = 0; k < D / 16; ++k) {
-            const uint32_t koff = (k >> 2) * (kTileKeys * 128) + (k & 3) * 32;
-            const uint32_t qoff = (k >> 2) * qcol_bytes + (k & 3) * 32;
-            umma_bf16(dcol, sw128_desc(kaddr + koff), sw128_desc(qaddr + qoff), idesc2, k > 0);
-          }
+          umma_commit(&sm.tfull[sl]);
         }
+        if (!ok) break;
         umma_commit(&sm.kempty[st]);
-        umma_commit(&sm.tfull[buf]);
       }
       if (ok && sweep == 1) umma_commit(&sm.qempty[qb]);
     }
@@ -258,100 +266,177 @@ __device__ __forceinline__ int row_pos(const ScoreParams& p, int r, int n) {
   return n - p.W + (r % p.W);
 }
 
-// Sweep 1 on one tile: update the running base-2 (max, sum) of the rows this
-// thread owns (row lrow of each 128-row half).
-__device__ __forceinline__ void sweep1_tile(const ScoreParams& p, uint32_t taddr, int lrow,
-                                            int nh, int n, int kb, float (&m)[2], float (&z)[2]) {
+__device__ __forceinline__ float max32(const float (&v)[32]) {
+  float t[11];
+#pragma unroll
+  for (int j = 0; j < 10; ++j) t[j] = fmax3(v[3 * j], v[3 * j + 1], v[3 * j + 2]);
+  t[10] = fmaxf(v[30], v[31]);
+  const float a = fmax3(t[0], t[1], t[2]), b = fmax3(t[3], t[4], t[5]);
+  const float c = fmax3(t[6], t[7], t[8]), e = fmax3(t[9], t[10], a);
+  return fmax3(b, c, e);
+}
+
+__device__ __forceinline__ float sum8(const float (&a)[8]) {
+  return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+}
+
+// One 32-key chunk of sweep 1 for one row: online base-2 (max, sum) update.
+__device__ __forceinline__ void s1_chunk(const uint32_t (&rr)[32], float c, bool full, int k0,
+                                         int tr, float& m, float& z) {
+  float v[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
+  if (!full) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (k0 + i > tr) v[i] = -INFINITY;
+  }
+  const float mx = max32(v);
+  if (mx == -INFINITY) return;
+  const float mnew = fmaxf(m, mx * c);
+  const float zs = z * ex2_approx(m - mnew);  // m = -inf -> 0
+  const float2 cc = make_float2(c, c), nm = make_float2(-mnew, -mnew);
+  float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 32; i += 2) {
+    const float2 t = ffma2(make_float2(v[i], v[i + 1]), cc, nm);
+    a[i & 7] += ex2_approx(t.x);
+    a[(i + 1) & 7] += ex2_approx(t.y);
+  }
+  z = zs + sum8(a);
+  m = mnew;
+}
+
+// One 32-row chunk of sweep 2 for this thread's key: sum of exp2(s*c - lse2_r)
+// into eight accumulators; nl = -lse2 of the chunk's rows (shared memory).
+__device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&rr)[32], bool full,
+                                         const float* nl, int r0, int k, int n, float (&a)[8]) {
   const float c = p.scale_log2;
-  for (int h = 0; h < 2; ++h) {
-    if (h >= nh) break;
-    const int r = h * 128 + lrow;
-    const bool row_ok = r < p.R;
-    const int tr = row_ok ? row_pos(p, r, n) : -1;
-    const bool full = (kb + kTileKeys - 1) <= (n - p.W);  // every key visible to every row
-#pragma unroll 1
-    for (int c0 = 0; c0 < kTileKeys; c0 += 32) {
-      float v[32];
-      tmem_ld32(taddr + h * 128 + c0, v);
-      if (!row_ok || tr < 0) continue;
-      float vmax = -INFINITY;
-      if (full) {
+  const float2 cc = make_float2(c, c);
+  if (full) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) vmax = fmaxf(vmax, v[i]);
-      } else {
+    for (int i = 0; i < 32; i += 4) {
+      const float4 l4 = lds4(nl + i);
+      const float2 t0 = ffma2(make_float2(__uint_as_float(rr[i]), __uint_as_float(rr[i + 1])), cc,
+                              make_float2(l4.x, l4.y));
+      const float2 t1 = ffma2(make_float2(__uint_as_float(rr[i + 2]), __uint_as_float(rr[i + 3])),
+                              cc, make_float2(l4.z, l4.w));
+      a[i & 7] += ex2_approx(t0.x);
+      a[(i + 1) & 7] += ex2_approx(t0.y);
+      a[(i + 2) & 7] += ex2_approx(t1.x);
+      a[(i + 3) & 7] += ex2_approx(t1.y);
+    }
+  } else {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          if (kb + c0 + i > tr) v[i] = -INFINITY;
-          vmax = fmaxf(vmax, v[i]);
-        }
-      }
-      if (vmax == -INFINITY) continue;
-      const float mnew = fmaxf(m[h], vmax * c);
-      float zz = z[h] * ex2_approx(m[h] - mnew);  // m = -inf -> 0
-      float acc0 = 0.f, acc1 = 0.f;
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        acc0 += ex2_approx(fmaf(v[i], c, -mnew));
-        acc1 += ex2_approx(fmaf(v[i + 1], c, -mnew));
-      }
-      z[h] = zz + (acc0 + acc1);
-      m[h] = mnew;
+    for (int i = 0; i < 32; ++i) {
+      const int r = r0 + i;
+      if (r < p.R && k <= row_pos(p, r, n))
+        a[i & 7] += ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
     }
   }
 }
 
-// Sweep 2 on one tile: this thread's key kb + lrow against all R rows.
-__device__ __forceinline__ void sweep2_tile(const ScoreParams& p, uint32_t taddr, int lrow, int n,
-                                            int kb, const float* lam, float* raw_unit) {
-  const float c = p.scale_log2;
-  const int k = kb + lrow;
-  const bool key_ok = k < n;
-  const bool full = (kb + kTileKeys - 1) < (n - p.W);  // every row sees every key of the tile
-  float acc0 = 0.f, acc1 = 0.f;
-  int c0 = 0;
-#pragma unroll 1
-  for (; c0 + 32 <= p.R_pad; c0 += 32) {
-    float v[32];
-    tmem_ld32(taddr + c0, v);
-    if (!key_ok) continue;
-    if (full && c0 + 32 <= p.R) {
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        acc0 += ex2_approx(fmaf(v[i], c, -lam[c0 + i]));
-        acc1 += ex2_approx(fmaf(v[i + 1], c, -lam[c0 + i + 1]));
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int r = c0 + i;
-        if (r < p.R && k <= row_pos(p, r, n)) acc0 += ex2_approx(fmaf(v[i], c, -lam[r]));
-      }
-    }
-  }
-  if (c0 < p.R_pad) {  // a 16-column tail
-    float v[16];
-    tmem_ld16(taddr + c0, v);
-    if (key_ok) {
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int r = c0 + i;
-        if (r < p.R && k <= row_pos(p, r, n)) acc0 += ex2_approx(fmaf(v[i], c, -lam[r]));
-      }
-    }
-  }
-  if (key_ok) raw_unit[k] = (acc0 + acc1) * p.inv_G;
+// ---- TMEM slot hand-off --------------------------------------------------
+// A warpgroup waits for slot g to be filled, copies its part of the slot into
+// registers, and releases the slot before doing any arithmetic, so the MMA of
+// later tiles overlaps the exponentials.
+
+__device__ __forceinline__ bool slot_acquire(const ScoreParams& p, const Smem& sm, uint32_t g,
+                                             bool ok) {
+  if (ok && !wait_bar(&sm.tfull[g % kSlots], (g / kSlots) & 1, p)) ok = false;
+  ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld needs the whole warp
+  if (ok) tc_fence_after();
+  return ok;
 }
 
-__device__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base, int wg,
-                           int first, int stride, int J) {
+__device__ __forceinline__ void slot_release(const Smem& sm, uint32_t g) {
+  tc_fence_before();
+  mbar_arrive(&sm.tempty[g % kSlots]);
+}
+
+template <int NCH>
+__device__ __forceinline__ void load_slot(uint32_t taddr, uint32_t (&r)[NCH][32]) {
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) tmem_ld32_async(taddr + c * 32, r[c]);
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) tmem_wait32(r[c]);
+}
+
+// Sweep 1, slot g: this thread's row `row` against the tile's 128 keys, in two
+// 64-column pieces (copy, then arithmetic); the slot is released after the
+// second copy.
+__device__ __forceinline__ void s1_slot(const ScoreParams& p, const Smem& sm, uint32_t lane_addr,
+                                        uint32_t g, bool& ok, int row, int n, int kb, float& m,
+                                        float& z) {
+  ok = slot_acquire(p, sm, g, ok);
+  const int tr = row < p.R ? row_pos(p, row, n) : -1;
+  const bool full = (kb + kTileKeys - 1) <= (n - p.W);  // every key visible to every row
+#pragma unroll
+  for (int piece = 0; piece < 2; ++piece) {
+    // Loaded even when the wait failed (the address is always inside this
+    // CTA's TMEM allocation; the values are then discarded): a conditional
+    // load would leave the array undefined on one path and spill it.
+    uint32_t r[2][32];
+    load_slot<2>(lane_addr + piece * 64, r);
+    if (piece == 1) slot_release(sm, g);
+    if (ok && tr >= 0) {
+      s1_chunk(r[0], p.scale_log2, full, kb + piece * 64, tr, m, z);
+      s1_chunk(r[1], p.scale_log2, full, kb + piece * 64 + 32, tr, m, z);
+    }
+  }
+}
+
+// Sweep 2, slot g: this thread's key k against rows r0 .. r0 + 32*nch, in
+// pieces of up to 64 columns; partial sum into a[8].
+template <int NCH>
+__device__ __forceinline__ void s2_piece(const ScoreParams& p, uint32_t taddr, bool ok, bool full,
+                                         const float* nl, int r0, int k, int n, float (&a)[8]) {
+  uint32_t r[NCH][32];
+  load_slot<NCH>(taddr, r);
+  if (!ok || k >= n) return;
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) s2_chunk(p, r[c], full, nl + c * 32, r0 + c * 32, k, n, a);
+}
+
+__device__ __forceinline__ void s2_slot(const ScoreParams& p, const Smem& sm, uint32_t lane_addr,
+                                        uint32_t g, bool& ok, int nch, int r0, int k, int n,
+                                        int kb, const float* nlam, float (&a)[8]) {
+  ok = slot_acquire(p, sm, g, ok);
+  const bool full = (kb + kTileKeys - 1 <= n - p.W) && (r0 + nch * 32 <= p.R);
+  for (int c = 0; c < nch; c += 2) {
+    if (c + 1 < nch)
+      s2_piece<2>(p, lane_addr + c * 32, ok, full, nlam + r0 + c * 32, r0 + c * 32, k, n, a);
+    else
+      s2_piece<1>(p, lane_addr + c * 32, ok, full, nlam + r0 + c * 32, r0 + c * 32, k, n, a);
+  }
+  slot_release(sm, g);
+}
+
+// Softmax warpgroup wg (0..3) owns TMEM slot wg.  Slot g of the tile stream
+// (tile t, 128-row group h -> g = t*nh + h) lands in slot g % 4, so with
+// nh = 2 warpgroup wg handles row group wg & 1 of the tiles t = wg >> 1 (mod 2)
+// and with nh = 1 the whole of tiles t = wg (mod 4).  No two warpgroups
+// share a slot or synchronise with each other; partial results go to global
+// memory (sweep 1: per-row (max, sum) per warpgroup; sweep 2: one partial sum
+// per 128-row group, added by the selection kernel).
+__device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base,
+                                           int wg, int first, int stride, int J) {
   const int warp = threadIdx.x >> 5;
-  const int quarter = warp & 3;           // TMEM lane quarter this warp may access
-  const int lrow = quarter * 32 + (threadIdx.x & 31);
-  const int wtid = threadIdx.x - (2 + 4 * wg) * 32;  // 0..127 within the warpgroup
+  const int quarter = warp & 3;                       // TMEM lane quarter of this warp
+  const int lrow = quarter * 32 + (threadIdx.x & 31);  // TMEM lane: row (sweep 1) / key (sweep 2)
+  const int wtid = threadIdx.x - (4 + 4 * wg) * 32;    // 0..127 within the warpgroup
   const int bar_id = 1 + wg;
-  const int nh = p.R_pad > 128 ? 2 : 1;
-  const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16);
-  float* lam_s = sm.lam[wg];
+  const int nh = p.R_pad > 128 ? 2 : 1;                // 128-row groups (slots) per tile
+  const int half = nh == 2 ? (wg & 1) : 0;             // row group of this warpgroup
+  const uint32_t tmod = nh == 2 ? 2 : 4, tres = nh == 2 ? (wg >> 1) : wg;
+  const int row = half * 128 + lrow;                   // sweep-1 row of this thread
+  const int r0 = half * 128;                           // sweep-2 first row
+  const int nch = (nh == 2 ? (half == 0 ? 128 : p.R_pad - 128) : p.R_pad) / 32;
+  const int PR = nh == 2 ? 128 : p.R_pad;              // rows per sweep-1 partial record
+  float* raw_out = half == 0 ? p.raw : p.raw1;
+  const uint32_t lane_addr =
+      tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + wg * kSlotCols;
+  float* nlam = sm.lam + wg * p.R_pad;  // -lse2 of the current sweep-2 unit
   uint32_t tile = 0;
   bool ok = true;
 
@@ -360,52 +445,46 @@ __device__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_b
     if (j < J) {
       const int t = first + j * stride;
       const ItemInfo it = item_info(p, t);
-      float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f};
+      float m = -INFINITY, z = 0.f;
       for (int i = 0; i < it.ntiles; ++i) {
         const uint32_t gt = tile + i;
-        if ((gt & 1) != static_cast<uint32_t>(wg)) continue;
-        if (ok && !wait_bar(&sm.tfull[wg], (gt >> 1) & 1, p)) ok = false;
-        ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld needs the whole warp
-        if (ok) {
-          tc_fence_after();
-          sweep1_tile(p, lane_addr + wg * p.tmem_buf_cols, lrow, nh, it.n,
-                      it.key0 + i * kTileKeys, m, z);
-        }
-        tc_fence_before();
-        mbar_arrive(&sm.tempty[wg]);
+        if (gt % tmod != tres) continue;
+        s1_slot(p, sm, lane_addr, gt * nh + half, ok, row, it.n, it.key0 + i * kTileKeys, m, z);
       }
       tile += it.ntiles;
-      // publish this warpgroup's partial of the chunk
-      float2* part = p.part + (static_cast<size_t>(t) * 2 + wg) * p.R_pad;
-      for (int h = 0; h < nh; ++h) {
-        const int r = h * 128 + lrow;
-        if (r < p.R_pad) part[r] = make_float2(m[h], z[h]);
-      }
+      // publish this warpgroup's (max, sum) partial of the chunk: entry
+      // [t][wg][lrow] of rows PR = 128 (two row groups) or R_pad (one)
+      if (row < p.R_pad)
+        p.part[(static_cast<size_t>(t) * kSoftmaxWGs + wg) * PR + lrow] = make_float2(m, z);
       __threadfence();
       named_bar_sync(bar_id, 128);
       if (wtid == 0) {
         const int old = atomicAdd(&p.cnt[it.u], 1);
         __threadfence();
-        sm.flag[wg] = (old == 2 * it.nchunks - 1);
+        sm.flag[wg] = (old == kSoftmaxWGs * it.nchunks - 1);
       }
       named_bar_sync(bar_id, 128);
       if (sm.flag[wg]) {
-        // Last arrival for this unit: merge every chunk's (max, sum) partials
-        // of each row into lse2 = M + log2(Z) in one pass, with eight
-        // independent loads in flight (this runs while the unit's other
-        // chunk-holders wait for it).
-        for (int h = 0; h < nh; ++h) {
-          const int r = h * 128 + lrow;
-          if (r >= p.R_pad) continue;
-          const float2* pp = p.part + static_cast<size_t>(it.cs) * 2 * p.R_pad + r;
-          const int nq = 2 * it.nchunks;
+        // Last arrival for this unit: merge every chunk's partials of each row
+        // into lse2 = M + log2(Z), one pass, eight independent loads in flight.
+        for (int r = wtid; r < p.R_pad; r += 128) {
+          // entries of row r: one per warpgroup and chunk, of which only the
+          // two warpgroups of r's row group wrote when nh = 2
+          const int per_chunk = nh == 2 ? 2 : kSoftmaxWGs;
+          const int nq = per_chunk * it.nchunks;
+          const float2* base =
+              p.part + static_cast<size_t>(it.cs) * kSoftmaxWGs * PR + (nh == 2 ? (r & 127) : r);
           float M = -INFINITY, Z = 0.f;
           for (int q0 = 0; q0 < nq; q0 += 8) {
             float2 e[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-              e[i] = q0 + i < nq ? __ldcg(&pp[static_cast<size_t>(q0 + i) * p.R_pad])
-                                 : make_float2(-INFINITY, 0.f);
+            for (int i = 0; i < 8; ++i) {
+              const int q = q0 + i;
+              // chunk q / per_chunk, warpgroup: nh=2 -> (r >> 7) + 2*(q & 1); nh=1 -> q & 3
+              const int w = nh == 2 ? ((r >> 7) + 2 * (q & 1)) : (q & 3);
+              e[i] = q < nq ? __ldcg(&base[(static_cast<size_t>(q / per_chunk) * kSoftmaxWGs + w) * PR])
+                            : make_float2(-INFINITY, 0.f);
+            }
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
               if (e[i].x == -INFINITY) continue;
@@ -446,26 +525,22 @@ __device__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_b
             }
           }
         }
-        sm.flag[2 + wg] = ready;
+        sm.flag[4 + wg] = ready;
       }
       named_bar_sync(bar_id, 128);
-      const bool have = sm.flag[2 + wg] != 0;
-      for (int r = wtid; r < p.R_pad; r += 128)
-        lam_s[r] = have ? __ldcg(&p.lam[static_cast<size_t>(it.u) * p.R_pad + r]) : INFINITY;
+      const bool have = sm.flag[4 + wg] != 0;
+      for (int r = r0 + wtid; r < r0 + nch * 32; r += 128)  // stored negated: exp2(s*c + (-lse2))
+        nlam[r] = have ? -__ldcg(&p.lam[static_cast<size_t>(it.u) * p.R_pad + r]) : -INFINITY;
       named_bar_sync(bar_id, 128);
-      float* raw_unit = p.raw + static_cast<size_t>(it.u) * p.S_cap;
+      float* out = raw_out + static_cast<size_t>(it.u) * p.S_cap;
       for (int i = 0; i < it.ntiles; ++i) {
         const uint32_t gt = tile + i;
-        if ((gt & 1) != static_cast<uint32_t>(wg)) continue;
-        if (ok && !wait_bar(&sm.tfull[wg], (gt >> 1) & 1, p)) ok = false;
-        ok = __all_sync(0xffffffffu, ok);
-        if (ok) {
-          tc_fence_after();
-          sweep2_tile(p, lane_addr + wg * p.tmem_buf_cols, lrow, it.n, it.key0 + i * kTileKeys,
-                      lam_s, raw_unit);
-        }
-        tc_fence_before();
-        mbar_arrive(&sm.tempty[wg]);
+        if (gt % tmod != tres) continue;
+        const int kb = it.key0 + i * kTileKeys;
+        const int k = kb + lrow;
+        float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        s2_slot(p, sm, lane_addr, gt * nh + half, ok, nch, r0, k, it.n, kb, nlam, a);
+        if (ok && k < it.n) out[k] = sum8(a) * p.inv_G;
       }
       tile += it.ntiles;
     }
@@ -489,15 +564,17 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.qfull[i], 1);
       mbar_init(&sm.qempty[i], 1);
+    }
+    for (int i = 0; i < kSlots; ++i) {
       mbar_init(&sm.tfull[i], 1);
-      mbar_init(&sm.tempty[i], 128);
+      mbar_init(&sm.tempty[i], 128);  // the 128 threads of the warpgroup that owns the tile
     }
     mbar_init(sm.done, 1);
     fence_barrier_init();
     fence_proxy_async();
   }
   if (warp == 1) {
-    tmem_alloc(sm.tmem_slot, 2 * p.tmem_buf_cols);
+    tmem_alloc(sm.tmem_slot, kSlots * kSlotCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -509,18 +586,19 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
   const int first = blockIdx.x, stride = gridDim.x;
   const int J = first < total ? (total - first + stride - 1) / stride : 0;
 
-  if (warp == 0) {
-    if ((threadIdx.x & 31) == 0) producer<D>(p, sm, first, stride, J);
-  } else if (warp == 1) {
-    if ((threadIdx.x & 31) == 0) mma_issuer<D>(p, sm, tmem_base, first, stride, J);
+  if (warp < 4) {
+    regs_dealloc<kRegsControl>();
+    if (warp == 0 && (threadIdx.x & 31) == 0) producer<D>(p, sm, first, stride, J);
+    if (warp == 1 && (threadIdx.x & 31) == 0) mma_issuer<D>(p, sm, tmem_base, first, stride, J);
   } else {
-    softmax_wg(p, sm, tmem_base, (warp - 2) >> 2, first, stride, J);
+    regs_alloc<kRegsSoftmax>();
+    softmax_wg(p, sm, tmem_base, (warp - 4) >> 2, first, stride, J);  // warpgroups 0..3
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 2 * p.tmem_buf_cols);
+    tmem_dealloc(tmem_base, kSlots * kSlotCols);
   }
 }
 
@@ -595,11 +673,18 @@ int score_smem_bytes(int d, int q_rows, int R_pad, int stages) {
   size_t off = 0;
   off += 2 * static_cast<size_t>(q_rows) * d * 2;
   off += static_cast<size_t>(stages) * kTileKeys * d * 2;
-  off += 2 * sizeof(float) * R_pad;
+  off += kSoftmaxWGs * sizeof(float) * R_pad;
   off = (off + 7) & ~size_t(7);
-  off += sizeof(uint64_t) * (2 * stages + 9);
-  off += sizeof(uint32_t) + 4 * sizeof(int);
+  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1);
+  off += sizeof(uint32_t) + 8 * sizeof(int);
   return static_cast<int>((off + 127) & ~size_t(127));
+}
+
+int score_kernel_regs(int d) {
+  cudaFuncAttributes a = {};
+  const cudaError_t e = d == 64 ? cudaFuncGetAttributes(&a, score_kernel<64>)
+                                : cudaFuncGetAttributes(&a, score_kernel<128>);
+  return e == cudaSuccess ? a.numRegs : -1;
 }
 
 cudaError_t score_set_smem(int d, size_t smem) {
