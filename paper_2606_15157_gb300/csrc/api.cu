@@ -58,7 +58,7 @@ bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 
 struct WsLayout {
   int n_units = 0, R = 0, R_pad = 0, max_items = 0;
-  size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item_unit = 0, part = 0,
+  size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
          lam = 0, raw = 0, raw1 = 0, total = 0;
 };
 
@@ -80,7 +80,7 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.cnt = take(sizeof(int) * std::max(w.n_units, 1));
   w.ready = take(sizeof(int) * std::max(w.n_units, 1));
   w.chunk_start = take(sizeof(int) * (w.n_units + 1));
-  w.item_unit = take(sizeof(int) * std::max(w.max_items, 1));
+  w.item = take(sizeof(int4) * std::max(w.max_items, 1));
   // sweep-1 partials: one record per (item, softmax warpgroup), of the rows of
   // that warpgroup's 128-row group
   const int part_rows = w.R_pad > 128 ? 128 : w.R_pad;
@@ -506,6 +506,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   const int grid = D.num_sms;
   const int tiles_max = (S_cap + kTileKeys - 1) / kTileKeys;
   const int chunk_tiles = std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid);
+  if (chunk_tiles > 0xFFFF) return KVEV_ENOTSUP;  // tiles per item are packed in 16 bits
   PrologueParams pp = {};
   pp.n_units = ws.n_units;
   pp.B = B;
@@ -523,7 +524,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   pp.ready = reinterpret_cast<int*>(wsb + ws.ready);
   pp.abort_flag = reinterpret_cast<int*>(wsb + ws.abort_flag);
   pp.chunk_start = reinterpret_cast<int*>(wsb + ws.chunk_start);
-  pp.item_unit = reinterpret_cast<int*>(wsb + ws.item_unit);
+  pp.item = reinterpret_cast<int4*>(wsb + ws.item);
   for (bool& b : P.launched) b = false;
   P.timed_call = P.timing;
   auto mark = [&](int k, int which) {
@@ -582,7 +583,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.inv_G = 1.0f / static_cast<float>(P.G);
     sp.lens = lens_ok;
     sp.chunk_start = pp.chunk_start;
-    sp.item_unit = pp.item_unit;
+    sp.item = pp.item;
     sp.cnt = pp.cnt;
     sp.ready = pp.ready;
     sp.abort_flag = pp.abort_flag;

@@ -85,48 +85,61 @@ struct ItemInfo {
   int u, s, h, ls, n, key0, ntiles, cs, nchunks;
 };
 
-__device__ __forceinline__ ItemInfo item_info(const ScoreParams& p, int t) {
+// Work item t from its packed record (written by the prologue: one 16-byte load).
+__device__ __forceinline__ int4 load_item(const ScoreParams& p, int t) { return __ldg(&p.item[t]); }
+
+__device__ __forceinline__ ItemInfo decode_item(const ScoreParams& p, int t, int4 r) {
   ItemInfo it;
-  it.u = p.item_unit[t];
-  it.cs = p.chunk_start[it.u];
-  it.nchunks = p.chunk_start[it.u + 1] - it.cs;
+  it.u = r.x;
+  it.n = r.y;
+  it.key0 = r.z;
+  it.ntiles = r.w & 0xFFFF;
+  it.nchunks = r.w >> 16;
+  it.cs = t - it.key0 / p.chunk_keys;
   const int per_layer = p.B * p.H_kv;
   it.ls = it.u / per_layer;
   const int rem = it.u - it.ls * per_layer;
   it.s = rem / p.H_kv;
   it.h = rem - it.s * p.H_kv;
-  it.n = p.lens[it.s];
-  const int c = t - it.cs;
-  it.key0 = c * p.chunk_keys;
-  int nk = it.n - it.key0;
-  if (nk > p.chunk_keys) nk = p.chunk_keys;
-  it.ntiles = (nk + kTileKeys - 1) / kTileKeys;
   return it;
 }
 
-// Bounded wait on an mbarrier phase; false if it ran out or another role aborted.
+// Items a role needs at step j of the lag-1 loop: j (sweep 1) and j-1
+// (sweep 2).  At step j it pulls the record of item j+1 into L1, so the load at
+// step j+1 is an L1 hit instead of a round trip to L2 on the critical path.
+__device__ __forceinline__ void prefetch_item(const ScoreParams& p, int first, int stride, int j, int J) {
+  if (j + 1 < J) asm volatile("prefetch.global.L1 [%0];" ::"l"(p.item + first + (j + 1) * stride));
+}
+
+// Bounded wait on an mbarrier phase; false if it ran out or another role
+// aborted.  Each try sleeps in hardware for up to kWaitSliceNs, so the abort
+// flag and the time limit are checked at least that often.
+constexpr uint32_t kWaitSliceNs = 20000;
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, const ScoreParams& p) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
-  uint32_t spins = 0;
-  while (!mbar_try_wait(bar, parity)) {
-    if ((++spins & 63u) == 0) {
-      if (ld_volatile(p.abort_flag)) return false;
-      if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
-        atomicExch(p.abort_flag, 1);
-        atomicOr(p.status, kStatusTimeout);
-        return false;
-      }
+  while (!mbar_try_wait_sleep(bar, parity, kWaitSliceNs)) {
+    if (ld_volatile(p.abort_flag)) return false;
+    if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
+      atomicExch(p.abort_flag, 1);
+      atomicOr(p.status, kStatusTimeout);
+      return false;
     }
   }
   return true;
+}
+
+// wait_bar by every lane of a warp; the warp agrees on the outcome (all lanes
+// see the same phase eventually, but a time-out may hit only some of them).
+__device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity, const ScoreParams& p) {
+  return __all_sync(0xffffffffu, wait_bar(bar, parity, p));
 }
 
 // Bounded wait used while shutting down: ignores the abort flag, gives up after
 // `ns` nanoseconds (asynchronous copies and MMAs finish on their own).
 __device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, uint64_t ns) {
   const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait(bar, parity))
+  while (!mbar_try_wait_sleep(bar, parity, kWaitSliceNs))
     if (globaltimer_ns() - t0 > ns) return;
 }
 
@@ -139,17 +152,19 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
   const uint32_t qbytes = static_cast<uint32_t>(p.R_pad) * D * 2;
   const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
   const uint64_t drop = policy_evict_first();  // second read: its last use
-  uint32_t tile = 0;
+  uint32_t tile = 0;            // tiles issued (for the drain after an abort)
+  uint32_t pst = 0, pph = 0;    // K stage ring: position and phase of the next tile
   int last_q_item = -1;
   int issued_q0 = 0, issued_q1 = 0;  // Q loads issued into each buffer
   bool ok = true;
   for (int j = 0; j <= J && ok; ++j) {
+    prefetch_item(p, first, stride, j, J);
     for (int sweep = 0; sweep < 2 && ok; ++sweep) {
       const int jj = sweep == 0 ? j : j - 1;
       if (sweep == 0 && j >= J) continue;
       if (sweep == 1 && j == 0) continue;
       const int t = first + jj * stride;
-      const ItemInfo it = item_info(p, t);
+      const ItemInfo it = decode_item(p, t, load_item(p, t));
       const CUtensorMap* kmap = &p.kmap[it.ls];
       if (sweep == 0) {
         const int qb = jj & 1;
@@ -165,8 +180,8 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
       }
       const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
       for (int i = 0; i < it.ntiles; ++i, ++tile) {
-        const uint32_t st = tile % p.stages;
-        const uint32_t ph = (tile / p.stages) & 1;
+        const uint32_t st = pst, ph = pph;
+        if (++pst == static_cast<uint32_t>(p.stages)) { pst = 0; pph ^= 1; }
         if (!wait_bar(&sm.kempty[st], ph ^ 1, p)) { ok = false; break; }
         uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kTileBytes;
         mbar_expect_tx(&sm.kfull[st], kTileBytes);
@@ -192,7 +207,8 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
 }
 
 // ---------------------------------------------------------------------------
-// MMA issuer (one thread): sweep 1 -> S = Q K^T, sweep 2 -> S^T = K Q^T.
+// MMA issuer (one warp; an elected lane issues): sweep 1 -> S = Q K^T,
+// sweep 2 -> S^T = K Q^T.
 // ---------------------------------------------------------------------------
 template <int D>
 __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_base, int first,
@@ -203,58 +219,57 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
   // sweep 2: N = rows of the group (128, or what is left of R_pad in the last group)
   const uint32_t idesc2a = idesc_bf16_f32(128, p.R_pad > 128 ? 128 : p.R_pad);
   const uint32_t idesc2b = idesc_bf16_f32(128, p.R_pad > 128 ? p.R_pad - 128 : 128);
-  const uint32_t qcol_bytes = static_cast<uint32_t>(p.q_rows) * 128;  // one 64-wide column block
-  uint32_t tile = 0, slot = 0;
+  // descriptor steps (address / 16) between the 64-wide column blocks of Q and of a K tile
+  const uint32_t qcol_step = static_cast<uint32_t>(p.q_rows) * 128 / 16;
+  constexpr uint32_t kcol_step = kTileKeys * 128 / 16;
+  uint32_t st = 0, kph = 0;  // K stage ring: position and phase of the next tile
+  uint32_t sl = 0, tph = 0;  // TMEM slot ring: position and phase of the next slot
   bool ok = true;
   for (int j = 0; j <= J && ok; ++j) {
+    prefetch_item(p, first, stride, j, J);
     for (int sweep = 0; sweep < 2 && ok; ++sweep) {
       const int jj = sweep == 0 ? j : j - 1;
       if (sweep == 0 && j >= J) continue;
       if (sweep == 1 && j == 0) continue;
       const int t = first + jj * stride;
-      const ItemInfo it = item_info(p, t);
+      const ItemInfo it = decode_item(p, t, load_item(p, t));
       const int qb = jj & 1;
-      const uint32_t qaddr = smem_u32(sm.qbuf) + qb * sm.qbytes;
-      if (sweep == 0) {
-        if (!wait_bar(&sm.qfull[qb], (jj >> 1) & 1, p)) { ok = false; break; }
-      }
-      for (int i = 0; i < it.ntiles; ++i, ++tile) {
-        const uint32_t st = tile % p.stages;
-        if (!wait_bar(&sm.kfull[st], (tile / p.stages) & 1, p)) { ok = false; break; }
-        const uint32_t kaddr = smem_u32(sm.kbuf) + st * kTileBytes;
+      const uint64_t qdesc0 = sw128_desc(smem_u32(sm.qbuf) + qb * sm.qbytes);
+      if (sweep == 0 && !wait_bar_warp(&sm.qfull[qb], (jj >> 1) & 1, p)) { ok = false; break; }
+      const bool s1 = sweep == 0;
+      const uint32_t astep = s1 ? qcol_step : kcol_step, bstep = s1 ? kcol_step : qcol_step;
+      for (int i = 0; i < it.ntiles; ++i) {
+        if (!wait_bar_warp(&sm.kfull[st], kph, p)) { ok = false; break; }
+        // Descriptors of the tile and of the Q row group, built once: a
+        // descriptor's low field is the address / 16, so the k-step offsets
+        // (all inside shared memory, no carry out of the field) are plain adds.
+        const uint64_t kdesc = sw128_desc(smem_u32(sm.kbuf) + st * kTileBytes);
         // One 128-column TMEM slot per 128-row group of Q: sweep 1 writes
         // S[rows of group h][keys], sweep 2 writes S^T[keys][rows of group h].
-        for (int h = 0; h < nh && ok; ++h, ++slot) {
-          const uint32_t sl = slot % kSlots;
-          if (!wait_bar(&sm.tempty[sl], ((slot / kSlots) & 1) ^ 1, p)) { ok = false; break; }
+        for (int h = 0; h < nh; ++h) {
+          if (!wait_bar_warp(&sm.tempty[sl], tph ^ 1, p)) { ok = false; break; }
           tc_fence_after();
           const uint32_t dcol = tmem_base + sl * kSlotCols;
-          if (sweep == 0) {
+          const uint64_t qdesc = qdesc0 + static_cast<uint64_t>(h * (128 * 128 / 16));
+          const uint32_t idesc = s1 ? idesc1 : (h == 0 ? idesc2a : idesc2b);
+          const uint64_t adesc = s1 ? qdesc : kdesc, bdesc = s1 ? kdesc : qdesc;
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-              const uint32_t koff = (k >> 2) * (kTileKeys * 128) + (k & 3) * 32;
-              const uint32_t qoff = (k >> 2) * qcol_bytes + h * (128 * 128) + (k & 3) * 32;
-              umma_bf16(dcol, sw128_desc(qaddr + qoff), sw128_desc(kaddr + koff), idesc1, k > 0);
-            }
-          } else {
-            const uint32_t idesc2 = h == 0 ? idesc2a : idesc2b;
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-              const uint32_t koff = (k >> 2) * (kTileKeys * 128) + (k & 3) * 32;
-              const uint32_t qoff = (k >> 2) * qcol_bytes + h * (128 * 128) + (k & 3) * 32;
-              umma_bf16(dcol, sw128_desc(kaddr + koff), sw128_desc(qaddr + qoff), idesc2, k > 0);
-            }
+          for (int k = 0; k < D / 16; ++k) {
+            const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
+            umma_bf16_elect(dcol, adesc + a, bdesc + b, idesc, k > 0);
           }
-          umma_commit(&sm.tfull[sl]);
+          umma_commit_elect(&sm.tfull[sl]);
+          if (++sl == kSlots) { sl = 0; tph ^= 1; }
         }
         if (!ok) break;
-        umma_commit(&sm.kempty[st]);
+        umma_commit_elect(&sm.kempty[st]);
+        if (++st == static_cast<uint32_t>(p.stages)) { st = 0; kph ^= 1; }
       }
-      if (ok && sweep == 1) umma_commit(&sm.qempty[qb]);
+      if (ok && sweep == 1) umma_commit_elect(&sm.qempty[qb]);
     }
   }
   // Every MMA issued so far has completed once `done` flips.
-  umma_commit(sm.done);
+  umma_commit_elect(sm.done);
   wait_bar_drain(sm.done, 0, 1000000000ull);
 }
 
@@ -428,7 +443,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   const int bar_id = 1 + wg;
   const int nh = p.R_pad > 128 ? 2 : 1;                // 128-row groups (slots) per tile
   const int half = nh == 2 ? (wg & 1) : 0;             // row group of this warpgroup
-  const uint32_t tmod = nh == 2 ? 2 : 4, tres = nh == 2 ? (wg >> 1) : wg;
+  const uint32_t tmask = nh == 2 ? 1 : 3, tres = nh == 2 ? (wg >> 1) : wg;  // own tiles: (t & tmask) == tres
   const int row = half * 128 + lrow;                   // sweep-1 row of this thread
   const int r0 = half * 128;                           // sweep-2 first row
   const int nch = (nh == 2 ? (half == 0 ? 128 : p.R_pad - 128) : p.R_pad) / 32;
@@ -441,14 +456,15 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   bool ok = true;
 
   for (int j = 0; j <= J; ++j) {
+    prefetch_item(p, first, stride, j, J);
     // ---------------- sweep 1 of item j ----------------
     if (j < J) {
       const int t = first + j * stride;
-      const ItemInfo it = item_info(p, t);
+      const ItemInfo it = decode_item(p, t, load_item(p, t));
       float m = -INFINITY, z = 0.f;
       for (int i = 0; i < it.ntiles; ++i) {
         const uint32_t gt = tile + i;
-        if (gt % tmod != tres) continue;
+        if ((gt & tmask) != tres) continue;
         s1_slot(p, sm, lane_addr, gt * nh + half, ok, row, it.n, it.key0 + i * kTileKeys, m, z);
       }
       tile += it.ntiles;
@@ -507,7 +523,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
     // ---------------- sweep 2 of item j-1 ----------------
     if (j > 0) {
       const int t = first + (j - 1) * stride;
-      const ItemInfo it = item_info(p, t);
+      const ItemInfo it = decode_item(p, t, load_item(p, t));
       if (wtid == 0) {
         int ready = ld_acquire(&p.ready[it.u]);
         if (!ready) {
@@ -535,7 +551,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       float* out = raw_out + static_cast<size_t>(it.u) * p.S_cap;
       for (int i = 0; i < it.ntiles; ++i) {
         const uint32_t gt = tile + i;
-        if (gt % tmod != tres) continue;
+        if ((gt & tmask) != tres) continue;
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
         float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
@@ -589,7 +605,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
   if (warp < 4) {
     regs_dealloc<kRegsControl>();
     if (warp == 0 && (threadIdx.x & 31) == 0) producer<D>(p, sm, first, stride, J);
-    if (warp == 1 && (threadIdx.x & 31) == 0) mma_issuer<D>(p, sm, tmem_base, first, stride, J);
+    if (warp == 1) mma_issuer<D>(p, sm, tmem_base, first, stride, J);  // whole warp
   } else {
     regs_alloc<kRegsSoftmax>();
     softmax_wg(p, sm, tmem_base, (warp - 4) >> 2, first, stride, J);  // warpgroups 0..3
@@ -658,7 +674,13 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     const int excl = carry + (w > 0 ? warp_sums[w - 1] : 0) + x - c;
     if (u < p.n_units) {
       p.chunk_start[u] = excl;
-      for (int q = 0; q < c; ++q) p.item_unit[excl + q] = u;
+      const int n = p.lens[(u % per_layer) / p.H_kv];
+      for (int q = 0; q < c; ++q) {
+        const int key0 = q * p.chunk_keys;
+        const int nk = min(p.chunk_keys, n - key0);
+        const int ntiles = (nk + kTileKeys - 1) / kTileKeys;
+        p.item[excl + q] = make_int4(u, n, key0, ntiles | (c << 16));
+      }
     }
     __syncthreads();
     if (tid == blockDim.x - 1) carry = excl + c;

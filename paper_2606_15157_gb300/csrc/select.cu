@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
   const int per_layer = p.B * p.H_kv;
   const int l = blockIdx.x / per_layer;
   const int rem = blockIdx.x - l * per_layer;
-  const int s = rem / p.H_kv, h = rem - s * p.H_kv;
+  const int s = rem / p.H_kv;
   const LayerDesc ld = p.layer[l];
   const int n = p.lens[s];
   int* cnt = p.out_count + static_cast<size_t>(l) * per_layer + rem;
