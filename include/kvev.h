@@ -228,6 +228,63 @@ KVEV_API int kvev_evict_prefill_noalloc(kvev_plan *plan, const void *const *K,
                                         void *out_V, int32_t *out_idx, int32_t *out_count,
                                         float *h2o_state, int32_t *device_status, void *stream);
 
+/* ---- decode phase ---------------------------------------------------------- */
+
+/* Decode arena: the retained caches kept across generated tokens, in
+ * caller-owned device memory laid out by the plan.  Layer l with a retained
+ * cache (prefill rule other than FULL) holds cap_l slots per (sequence, KV
+ * head): cap_l = b_l for layers with a decode-phase rule (H2O, TOVA,
+ * StreamingLLM) and b_l + growth for append-only layers (decode rule FULL).
+ * Slot (s, h, j) of layer l is row row_offset(l) + (s*H_kv + h)*cap_l + j of
+ * dec_K / dec_V (bf16 [rows][d]).  The state buffer (dec_state, 256-byte
+ * aligned, kvev_decode_state_offsets) holds int32 lens[B] (sequence lengths,
+ * advanced by every step), int32 count[units] (occupied slots), int32
+ * evicted[units] (position evicted by the last step, -1 if none), int32
+ * pos[rows] (position held by a slot, -1 = empty) and fp32 acc[rows] (H2O:
+ * accumulated attention; TOVA: the last step's attention), where unit
+ * unit_offset(l) + s*H_kv + h.  Slot order carries no meaning.
+ * EINVAL when a layer with a FULL prefill rule has a decode-phase rule (its
+ * cache is the caller's own). */
+KVEV_API int kvev_decode_query(const kvev_plan *plan, int B, int growth, int64_t *rows,
+                               size_t *state_bytes);
+KVEV_API int kvev_decode_layer(const kvev_plan *plan, int B, int growth, int layer,
+                               int64_t *row_offset, int *cap, int *unit_offset);
+/* offsets[5] = byte offsets in dec_state of lens, count, evicted, pos, acc. */
+KVEV_API int kvev_decode_state_offsets(const kvev_plan *plan, int B, int growth, size_t *offsets);
+
+/* Fill the arena from the output of kvev_evict_prefill() (same plan and B):
+ * slot j < out_count of each unit takes packed row j (its K/V rows, its
+ * position, and for H2O prefill layers its h2o_state score as the initial
+ * acc, 0 elsewhere or when h2o_state is NULL); other slots are marked empty;
+ * lens is copied from lens_dev.  Asynchronous on `stream`.  EINVAL on null or
+ * misaligned pointers (rows 16-byte, state 256-byte). */
+KVEV_API int kvev_decode_init(kvev_plan *plan, int B, int growth, const void *pre_K,
+                              const void *pre_V, const int32_t *pre_idx, const int32_t *pre_count,
+                              const float *h2o_state, const int32_t *lens_dev, void *dec_K,
+                              void *dec_V, void *dec_state, void *stream);
+
+/* One decode step (Sec. 2.1's cited rules in their decode phase; the new
+ * token sits at position lens[s] and lens advances by one):
+ *   k_new[L], v_new[L]  host arrays of device pointers, bf16 [B][H_kv][d]
+ *                       (NULL for layers without an arena);
+ *   q_new[L]            bf16 [B][H_q][d], the new token's queries (needed for
+ *                       H2O and TOVA layers only).
+ *   H2O:  p_j = (1/G) sum over the group's query heads of
+ *         softmax_j(q . k_j / sqrt(d)) over the retained slots and the new
+ *         token; acc += p; once b slots are held, the slot with the smallest
+ *         acc among positions < lens+1-r (r = h2o_recent, or floor(b/2)) is
+ *         evicted (ties: the higher position) and the new token takes it.
+ *   TOVA: the same with acc = p (no accumulation) and r = 0, so the new token
+ *         itself may be the one evicted.
+ *   StreamingLLM: once sink + recent slots are held, the smallest position
+ *         >= sink is evicted.
+ *   FULL: append (count must stay <= cap, else the device status records an
+ *         error).
+ * Asynchronous; ENOTSUP if d is not 64/128 or G not 1, 2, 4 or 8. */
+KVEV_API int kvev_decode_step(kvev_plan *plan, int B, int growth, void *dec_K, void *dec_V,
+                              void *dec_state, const void *const *k_new, const void *const *v_new,
+                              const void *const *q_new, void *stream);
+
 /* ---- measurement ---------------------------------------------------------- */
 
 /* Kernels of one kvev_evict_prefill() call, in launch order. */

@@ -664,6 +664,222 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
 }  // namespace
 
 // ---------------------------------------------------------------------------
+// Decode phase
+// ---------------------------------------------------------------------------
+
+namespace {
+
+struct DecLayout {
+  int units = 0;
+  int64_t rows = 0;
+  size_t lens = 0, count = 0, evicted = 0, pos = 0, acc = 0, total = 0;
+  std::vector<int> cap, unit_off;
+  std::vector<int64_t> row_off;
+};
+
+// Arena layout for B sequences; growth = extra slots of append-only layers.
+// Returns KVEV_EINVAL for a layer that has a decode-phase rule but no
+// retained rows (a FULL prefill layer keeps the caller's own cache).
+int dec_layout(const kvev_plan& P, int B, int growth, DecLayout& d) {
+  if (B < 0 || growth < 0) return KVEV_EINVAL;
+  d.cap.assign(P.L, 0);
+  d.unit_off.assign(P.L, 0);
+  d.row_off.assign(P.L, 0);
+  for (int l = 0; l < P.L; ++l) {
+    const int md = P.route_dec[l];
+    d.unit_off[l] = d.units;
+    d.row_off[l] = d.rows;
+    if (P.slots[l] == 0) {
+      if (md != KVEV_FULL) return KVEV_EINVAL;
+      continue;
+    }
+    d.cap[l] = P.slots[l] + (md == KVEV_FULL ? growth : 0);
+    d.units += B * P.H_kv;
+    d.rows += static_cast<int64_t>(B) * P.H_kv * d.cap[l];
+  }
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, kWsAlign);
+    return o;
+  };
+  d.lens = take(sizeof(int32_t) * std::max(B, 1));
+  d.count = take(sizeof(int32_t) * std::max(d.units, 1));
+  d.evicted = take(sizeof(int32_t) * std::max(d.units, 1));
+  d.pos = take(sizeof(int32_t) * std::max<int64_t>(d.rows, 1));
+  d.acc = take(sizeof(float) * std::max<int64_t>(d.rows, 1));
+  d.total = off;
+  return KVEV_OK;
+}
+
+int dec_params(const kvev_plan& P, int B, const DecLayout& d, DecodeParams& dp) {
+  std::memset(&dp, 0, sizeof(dp));
+  dp.L = P.L;
+  dp.B = B;
+  dp.H_kv = P.H_kv;
+  dp.H_q = P.H_q;
+  dp.G = P.G;
+  dp.d = P.d;
+  dp.units = d.units;
+  dp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));
+  int64_t pre_off = 0;
+  for (int l = 0; l < P.L; ++l) {
+    DecLayer& y = dp.layer[l];
+    const int md = P.route_dec[l], b = P.budget[l];
+    y.method = md;
+    y.b = b;
+    y.cap = d.cap[l];
+    y.unit_off = d.unit_off[l];
+    y.row_off = d.row_off[l];
+    y.pre_method = P.route_pre[l];
+    y.pre_slots = P.slots[l];
+    y.pre_row_off = pre_off;
+    pre_off += rows_per_layer(P, B, l);
+    if (y.cap == 0) continue;
+    if (md == KVEV_H2O || md == KVEV_TOVA) {
+      y.r = md == KVEV_TOVA ? 0 : (P.h2o_recent < 0 ? b / 2 : P.h2o_recent);
+      if (b < 1 || y.r >= b) return KVEV_EINVAL;  // at least one slot must be evictable
+    } else if (md == KVEV_STREAMING) {
+      if (P.sink < 0 || b <= P.sink) return KVEV_EINVAL;
+      y.sink = P.sink;
+      y.recent = P.recent < 0 ? b - P.sink : std::min(P.recent, b - P.sink);
+    }
+  }
+  return KVEV_OK;
+}
+
+// Shared memory of the step kernel: the logits of the largest H2O/TOVA unit.
+size_t dec_smem(const kvev_plan& P, const DecLayout& d) {
+  int cap = 0;
+  for (int l = 0; l < P.L; ++l)
+    if (d.cap[l] > 0 && (P.route_dec[l] == KVEV_H2O || P.route_dec[l] == KVEV_TOVA))
+      cap = std::max(cap, d.cap[l]);
+  return cap == 0 ? 0 : sizeof(float) * static_cast<size_t>(P.G) * (cap + 1);
+}
+
+void set_state_ptrs(DecodeParams& dp, const DecLayout& d, void* dec_K, void* dec_V, void* state) {
+  uint8_t* sb = static_cast<uint8_t*>(state);
+  dp.K = dec_K;
+  dp.V = dec_V;
+  dp.lens = reinterpret_cast<int32_t*>(sb + d.lens);
+  dp.count = reinterpret_cast<int32_t*>(sb + d.count);
+  dp.evicted = reinterpret_cast<int32_t*>(sb + d.evicted);
+  dp.pos = reinterpret_cast<int32_t*>(sb + d.pos);
+  dp.acc = reinterpret_cast<float*>(sb + d.acc);
+}
+
+}  // namespace
+
+extern "C" int kvev_decode_query(const kvev_plan* plan, int B, int growth, int64_t* rows,
+                                 size_t* state_bytes) {
+  if (!plan) return KVEV_EINVAL;
+  DecLayout d;
+  const int rc = dec_layout(*plan, B, growth, d);
+  if (rc != KVEV_OK) return rc;
+  if (rows) *rows = d.rows;
+  if (state_bytes) *state_bytes = d.total;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_decode_layer(const kvev_plan* plan, int B, int growth, int layer,
+                                 int64_t* row_offset, int* cap, int* unit_offset) {
+  if (!plan || layer < 0 || layer >= plan->L) return KVEV_EINVAL;
+  DecLayout d;
+  const int rc = dec_layout(*plan, B, growth, d);
+  if (rc != KVEV_OK) return rc;
+  if (row_offset) *row_offset = d.row_off[layer];
+  if (cap) *cap = d.cap[layer];
+  if (unit_offset) *unit_offset = d.unit_off[layer];
+  return KVEV_OK;
+}
+
+extern "C" int kvev_decode_state_offsets(const kvev_plan* plan, int B, int growth, size_t* offsets) {
+  if (!plan || !offsets) return KVEV_EINVAL;
+  DecLayout d;
+  const int rc = dec_layout(*plan, B, growth, d);
+  if (rc != KVEV_OK) return rc;
+  offsets[0] = d.lens;
+  offsets[1] = d.count;
+  offsets[2] = d.evicted;
+  offsets[3] = d.pos;
+  offsets[4] = d.acc;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_decode_init(kvev_plan* plan, int B, int growth, const void* pre_K,
+                                const void* pre_V, const int32_t* pre_idx,
+                                const int32_t* pre_count, const float* h2o_state,
+                                const int32_t* lens_dev, void* dec_K, void* dec_V, void* dec_state,
+                                void* stream) {
+  if (!plan || B < 0) return KVEV_EINVAL;
+  kvev_plan& P = *plan;
+  DecLayout d;
+  int rc = dec_layout(P, B, growth, d);
+  if (rc != KVEV_OK) return rc;
+  if (B == 0 || d.units == 0) return KVEV_OK;
+  if (!pre_K || !pre_V || !pre_idx || !pre_count || !lens_dev || !dec_K || !dec_V || !dec_state)
+    return KVEV_EINVAL;
+  if (!aligned16(pre_K) || !aligned16(pre_V) || !aligned16(dec_K) || !aligned16(dec_V) ||
+      (reinterpret_cast<uintptr_t>(dec_state) & 255u))
+    return KVEV_EINVAL;
+  DecodeParams dp;
+  rc = dec_params(P, B, d, dp);
+  if (rc != KVEV_OK) return rc;
+  rc = ensure_device(plan);
+  if (rc != KVEV_OK) return rc;
+  set_state_ptrs(dp, d, dec_K, dec_V, dec_state);
+  dp.status = P.ctx.status;
+  dp.pre_K = pre_K;
+  dp.pre_V = pre_V;
+  dp.pre_idx = pre_idx;
+  dp.pre_count = pre_count;
+  dp.h2o_state = h2o_state;
+  dp.lens_in = lens_dev;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P.last_stream = s;
+  return launch_decode_init(dp, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
+}
+
+extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_V,
+                                void* dec_state, const void* const* k_new,
+                                const void* const* v_new, const void* const* q_new,
+                                void* stream) {
+  if (!plan || B < 0) return KVEV_EINVAL;
+  kvev_plan& P = *plan;
+  DecLayout d;
+  int rc = dec_layout(P, B, growth, d);
+  if (rc != KVEV_OK) return rc;
+  if (B == 0) return KVEV_OK;
+  if (!dec_state || (reinterpret_cast<uintptr_t>(dec_state) & 255u)) return KVEV_EINVAL;
+  if (d.units > 0) {
+    if (!dec_K || !dec_V || !k_new || !v_new || !q_new || !aligned16(dec_K) || !aligned16(dec_V))
+      return KVEV_EINVAL;
+    if (!decode_supported(P.d, P.G)) return KVEV_ENOTSUP;
+  }
+  DecodeParams dp;
+  rc = dec_params(P, B, d, dp);
+  if (rc != KVEV_OK) return rc;
+  for (int l = 0; l < P.L; ++l) {
+    if (d.cap[l] == 0) continue;
+    if (!k_new[l] || !v_new[l] || !aligned16(k_new[l]) || !aligned16(v_new[l])) return KVEV_EINVAL;
+    const bool attends = P.route_dec[l] == KVEV_H2O || P.route_dec[l] == KVEV_TOVA;
+    if (attends && (!q_new[l] || !aligned16(q_new[l]))) return KVEV_EINVAL;
+    dp.k_new[l] = k_new[l];
+    dp.v_new[l] = v_new[l];
+    dp.q_new[l] = q_new[l];
+  }
+  rc = ensure_device(plan);
+  if (rc != KVEV_OK) return rc;
+  const size_t smem = dec_smem(P, d);
+  if (smem + 1024 > static_cast<size_t>(P.ctx.smem_optin)) return KVEV_ENOTSUP;
+  set_state_ptrs(dp, d, dec_K, dec_V, dec_state);
+  dp.status = P.ctx.status;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P.last_stream = s;
+  return launch_decode_step(dp, smem, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
+}
+
+// ---------------------------------------------------------------------------
 // Prefill eviction without allocation: the workspace is a file-scope device
 // array instead of caller memory.  Its name is only a host-side stand-in, so
 // host code obtains the array's device address per device with

@@ -1,0 +1,392 @@
+// decode.cu -- decode-phase update of the retained caches, one generated token
+// per call, for every layer of a route in one launch (the decode step of the
+// rules Sec. 2.1 cites: H2O accumulates the new token's attention, TOVA keeps
+// only the current step's attention, StreamingLLM keeps sinks + a rolling
+// window, and a layer without a decode-phase rule appends).
+//
+// Decode arena (caller-owned device memory, layout from the plan): layer l
+// holds B*H_kv*cap_l slots, slot (s, h, j) at row row_off(l) + (s*H_kv + h) *
+// cap_l + j of dec_K / dec_V.  The state buffer holds lens[B], and per unit u
+// = unit_off(l) + s*H_kv + h: count[u], evicted[u], and per slot pos (the
+// position it holds, -1 = empty) and acc (H2O: accumulated attention; TOVA:
+// the last step's attention).  Slot order carries no meaning: an evicted
+// slot is overwritten by the new token.
+//
+// One CTA per unit.  H2O / TOVA: the G query rows of the new token attend to
+// every retained slot and to the new token, p_j = (1/G) sum_g softmax_j(q_g .
+// k_j / sqrt(d)); acc += p (H2O) or acc = p (TOVA).  When the unit already
+// holds b slots, the slot with the smallest acc among positions older than
+// the protected recent window (r = h2o_recent for H2O, 0 for TOVA) is
+// evicted, ties to the higher position, and the new token takes its place
+// (unless the new token itself is the one evicted).  The retained K rows are
+// streamed once (16-byte loads, d/8 lanes per row); logits stay in shared
+// memory.
+#include "kvev_internal.cuh"
+
+namespace kvev {
+
+namespace {
+
+constexpr int kDecodeThreads = 256;
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// Unit index -> layer: the last layer whose first unit is <= u (layers
+// without slots own no units and share their unit_off with the next layer).
+__device__ __forceinline__ int find_dec_layer(const DecodeParams& p, int u) {
+  int lo = 0, hi = p.L - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.layer[mid].unit_off <= u) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+struct DecShared {
+  float f[kDecodeThreads / 32];
+  int i[2 * (kDecodeThreads / 32)];
+};
+
+__device__ __forceinline__ float block_max(float v, DecShared& sh) {
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float r = sh.f[0];
+  for (int i = 1; i < kDecodeThreads / 32; ++i) r = fmaxf(r, sh.f[i]);
+  return r;
+}
+
+__device__ __forceinline__ float block_sum(float v, DecShared& sh) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float r = 0.f;
+  for (int i = 0; i < kDecodeThreads / 32; ++i) r += sh.f[i];
+  return r;
+}
+
+// Eviction order: smaller key first, then higher position first.
+__device__ __forceinline__ bool evict_before(float a, int pa, float b, int pb) {
+  return a < b || (a == b && pa > pb);
+}
+
+// Block-wide first candidate in eviction order (candidates have pos >= 0);
+// returns its slot, -1 if there is none.
+__device__ __forceinline__ int block_evict_choice(float a, int pos, int slot, DecShared& sh) {
+  for (int o = 16; o > 0; o >>= 1) {
+    const float a2 = __shfl_xor_sync(0xffffffffu, a, o);
+    const int p2 = __shfl_xor_sync(0xffffffffu, pos, o);
+    const int s2 = __shfl_xor_sync(0xffffffffu, slot, o);
+    if (p2 >= 0 && (pos < 0 || evict_before(a2, p2, a, pos))) {
+      a = a2;
+      pos = p2;
+      slot = s2;
+    }
+  }
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) {
+    const int w = threadIdx.x >> 5;
+    sh.f[w] = a;
+    sh.i[2 * w] = pos;
+    sh.i[2 * w + 1] = slot;
+  }
+  __syncthreads();
+  float ba = sh.f[0];
+  int bp = sh.i[0], bs = sh.i[1];
+  for (int i = 1; i < kDecodeThreads / 32; ++i) {
+    const int pi = sh.i[2 * i];
+    if (pi >= 0 && (bp < 0 || evict_before(sh.f[i], pi, ba, bp))) {
+      ba = sh.f[i];
+      bp = pi;
+      bs = sh.i[2 * i + 1];
+    }
+  }
+  return bp < 0 ? -1 : bs;
+}
+
+// Copy one d-wide bf16 row (16-byte vectors) with the whole block.
+__device__ __forceinline__ void copy_row(uint16_t* dst, const uint16_t* src, int d) {
+  for (int i = threadIdx.x; i < d / 8; i += blockDim.x)
+    reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+}
+
+struct UnitRef {
+  int l, s, h, u;
+  size_t rows0;  // first slot row of the unit
+};
+
+// Put the new token into slot dst (its K/V row, position n, key acc_new) and
+// finish the unit's bookkeeping.  Called by the whole block.
+__device__ __forceinline__ void place_new(const DecodeParams& p, const UnitRef& r, int D, int dst, int n,
+                                          float acc_new, int new_count, int evicted_pos) {
+  if (dst >= 0) {
+    const size_t src = static_cast<size_t>(r.s) * p.H_kv + r.h;
+    copy_row(static_cast<uint16_t*>(p.K) + (r.rows0 + dst) * D,
+             static_cast<const uint16_t*>(p.k_new[r.l]) + src * D, D);
+    copy_row(static_cast<uint16_t*>(p.V) + (r.rows0 + dst) * D,
+             static_cast<const uint16_t*>(p.v_new[r.l]) + src * D, D);
+  }
+  if (threadIdx.x == 0) {
+    if (dst >= 0) {
+      p.pos[r.rows0 + dst] = n;
+      p.acc[r.rows0 + dst] = acc_new;
+    }
+    p.count[r.u] = new_count;
+    p.evicted[r.u] = evicted_pos;
+  }
+}
+
+// H2O / TOVA unit.  lg: [G][cap + 1] floats of shared memory.
+template <int D, int G>
+__device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int n, int c,
+                            float* lg, DecShared& sh) {
+  constexpr int LPS = D / 8;     // lanes per slot row (16 bytes each)
+  constexpr int SPW = 32 / LPS;  // slot rows per warp per pass
+  constexpr int SPB = SPW * (kDecodeThreads / 32);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int sub = lane % LPS, grp = lane / LPS;
+  const int ld = ly.cap + 1;  // row stride of lg
+  const uint16_t* Kb = static_cast<const uint16_t*>(p.K) + r.rows0 * D;
+  const uint16_t* qn =
+      static_cast<const uint16_t*>(p.q_new[r.l]) + (static_cast<size_t>(r.s) * p.H_q + r.h * G) * D;
+  const uint16_t* kn = static_cast<const uint16_t*>(p.k_new[r.l]) + (static_cast<size_t>(r.s) * p.H_kv + r.h) * D;
+
+  // this lane's 8 elements of each query row, scaled into the exp2 domain
+  float q[G][8];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const uint4 v = *reinterpret_cast<const uint4*>(qn + g * D + sub * 8);
+    const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      q[g][2 * e] = bf16_lo(w4[e]) * p.scale_log2;
+      q[g][2 * e + 1] = bf16_hi(w4[e]) * p.scale_log2;
+    }
+  }
+  // logits (base 2) of slots 0..c-1 and of the new token at index c
+  const int cnt = c + 1;
+  for (int j0 = 0; j0 < cnt; j0 += SPB) {
+    const int j = j0 + warp * SPW + grp;
+    uint4 kv = make_uint4(0, 0, 0, 0);
+    if (j < c) kv = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j) * D + sub * 8));
+    else if (j == c) kv = *reinterpret_cast<const uint4*>(kn + sub * 8);
+    const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
+    float kf[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      kf[2 * e] = bf16_lo(w4[e]);
+      kf[2 * e + 1] = bf16_hi(w4[e]);
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float a = 0.f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) a = fmaf(q[g][e], kf[e], a);
+#pragma unroll
+      for (int o = LPS / 2; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+      if (sub == 0 && j < cnt) lg[g * ld + j] = a;
+    }
+  }
+  __syncthreads();
+  // per-head softmax statistics
+  float mg[G], zg[G];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float m = -INFINITY;
+    for (int j = threadIdx.x; j < cnt; j += blockDim.x) m = fmaxf(m, lg[g * ld + j]);
+    mg[g] = block_max(m, sh);
+    float z = 0.f;
+    for (int j = threadIdx.x; j < cnt; j += blockDim.x) z += exp2f(lg[g * ld + j] - mg[g]);
+    zg[g] = block_sum(z, sh);
+  }
+  // group-mean attention -> new keys (each thread overwrites row 0 at its own j only)
+  const float* accr = p.acc + r.rows0;
+  const int32_t* posr = p.pos + r.rows0;
+  const int limit = n + 1 - ly.r;  // positions >= limit are protected
+  float ba = INFINITY;
+  int bp = -1, bs = -1;
+  for (int j = threadIdx.x; j < cnt; j += blockDim.x) {
+    float pj = 0.f;
+#pragma unroll
+    for (int g = 0; g < G; ++g) pj += exp2f(lg[g * ld + j] - mg[g]) / zg[g];
+    pj *= 1.0f / static_cast<float>(G);
+    const float a = (ly.method == KVEV_H2O && j < c) ? accr[j] + pj : pj;
+    lg[j] = a;
+    const int pos = j < c ? posr[j] : n;
+    if (pos >= 0 && pos < limit && (bp < 0 || evict_before(a, pos, ba, bp))) {
+      ba = a;
+      bp = pos;
+      bs = j;
+    }
+  }
+  const bool full = c >= ly.b;
+  const int ev = full ? block_evict_choice(ba, bp, bs, sh) : -1;  // c = the new token
+  __syncthreads();
+  const int evicted_pos = ev < 0 ? -1 : (ev < c ? posr[ev] : n);
+  __syncthreads();  // every thread has read posr[ev] before it is overwritten
+  for (int j = threadIdx.x; j < c; j += blockDim.x)
+    if (j != ev) p.acc[r.rows0 + j] = lg[j];
+  if (!full) {
+    if (c >= ly.cap) {  // never for a consistent state: slots of an evicting layer stay <= b
+      if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+      return;
+    }
+    place_new(p, r, D, c, n, lg[c], c + 1, -1);
+  } else if (ev < 0) {  // no evictable slot (protected window covers the cache)
+    if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+  } else {
+    place_new(p, r, D, ev < c ? ev : -1, n, lg[c], c, evicted_pos);
+  }
+}
+
+// StreamingLLM unit: the oldest non-sink slot makes room once sink + recent
+// slots are held; positions are read from the state, no attention.
+__device__ void stream_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int D, int n, int c,
+                            DecShared& sh) {
+  const int capacity = ly.sink + ly.recent;
+  if (c + 1 <= capacity) {
+    if (c >= ly.cap) {
+      if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+      return;
+    }
+    place_new(p, r, D, c, n, 0.f, c + 1, -1);
+    return;
+  }
+  // smallest position >= sink among the slots and the new token (eviction key = position)
+  float ba = INFINITY;
+  int bp = -1, bs = -1;
+  for (int j = threadIdx.x; j <= c; j += blockDim.x) {
+    const int pos = j < c ? p.pos[r.rows0 + j] : n;
+    const float key = static_cast<float>(pos);  // exact: positions < 2^24
+    if (pos >= ly.sink && (bp < 0 || key < ba)) {
+      ba = key;
+      bp = pos;
+      bs = j;
+    }
+  }
+  // positions are distinct, so "smallest key" decides alone
+  const int ev = block_evict_choice(ba, bp, bs, sh);
+  __syncthreads();
+  const int evicted_pos = ev < 0 ? -1 : (ev < c ? p.pos[r.rows0 + ev] : n);
+  __syncthreads();
+  if (ev < 0) {
+    if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+    return;
+  }
+  place_new(p, r, D, ev < c ? ev : -1, n, 0.f, c, evicted_pos);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kDecodeThreads) decode_step_kernel(const __grid_constant__ DecodeParams p) {
+  extern __shared__ float lg[];
+  __shared__ DecShared sh;
+  const int u = blockIdx.x;
+  const int l = find_dec_layer(p, u);
+  const DecLayer& ly = p.layer[l];
+  const int rem = u - ly.unit_off;
+  UnitRef r;
+  r.l = l;
+  r.s = rem / p.H_kv;
+  r.h = rem - r.s * p.H_kv;
+  r.u = u;
+  r.rows0 = static_cast<size_t>(ly.row_off) + static_cast<size_t>(rem) * ly.cap;
+  const int n = p.lens[r.s];
+  const int c = p.count[u];
+  if (c < 0 || c > ly.cap) {
+    if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+    return;
+  }
+  if (ly.method == KVEV_H2O || ly.method == KVEV_TOVA) attend_unit<D, G>(p, ly, r, n, c, lg, sh);
+  else if (ly.method == KVEV_STREAMING) stream_unit(p, ly, r, D, n, c, sh);
+  else if (c < ly.cap) place_new(p, r, D, c, n, 0.f, c + 1, -1);  // append only
+  else if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+}
+
+// After every unit of the step: the sequences are one token longer.
+__global__ void decode_advance_kernel(int32_t* lens, int B) {
+  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < B; s += gridDim.x * blockDim.x) lens[s] += 1;
+}
+
+// Decode arena from the packed prefill output: slot j < kept count of unit
+// (l, s, h) takes prefill row j (its position and, for H2O prefill layers,
+// its score as the initial acc); the remaining slots are marked empty.
+__global__ void __launch_bounds__(kDecodeThreads) decode_init_kernel(const __grid_constant__ DecodeParams p) {
+  const int u = blockIdx.x;
+  const int l = find_dec_layer(p, u);
+  const DecLayer& ly = p.layer[l];
+  const int rem = u - ly.unit_off;
+  const size_t rows0 = static_cast<size_t>(ly.row_off) + static_cast<size_t>(rem) * ly.cap;
+  const size_t pre0 = static_cast<size_t>(ly.pre_row_off) + static_cast<size_t>(rem) * ly.pre_slots;
+  int c = p.pre_count[static_cast<size_t>(l) * p.B * p.H_kv + rem];
+  if (c < 0 || c > ly.pre_slots) {
+    if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+    c = 0;
+  }
+  const int vec = p.d / 8;  // 16-byte vectors per row
+  for (int i = threadIdx.x; i < c * vec; i += blockDim.x) {
+    const int j = i / vec, e = i - j * vec;
+    reinterpret_cast<uint4*>(p.K)[(rows0 + j) * vec + e] = reinterpret_cast<const uint4*>(p.pre_K)[(pre0 + j) * vec + e];
+    reinterpret_cast<uint4*>(p.V)[(rows0 + j) * vec + e] = reinterpret_cast<const uint4*>(p.pre_V)[(pre0 + j) * vec + e];
+  }
+  const bool seed_acc = ly.pre_method == KVEV_H2O && p.h2o_state != nullptr;
+  for (int j = threadIdx.x; j < ly.cap; j += blockDim.x) {
+    p.pos[rows0 + j] = j < c ? p.pre_idx[pre0 + j] : -1;
+    p.acc[rows0 + j] = (j < c && seed_acc) ? p.h2o_state[pre0 + j] : 0.f;
+  }
+  if (threadIdx.x == 0) {
+    p.count[u] = c;
+    p.evicted[u] = -1;
+  }
+  if (u == 0)  // the first unit also copies the sequence lengths
+    for (int i = threadIdx.x; i < p.B; i += blockDim.x) p.lens[i] = p.lens_in[i];
+}
+
+template <int D, int G>
+cudaError_t launch_step_dg(const DecodeParams& p, size_t smem, cudaStream_t st) {
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(decode_step_kernel<D, G>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  decode_step_kernel<D, G><<<p.units, kDecodeThreads, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_step_d(const DecodeParams& p, size_t smem, cudaStream_t st) {
+  switch (p.G) {
+    case 1: return launch_step_dg<D, 1>(p, smem, st);
+    case 2: return launch_step_dg<D, 2>(p, smem, st);
+    case 4: return launch_step_dg<D, 4>(p, smem, st);
+    case 8: return launch_step_dg<D, 8>(p, smem, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+bool decode_supported(int d, int G) {
+  return (d == 64 || d == 128) && (G == 1 || G == 2 || G == 4 || G == 8);
+}
+
+cudaError_t launch_decode_init(const DecodeParams& p, cudaStream_t st) {
+  if (p.units == 0) return cudaSuccess;
+  decode_init_kernel<<<p.units, kDecodeThreads, 0, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_step(const DecodeParams& p, size_t smem, cudaStream_t st) {
+  if (p.units > 0) {
+    const cudaError_t e = p.d == 64 ? launch_step_d<64>(p, smem, st) : launch_step_d<128>(p, smem, st);
+    if (e != cudaSuccess) return e;
+  }
+  decode_advance_kernel<<<1, 256, 0, st>>>(p.lens, p.B);
+  return cudaGetLastError();
+}
+
+}  // namespace kvev

@@ -99,6 +99,44 @@ struct SelectParams {
   int* out_count;     // [L][B][H_kv]
 };
 
+// Per-layer description of the decode arena.
+struct DecLayer {
+  int method;         // decode-phase operator (KVEV_*); FULL = append only
+  int b;              // budget: slots kept by an evicting layer
+  int cap;            // slots per unit in the arena (0: the layer has no arena)
+  int r;              // H2O / TOVA protected recent window
+  int sink, recent;   // StreamingLLM
+  int pre_method;     // prefill operator (its packed rows seed the arena)
+  int pre_slots;      // prefill slots per unit (b_l)
+  int unit_off;       // first unit of the layer
+  long long row_off;  // first arena slot row of the layer
+  long long pre_row_off;  // first packed prefill row of the layer
+};
+
+struct DecodeParams {
+  DecLayer layer[kMaxLayers];
+  const void* k_new[kMaxLayers];  // [B][H_kv][d] bf16 per layer
+  const void* v_new[kMaxLayers];  // [B][H_kv][d]
+  const void* q_new[kMaxLayers];  // [B][H_q][d]
+  int L, B, H_kv, H_q, G, d, units;
+  float scale_log2;   // log2(e) / sqrt(d)
+  void* K;            // arena rows [rows][d] bf16
+  void* V;
+  int32_t* pos;       // [rows]
+  float* acc;         // [rows]
+  int32_t* count;     // [units]
+  int32_t* evicted;   // [units]: position evicted by the last step, -1 = none
+  int32_t* lens;      // [B]
+  int* status;
+  // initialisation from the packed prefill output
+  const void* pre_K;
+  const void* pre_V;
+  const int32_t* pre_idx;
+  const int32_t* pre_count;  // [L][B][H_kv]
+  const float* h2o_state;    // nullable
+  const int32_t* lens_in;    // [B]
+};
+
 struct GatherParams {
   LayerDesc layer[kMaxLayers];
   const void* K[kMaxLayers];
@@ -448,6 +486,9 @@ namespace kvev {
 cudaError_t launch_prologue(const PrologueParams& p, cudaStream_t s);
 cudaError_t launch_score(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
 int score_smem_bytes(int d, int q_rows, int R_pad, int stages);
+bool decode_supported(int d, int G);
+cudaError_t launch_decode_init(const DecodeParams& p, cudaStream_t s);
+cudaError_t launch_decode_step(const DecodeParams& p, size_t smem, cudaStream_t s);
 int score_kernel_regs(int d);
 cudaError_t score_set_smem(int d, size_t smem);
 cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s);

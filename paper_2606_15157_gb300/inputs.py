@@ -270,6 +270,22 @@ def config_decode(seed: int = 0, B: int = 16, n0: int = 16384, steps: int = 256,
         sink_tokens=4, sink_scale=4.0, route_decode=dec, decode_steps=steps)
 
 
+def config_decode_mixed(seed: int = 0, steps: int = 24, d: int = 128) -> Workload:
+    """Every decode-phase rule at a size the oracle replays step by step: 8 layers,
+    GQA 8/2 heads, batch 2 with ragged lengths, W=16.  Prefill -> decode rules:
+    SnapKV->append, H2O->H2O, StreamingLLM->StreamingLLM, H2O->TOVA, SnapKV->TOVA,
+    StreamingLLM->append, H2O (budget above the length: identity prefill, the
+    decode cache fills up to b first)->H2O, SnapKV->H2O (acc starts at 0)."""
+    route = np.array([SNAPKV, H2O, STREAMING, H2O, SNAPKV, STREAMING, H2O, SNAPKV], np.int32)
+    dec = np.array([FULL, H2O, STREAMING, TOVA, TOVA, FULL, H2O, H2O], np.int32)
+    budget = np.array([256, 192, 128, 160, 200, 96, 3000, 144], np.int32)
+    return Workload(
+        name=f"decode_mixed_d{d}", L=8, H_q=8, H_kv=2, d=d, B=2,
+        lens=np.array([2990, 2731], np.int32), S_cap=3072, W=16, pool_kernel=7,
+        pool_type=POOL_AVG, route=route, budget=budget, sink=4, seed=seed, sink_tokens=4,
+        sink_scale=4.0, route_decode=dec, decode_steps=steps)
+
+
 # --------------------------------------------------------------------------
 # Host tensor generation (small and sampled cases)
 # --------------------------------------------------------------------------

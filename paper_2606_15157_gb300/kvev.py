@@ -28,7 +28,9 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_destroy", "kvev_plan_query", "kvev_plan_layer_offset",
            "kvev_evict_prefill", "kvev_status", "kvev_plan_set_wait_limit",
            "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
-           "kvev_plan_last_timings", "kvev_evict_prefill_noalloc"]
+           "kvev_plan_last_timings", "kvev_evict_prefill_noalloc", "kvev_decode_query",
+           "kvev_decode_layer", "kvev_decode_state_offsets", "kvev_decode_init",
+           "kvev_decode_step"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
 
 
@@ -71,6 +73,12 @@ def load(path: str = LIB_PATH):
         L.kvev_evict_prefill_noalloc.argtypes = [vp, vp, vp, vp, vp, C.c_int, C.c_int, vp, vp,
                                                  vp, vp, vp, vp, vp]
         L.kvev_plan_last_timings.argtypes = [vp, vp, C.c_int]
+        L.kvev_decode_query.argtypes = [vp, C.c_int, C.c_int, P(i64), P(sz)]
+        L.kvev_decode_layer.argtypes = [vp, C.c_int, C.c_int, C.c_int, P(i64), P(C.c_int),
+                                        P(C.c_int)]
+        L.kvev_decode_state_offsets.argtypes = [vp, C.c_int, C.c_int, P(sz)]
+        L.kvev_decode_init.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+        L.kvev_decode_step.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
         for name in EXPORTS:
             if name != "kvev_plan_destroy":
                 getattr(L, name).restype = C.c_int
@@ -161,6 +169,41 @@ def kvev_evict_prefill_noalloc(handle, K_ptrs, V_ptrs, Q_ptrs, lens_ptr, B, S_ca
     Qa = arr(*Q_ptrs) if Q_ptrs is not None else None
     return load().kvev_evict_prefill_noalloc(handle, Ka, Va, Qa, lens_ptr, B, S_cap, out_K, out_V,
                                              out_idx, out_count, h2o_state, device_status, stream)
+
+
+def kvev_decode_query(handle: int, B: int, growth: int):
+    rows, state = C.c_int64(), C.c_size_t()
+    _check(load().kvev_decode_query(handle, B, growth, C.byref(rows), C.byref(state)),
+           "kvev_decode_query")
+    return rows.value, state.value
+
+
+def kvev_decode_layer(handle: int, B: int, growth: int, layer: int):
+    """(first arena row, slots per unit, first unit) of a layer."""
+    off, cap, u0 = C.c_int64(), C.c_int(), C.c_int()
+    _check(load().kvev_decode_layer(handle, B, growth, layer, C.byref(off), C.byref(cap),
+                                    C.byref(u0)), "kvev_decode_layer")
+    return off.value, cap.value, u0.value
+
+
+def kvev_decode_state_offsets(handle: int, B: int, growth: int):
+    """Byte offsets of lens, count, evicted, pos, acc in the state buffer."""
+    offs = (C.c_size_t * 5)()
+    _check(load().kvev_decode_state_offsets(handle, B, growth, offs), "kvev_decode_state_offsets")
+    return dict(zip(("lens", "count", "evicted", "pos", "acc"), list(offs)))
+
+
+def kvev_decode_init(handle, B, growth, pre_K, pre_V, pre_idx, pre_count, h2o_state, lens_ptr,
+                     dec_K, dec_V, dec_state, stream) -> int:
+    return load().kvev_decode_init(handle, B, growth, pre_K, pre_V, pre_idx, pre_count, h2o_state,
+                                   lens_ptr, dec_K, dec_V, dec_state, stream)
+
+
+def kvev_decode_step(handle, B, growth, dec_K, dec_V, dec_state, k_ptrs, v_ptrs, q_ptrs,
+                     stream) -> int:
+    arr = C.c_void_p * len(k_ptrs)
+    return load().kvev_decode_step(handle, B, growth, dec_K, dec_V, dec_state, arr(*k_ptrs),
+                                   arr(*v_ptrs), arr(*q_ptrs), stream)
 
 
 def kvev_status(handle: int) -> int:
@@ -278,3 +321,64 @@ class Plan:
         off = kvev_plan_scores_offset(self.handle, B, S_cap, layer)
         n = B * self.H_kv * S_cap
         return bufs["workspace"][off: off + 4 * n].view(torch.float32).view(B, self.H_kv, S_cap)
+
+
+class DecodeArena:
+    """Decode-phase caches of a Plan for B sequences (torch CUDA tensors as memory)."""
+
+    def __init__(self, plan: "Plan", B: int, growth: int = 0, device="cuda"):
+        import torch
+        self.plan, self.B, self.growth = plan, B, growth
+        self.rows, state_bytes = kvev_decode_query(plan.handle, B, growth)
+        self.K = torch.empty((max(self.rows, 1), plan.d), dtype=torch.bfloat16, device=device)
+        self.V = torch.empty_like(self.K)
+        self.state = torch.zeros(max(state_bytes, 256), dtype=torch.uint8, device=device)
+        self.off = kvev_decode_state_offsets(plan.handle, B, growth)
+        self.layers = [kvev_decode_layer(plan.handle, B, growth, l) for l in range(plan.L)]
+        self.units = sum(B * plan.H_kv for (_, cap, _) in self.layers if cap > 0)
+
+    def _view(self, name, dtype, n):
+        import torch
+        o = self.off[name]
+        return self.state[o: o + 4 * n].view(dtype)
+
+    def lens(self):
+        import torch
+        return self._view("lens", torch.int32, self.B)
+
+    def count(self):
+        import torch
+        return self._view("count", torch.int32, self.units)
+
+    def evicted(self):
+        import torch
+        return self._view("evicted", torch.int32, self.units)
+
+    def pos(self):
+        import torch
+        return self._view("pos", torch.int32, self.rows)
+
+    def acc(self):
+        import torch
+        return self._view("acc", torch.float32, self.rows)
+
+    def init_from_prefill(self, bufs, lens, stream=None):
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        _check(kvev_decode_init(self.plan.handle, self.B, self.growth, bufs["out_K"].data_ptr(),
+                                bufs["out_V"].data_ptr(), bufs["out_idx"].data_ptr(),
+                                bufs["out_count"].data_ptr(), bufs["h2o_state"].data_ptr(),
+                                lens.data_ptr(), self.K.data_ptr(), self.V.data_ptr(),
+                                self.state.data_ptr(), stream.cuda_stream), "kvev_decode_init")
+
+    def step(self, k_new, v_new, q_new, stream=None):
+        """k_new, v_new, q_new: per-layer CUDA tensors (or None for layers without an arena)."""
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        ptr = lambda t: None if t is None else t.data_ptr()
+        _check(kvev_decode_step(self.plan.handle, self.B, self.growth, self.K.data_ptr(),
+                                self.V.data_ptr(), self.state.data_ptr(), [ptr(t) for t in k_new],
+                                [ptr(t) for t in v_new], [ptr(t) for t in q_new],
+                                stream.cuda_stream), "kvev_decode_step")

@@ -170,3 +170,51 @@ def test_evict_argument_errors_before_device_work(kv):
     assert kv.kvev_evict_prefill(**dict(args, workspace_bytes=64)) == kv.ENOMEM
     assert kv.kvev_evict_prefill(**dict(args, B=0)) == kv.OK                          # nothing to do
     kv.kvev_plan_destroy(h)
+
+
+def test_decode_arena_layout(kv):
+    wl = gen.config_decode_mixed()
+    plan = kv.Plan.from_workload(wl)
+    B, growth, H = wl.B, 32, wl.H_kv
+    rows, state = kv.kvev_decode_query(plan.handle, B, growth)
+    caps, row_offs, unit_offs = [], [], []
+    for l in range(wl.L):
+        off, cap, u0 = kv.kvev_decode_layer(plan.handle, B, growth, l)
+        row_offs.append(off)
+        caps.append(cap)
+        unit_offs.append(u0)
+    # evicting decode rules keep b slots, append-only layers b + growth
+    exp_caps = [int(wl.budget[l]) + (growth if wl.route_decode[l] == kv.FULL else 0)
+                for l in range(wl.L)]
+    assert caps == exp_caps
+    assert row_offs == list(np.cumsum([0] + [B * H * c for c in exp_caps])[:-1])
+    assert unit_offs == [B * H * l for l in range(wl.L)]
+    assert rows == sum(B * H * c for c in exp_caps)
+    offs = kv.kvev_decode_state_offsets(plan.handle, B, growth)
+    units = wl.L * B * H
+    assert offs["lens"] == 0 and all(v % 256 == 0 for v in offs.values())
+    assert offs["count"] >= 4 * B and offs["evicted"] >= offs["count"] + 4 * units
+    assert offs["pos"] >= offs["evicted"] + 4 * units and offs["acc"] >= offs["pos"] + 4 * rows
+    assert state >= offs["acc"] + 4 * rows
+    plan.close()
+
+
+def test_decode_layout_rejects_rules_without_a_retained_cache(kv):
+    # a FULL prefill layer keeps the caller's own cache: no decode-phase rule on it
+    h = kv.kvev_plan_create(2, 4, 2, 64, [kv.FULL, kv.H2O], [kv.H2O, kv.H2O], [64, 64], 8, 5,
+                            kv.POOL_MAX, 4)
+    with pytest.raises(kv.KvevError):
+        kv.kvev_decode_query(h, 1, 0)
+    kv.kvev_plan_destroy(h)
+    h = kv.kvev_plan_create(2, 4, 2, 64, [kv.FULL, kv.H2O], [kv.FULL, kv.TOVA], [64, 64], 8, 5,
+                            kv.POOL_MAX, 4)
+    rows, _ = kv.kvev_decode_query(h, 3, 10)
+    assert rows == 3 * 2 * 64   # the FULL layer has no arena, TOVA keeps b slots
+    fake = 1 << 20
+    assert kv.kvev_decode_step(h, 3, 10, fake, fake, fake + 16, [None, fake], [None, fake],
+                               [None, fake], None) == kv.EINVAL   # state must be 256-B aligned
+    assert kv.kvev_decode_step(h, 3, 10, fake, fake, fake, [None, fake], [None, fake],
+                               [None, None], None) == kv.EINVAL   # TOVA needs the queries
+    assert kv.kvev_decode_step(h, 0, 10, fake, fake, fake, [None, fake], [None, fake],
+                               [None, fake], None) == kv.OK       # nothing to do
+    kv.kvev_plan_destroy(h)
