@@ -425,13 +425,127 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
             "steps": n}
 
 
+def decode_step_bytes(wl, counts):
+    """Algorithmic bytes of one decode step: for H2O/TOVA units the retained K rows,
+    the new token's k/q, the slots' positions and acc (read and written); for every
+    unit the new K/V row written (and StreamingLLM's position scan)."""
+    row = wl.d * 2
+    tot = 0
+    for l in range(wl.L):
+        md = int(wl.route_decode[l])
+        c = counts[l]
+        units = wl.B * wl.H_kv
+        if md in (gen.H2O, gen.TOVA):
+            tot += units * (c * row + c * 12 + row * (1 + wl.G) + 2 * row)
+        elif md == gen.STREAMING:
+            tot += units * (c * 4 + 2 * row)
+        elif wl.route[l] != gen.FULL:
+            tot += units * 2 * row
+    return tot
+
+
+def run_decode(args, rank, world, local_rank):
+    """Decode workload: batch 16, 16K-token caches compacted to 2048 slots by the
+    prefill eviction (not timed), then one kvev_decode_step per generated token."""
+    import torch
+    from paper_2606_15157_gb300 import kvev
+
+    torch.cuda.set_device(local_rank)
+    dist = world > 1
+    if dist:
+        import torch.distributed as td
+    wl = gen.config_decode(seed=rank)
+    total = args.warmup + args.steps
+    growth = total
+    plan = kvev.Plan.from_workload(wl)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    need_q = lambda l: wl.route[l] in (gen.SNAPKV, gen.H2O)
+    dev = {l: gen.device_layer(wl, l, need_q=need_q(l)) for l in range(wl.L)}
+    plan.evict_prefill([dev[l][0] for l in range(wl.L)], [dev[l][1] for l in range(wl.L)],
+                       [dev[l][2] for l in range(wl.L)], lens, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    del dev
+    arena = kvev.DecodeArena(plan, wl.B, growth)
+    arena.init_from_prefill(bufs, lens)
+    # every step's new tokens, resident in HBM before the timed region
+    toks = [[gen.device_decode_tokens(wl, t, l) for l in range(wl.L)] for t in range(total)]
+    torch.cuda.synchronize()
+    counts = [int(wl.budget[l]) for l in range(wl.L)]
+    step_bytes = decode_step_bytes(wl, counts)
+    stream = torch.cuda.current_stream()
+
+    def run(t):
+        k = [x[0] for x in toks[t]]
+        v = [x[1] for x in toks[t]]
+        q = [x[2] for x in toks[t]]
+        arena.step(k, v, q, stream)
+
+    for t in range(args.warmup):
+        run(t)
+    if dist:
+        td.barrier()
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    with ClockSampler(local_rank) as clk:
+        if dist:
+            td.barrier()
+        torch.cuda.synchronize()
+        evs[0].record(stream)
+        for i in range(args.steps):
+            run(args.warmup + i)
+            evs[i + 1].record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            td.barrier()
+    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    ms = evs[0].elapsed_time(evs[-1]) / args.steps
+    if dist:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        td.all_reduce(t, op=td.ReduceOp.MAX)
+        ms = float(t.item())
+    assert plan.status() == kvev.OK
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    value = world * step_bytes / (ms / 1e3) / 1e9
+    achieved = step_bytes / (statistics.median(per) / 1e3) / 1e9
+    if rank == 0:
+        out = {
+            "metric": "KV decode-step GB/s (retained-cache update per generated token)",
+            "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; shapes of LLaMA-3.1-8B decode with compacted caches)",
+            "config": {"workload": wl.name, "layers": wl.L, "batch": wl.B, "cache_slots": 2048,
+                       "route_decode": {"h2o": int((wl.route_decode == gen.H2O).sum()),
+                                        "streaming": int((wl.route_decode == gen.STREAMING).sum()),
+                                        "append": int(((wl.route_decode == gen.FULL) &
+                                                       (wl.route != gen.FULL)).sum())},
+                       "l2": "retained K of the H2O layers (470 MB) larger than L2",
+                       "parallelism": f"independent batch per GPU x{world}"},
+            "tokens_per_s": world * wl.B / (ms / 1e3),
+            "roofline": {"kernel": "decode_step_kernel", "bound": "hbm", "achieved": achieved,
+                         "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                         "traffic": None},
+            "clocks": clk.summary(),
+            "gpu_launches": 2 * args.steps,
+            "e2e": None, "cpu_baseline": None,
+        }
+        print(json.dumps(out), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="long", choices=["long", "long32k", "homog8k", "hetero8k"])
+    ap.add_argument("--workload", default="long",
+                    choices=["long", "long32k", "homog8k", "hetero8k", "decode"])
     ap.add_argument("--batch", type=int, default=None,
                     help="use only the first B sequences of the 'long' workload (profiling)")
     ap.add_argument("--e2e-steps", type=int, default=5)
@@ -452,6 +566,8 @@ def main():
         td.init_process_group("nccl")
     if args.impl == "reference":
         run_reference(args, rank, world)
+    elif args.workload == "decode":
+        run_decode(args, rank, world, local_rank)
     else:
         run_ours(args, rank, world, local_rank)
     if world > 1 and args.impl == "ours":

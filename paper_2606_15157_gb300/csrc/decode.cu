@@ -167,28 +167,61 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
       q[g][2 * e + 1] = bf16_hi(w4[e]) * p.scale_log2;
     }
   }
-  // logits (base 2) of slots 0..c-1 and of the new token at index c
+  // logits (base 2) of slots 0..c-1 and of the new token at index c; kU row
+  // passes per iteration, their loads issued before any arithmetic
+  constexpr int kU = 4;
   const int cnt = c + 1;
-  for (int j0 = 0; j0 < cnt; j0 += SPB) {
-    const int j = j0 + warp * SPW + grp;
-    uint4 kv = make_uint4(0, 0, 0, 0);
-    if (j < c) kv = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j) * D + sub * 8));
-    else if (j == c) kv = *reinterpret_cast<const uint4*>(kn + sub * 8);
-    const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
-    float kf[8];
+  for (int j0 = 0; j0 < cnt; j0 += kU * SPB) {
+    uint4 kv[kU];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      kf[2 * e] = bf16_lo(w4[e]);
-      kf[2 * e + 1] = bf16_hi(w4[e]);
+    for (int u = 0; u < kU; ++u) {
+      const int j = j0 + u * SPB + warp * SPW + grp;
+      kv[u] = make_uint4(0, 0, 0, 0);
+      if (j < c) kv[u] = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j) * D + sub * 8));
+      else if (j == c) kv[u] = *reinterpret_cast<const uint4*>(kn + sub * 8);
     }
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float a = 0.f;
+    for (int u = 0; u < kU; ++u) {
+      const int j = j0 + u * SPB + warp * SPW + grp;
+      const uint32_t w4[4] = {kv[u].x, kv[u].y, kv[u].z, kv[u].w};
+      float kf[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) a = fmaf(q[g][e], kf[e], a);
+      for (int e = 0; e < 4; ++e) {
+        kf[2 * e] = bf16_lo(w4[e]);
+        kf[2 * e + 1] = bf16_hi(w4[e]);
+      }
+      float a[G];
 #pragma unroll
-      for (int o = LPS / 2; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-      if (sub == 0 && j < cnt) lg[g * ld + j] = a;
+      for (int g = 0; g < G; ++g) {
+        a[g] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[g] = fmaf(q[g][e], kf[e], a[g]);
+      }
+      // Sum each head's partials over the row's LPS lanes, splitting the G
+      // values between lane halves at every step (log2(LPS) + G - 1 shuffles
+      // instead of G * log2(LPS)); afterwards lane `sub` holds the total of
+      // head sub / (LPS / G).
+      int nv = G;
+#pragma unroll
+      for (int o = LPS / 2; o > 0; o >>= 1) {
+        if (nv > 1) {
+          const bool upper = (sub & o) != 0;
+          const int half = nv / 2;
+#pragma unroll
+          for (int i = 0; i < G / 2; ++i) {
+            if (i < half) {
+              const float send = upper ? a[i] : a[i + half];
+              const float keep = upper ? a[i + half] : a[i];
+              a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+            }
+          }
+          nv = half;
+        } else {
+          a[0] += __shfl_xor_sync(0xffffffffu, a[0], o);
+        }
+      }
+      constexpr int kLanesPerHead = LPS / G;
+      if (sub % kLanesPerHead == 0 && j < cnt) lg[(sub / kLanesPerHead) * ld + j] = a[0];
     }
   }
   __syncthreads();
