@@ -454,7 +454,7 @@ def run_decode(args, rank, world, local_rank):
     dist = world > 1
     if dist:
         import torch.distributed as td
-    wl = gen.config_decode(seed=rank)
+    wl = gen.config_decode(seed=rank, B=args.batch or 16)
     total = args.warmup + args.steps
     growth = total
     plan = kvev.Plan.from_workload(wl)
@@ -547,7 +547,8 @@ def main():
     ap.add_argument("--workload", default="long",
                     choices=["long", "long32k", "homog8k", "hetero8k", "decode"])
     ap.add_argument("--batch", type=int, default=None,
-                    help="use only the first B sequences of the 'long' workload (profiling)")
+                    help="use only the first B sequences of the 'long' workload, or B sequences "
+                         "in the decode workload (profiling)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
