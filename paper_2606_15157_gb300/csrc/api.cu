@@ -59,7 +59,7 @@ bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 struct WsLayout {
   int n_units = 0, R = 0, R_pad = 0, max_items = 0;
   size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
-         lam = 0, raw = 0, raw1 = 0, total = 0;
+         lam = 0, raw = 0, total = 0;
 };
 
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
@@ -81,15 +81,9 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.ready = take(sizeof(int) * std::max(w.n_units, 1));
   w.chunk_start = take(sizeof(int) * (w.n_units + 1));
   w.item = take(sizeof(int4) * std::max(w.max_items, 1));
-  // sweep-1 partials: one record per (item, softmax warpgroup), of the rows of
-  // that warpgroup's 128-row group
-  const int part_rows = w.R_pad > 128 ? 128 : w.R_pad;
-  w.part = take(sizeof(float2) * kSoftmaxWGs * static_cast<size_t>(w.max_items) * part_rows);
+  w.part = take(sizeof(float2) * static_cast<size_t>(w.max_items) * w.R_pad);  // one per chunk
   w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
   w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
-  // with two row groups the score kernel writes each score as two partial sums
-  // (rows 0-127 into raw, the rest into raw1); the selection kernel adds them
-  w.raw1 = take(w.R_pad > 128 ? sizeof(float) * static_cast<size_t>(w.n_units) * S_cap : 0);
   w.total = off;
   return w;
 }
@@ -591,7 +585,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.part = reinterpret_cast<float2*>(wsb + ws.part);
     sp.lam = reinterpret_cast<float*>(wsb + ws.lam);
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
-    sp.raw1 = ws.R_pad > 128 ? reinterpret_cast<float*>(wsb + ws.raw1) : nullptr;
     sp.wait_ns = P.wait_ns;
     sp.stall_unit = P.stall_unit;
     mark(KVEV_K_SCORE, 0);
@@ -629,7 +622,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.sink = P.sink;
   sel.lens = lens_ok;
   sel.raw = reinterpret_cast<float*>(wsb + ws.raw);
-  sel.raw1 = ws.R_pad > 128 ? reinterpret_cast<const float*>(wsb + ws.raw1) : nullptr;
   sel.out_idx = out_idx;
   sel.out_count = out_count;
   const size_t sel_smem = ws.n_units > 0 ? sizeof(uint32_t) * static_cast<size_t>(S_cap) : 0;

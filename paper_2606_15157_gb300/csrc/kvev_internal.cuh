@@ -23,12 +23,12 @@ constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel 
 constexpr int kScoreThreads = 128 * (1 + kSoftmaxWGs);  // + warpgroup 0: TMA warp, MMA warp, 2 idle
 constexpr int kSlots = 4;             // TMEM accumulator slots of the score kernel
 constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 512 columns)
-// Register split of the score kernel (setmaxnreg): warpgroup 0 shrinks to 56,
+// Register split of the score kernel (setmaxnreg): warpgroup 0 shrinks to 64,
 // the softmax warpgroups grow to 104.  The CTA must be launched with at least
-// 128 * 56 + 512 * 104 = 60416 registers (96 per thread x 640): the host
+// 128 * 64 + 512 * 104 = 61440 registers (96 per thread x 640): the host
 // checks the compiled allocation before launching, since an increase that the
 // launch pool cannot cover would never complete.
-constexpr int kRegsControl = 56;
+constexpr int kRegsControl = 64;
 constexpr int kRegsSoftmax = 104;
 constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
 constexpr int kSelectThreads = 512;
@@ -80,11 +80,9 @@ struct ScoreParams {
   int* ready;
   int* abort_flag;
   int* status;
-  float2* part;       // [items][4][PR] per-row (max, sum) partials per softmax warpgroup,
-                      // base-2 units; PR = 128 when R_pad > 128, else R_pad
+  float2* part;       // [items][R_pad] per-row (max, sum) of each chunk, base-2 units
   float* lam;         // [n_units][R_pad] per-row log2-sum-exp
-  float* raw;         // [n_units][S_cap] window scores (rows 0-127 partial when R_pad > 128)
-  float* raw1;        // [n_units][S_cap] rows 128+ partial when R_pad > 128
+  float* raw;         // [n_units][S_cap] window scores
   long long wait_ns;
   int stall_unit;
 };
@@ -93,8 +91,7 @@ struct SelectParams {
   LayerDesc layer[kMaxLayers];
   int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink;
   const int* lens;
-  float* raw;         // [n_units][S_cap]
-  const float* raw1;  // second partial of each score (R_pad > 128), or nullptr
+  const float* raw;   // [n_units][S_cap]
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
 };
@@ -177,6 +174,15 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// mbarrier arrive from the lane that elect.sync picks in a converged warp.
+__device__ __forceinline__ void mbar_arrive_elect(uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}" ::"r"(smem_u32(bar))
+      : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {

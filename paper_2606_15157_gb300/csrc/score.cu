@@ -43,7 +43,13 @@ struct Smem {
   uint8_t* qbuf;     // two Q buffers of qbytes each, indexed arithmetically (a dynamically
   uint32_t qbytes;   // indexed member array would push the whole struct to local memory)
   uint8_t* kbuf;     // stages * tile bytes
-  float* lam;        // [4][R_pad]: per-warpgroup copy of -lse2 of the current sweep-2 unit
+  float* lam;        // [2][R_pad]: -lse2 of the units of the next two sweep-2 entries
+  float* red;        // [2][kSoftmaxWGs][128]: per-warpgroup partial key sums of a sweep-2 tile
+  float2* pc;        // [kSoftmaxWGs][R_pad]: per-warpgroup (max, sum) of a sweep-1 item
+  uint64_t* lfull;   // [2] lam buffer written by the normaliser warp
+  uint64_t* lempty;  // [2] lam buffer read by the softmax warpgroups
+  uint64_t* pfull;   // partials of a sweep-1 entry written to pc by the softmax threads
+  uint64_t* pempty;  // pc read by the publisher warp
   uint64_t* kfull;
   uint64_t* kempty;
   uint64_t* qfull;
@@ -52,23 +58,39 @@ struct Smem {
   uint64_t* tempty;
   uint64_t* done;
   uint32_t* tmem_slot;
-  int* flag;         // [8]: [wg] last-arrival of sweep 1, [4+wg] ready of sweep 2
+  int* flag;         // [2]: scratch of the publisher warp
 };
+
+__host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int R_pad, int stages,
+                                                      size_t* koff, size_t* loff, size_t* roff,
+                                                      size_t* poff, size_t* boff) {
+  size_t off = 2 * static_cast<size_t>(q_rows) * D * 2;
+  *koff = off;
+  off += static_cast<size_t>(stages) * kTileKeys * D * 2;
+  *loff = off;
+  off += sizeof(float) * 2 * R_pad;
+  *roff = off;
+  off += sizeof(float) * 2 * kSoftmaxWGs * 128;
+  off = (off + 7) & ~size_t(7);
+  *poff = off;
+  off += sizeof(float2) * kSoftmaxWGs * R_pad;
+  *boff = off;
+  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6);
+  off += sizeof(uint32_t) + 2 * sizeof(int);
+  return off;
+}
 
 __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D) {
   Smem s;
-  size_t off = 0;
-  const size_t qbytes = static_cast<size_t>(p.q_rows) * D * 2;
-  const size_t tbytes = static_cast<size_t>(kTileKeys) * D * 2;
-  s.qbuf = base + off;
-  s.qbytes = static_cast<uint32_t>(qbytes);
-  off += 2 * qbytes;
-  s.kbuf = base + off;
-  off += tbytes * p.stages;
-  s.lam = reinterpret_cast<float*>(base + off);
-  off += kSoftmaxWGs * sizeof(float) * p.R_pad;
-  off = (off + 7) & ~size_t(7);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base + off);
+  size_t koff, loff, roff, poff, boff;
+  smem_size(D, p.q_rows, p.R_pad, p.stages, &koff, &loff, &roff, &poff, &boff);
+  s.qbuf = base;
+  s.qbytes = static_cast<uint32_t>(p.q_rows) * D * 2;
+  s.kbuf = base + koff;
+  s.lam = reinterpret_cast<float*>(base + loff);
+  s.red = reinterpret_cast<float*>(base + roff);
+  s.pc = reinterpret_cast<float2*>(base + poff);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + boff);
   s.kfull = bars;
   s.kempty = bars + p.stages;
   s.qfull = bars + 2 * p.stages;
@@ -76,7 +98,11 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   s.tfull = s.qempty + 2;
   s.tempty = s.tfull + kSlots;
   s.done = s.tempty + kSlots;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.done + 1);
+  s.lfull = s.done + 1;
+  s.lempty = s.lfull + 2;
+  s.pfull = s.lempty + 2;
+  s.pempty = s.pfull + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.pempty + 1);
   s.flag = reinterpret_cast<int*>(s.tmem_slot + 1);
   return s;
 }
@@ -110,6 +136,33 @@ __device__ __forceinline__ ItemInfo decode_item(const ScoreParams& p, int t, int
 __device__ __forceinline__ void prefetch_item(const ScoreParams& p, int first, int stride, int j, int J) {
   if (j + 1 < J) asm volatile("prefetch.global.L1 [%0];" ::"l"(p.item + first + (j + 1) * stride));
 }
+
+// A CTA's work entries in order: at step j = 0 .. J + kLag - 1, sweep 1 of
+// item j (j < J), then sweep 2 of item j - kLag (j >= kLag).  Sweep 2 of an
+// item runs kLag sweep-1 items after its own sweep 1, so the unit's row
+// normalisers (which need every chunk of the unit, some of them on other
+// CTAs) are almost always published by then.  Every entry loads its own Q
+// (buffer e mod 2 for entry e).
+constexpr int kLag = 2;
+struct EntryIter {
+  int J, j = 0, sweep = -1;
+  __device__ __forceinline__ explicit EntryIter(int J_) : J(J_) {}
+  // Next entry: item index jj (of this CTA) and sweep; false at the end.
+  __device__ __forceinline__ bool next(int& jj, int& sw) {
+    for (;;) {
+      if (++sweep == 2) {
+        sweep = 0;
+        ++j;
+      }
+      if (j >= J + kLag) return false;
+      jj = sweep == 0 ? j : j - kLag;
+      if (jj >= 0 && jj < J) {
+        sw = sweep;
+        return true;
+      }
+    }
+  }
+};
 
 // Bounded wait on an mbarrier phase; false if it ran out or another role
 // aborted.  Each try sleeps in hardware for up to kWaitSliceNs, so the abort
@@ -147,52 +200,60 @@ __device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, u
 // Producer: TMA loads of Q (once per item) and of K tiles (twice per item).
 // ---------------------------------------------------------------------------
 template <int D>
+__device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uint32_t e, const ItemInfo& it) {
+  const uint32_t qb = e & 1;
+  mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R_pad) * D * 2);
+  const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
+#pragma unroll
+  for (int kc = 0; kc < D / 64; ++kc)
+    tma_load_2d(sm.qbuf + qb * sm.qbytes + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
+                kc * 64, qrow, &sm.qfull[qb]);
+}
+
+template <int D>
 __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
-  const uint32_t qbytes = static_cast<uint32_t>(p.R_pad) * D * 2;
   const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
   const uint64_t drop = policy_evict_first();  // second read: its last use
   uint32_t tile = 0;            // tiles issued (for the drain after an abort)
   uint32_t pst = 0, pph = 0;    // K stage ring: position and phase of the next tile
-  int last_q_item = -1;
-  int issued_q0 = 0, issued_q1 = 0;  // Q loads issued into each buffer
+  uint32_t q_issued = 0;        // entries whose Q load has been issued
   bool ok = true;
-  for (int j = 0; j <= J && ok; ++j) {
-    prefetch_item(p, first, stride, j, J);
-    for (int sweep = 0; sweep < 2 && ok; ++sweep) {
-      const int jj = sweep == 0 ? j : j - 1;
-      if (sweep == 0 && j >= J) continue;
-      if (sweep == 1 && j == 0) continue;
-      const int t = first + jj * stride;
-      const ItemInfo it = decode_item(p, t, load_item(p, t));
-      const CUtensorMap* kmap = &p.kmap[it.ls];
-      if (sweep == 0) {
-        const int qb = jj & 1;
-        if (!wait_bar(&sm.qempty[qb], ((jj >> 1) & 1) ^ 1, p)) { ok = false; break; }
-        mbar_expect_tx(&sm.qfull[qb], qbytes);
-        const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
-#pragma unroll
-        for (int kc = 0; kc < D / 64; ++kc)
-          tma_load_2d(sm.qbuf + qb * sm.qbytes + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
-                      kc * 64, qrow, &sm.qfull[qb]);
-        if (qb == 0) issued_q0 = jj + 1; else issued_q1 = jj + 1;
-        last_q_item = jj;
+  EntryIter ei(J);
+  int jj, sw;
+  for (uint32_t e = 0; ok && ei.next(jj, sw); ++e) {
+    const int t = first + jj * stride;
+    if (sw == 0) prefetch_item(p, first, stride, jj, J);
+    const ItemInfo it = decode_item(p, t, load_item(p, t));
+    if (q_issued == e) {
+      if (!wait_bar(&sm.qempty[e & 1], ((e >> 1) & 1) ^ 1, p)) { ok = false; break; }
+      load_q<D>(p, sm, e, it);
+      ++q_issued;
+    }
+    // the next entry's Q goes out as soon as its buffer is released
+    EntryIter la = ei;
+    int jn, swn;
+    const bool has_next = la.next(jn, swn);
+    const CUtensorMap* kmap = &p.kmap[it.ls];
+    const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
+    for (int i = 0; i < it.ntiles; ++i, ++tile) {
+      if (has_next && q_issued == e + 1 &&
+          mbar_try_wait(&sm.qempty[(e + 1) & 1], (((e + 1) >> 1) & 1) ^ 1)) {
+        const int tn = first + jn * stride;
+        load_q<D>(p, sm, e + 1, decode_item(p, tn, load_item(p, tn)));
+        ++q_issued;
       }
-      const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
-      for (int i = 0; i < it.ntiles; ++i, ++tile) {
-        const uint32_t st = pst, ph = pph;
-        if (++pst == static_cast<uint32_t>(p.stages)) { pst = 0; pph ^= 1; }
-        if (!wait_bar(&sm.kempty[st], ph ^ 1, p)) { ok = false; break; }
-        uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kTileBytes;
-        mbar_expect_tx(&sm.kfull[st], kTileBytes);
+      const uint32_t st = pst, ph = pph;
+      if (++pst == static_cast<uint32_t>(p.stages)) { pst = 0; pph ^= 1; }
+      if (!wait_bar(&sm.kempty[st], ph ^ 1, p)) { ok = false; break; }
+      uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kTileBytes;
+      mbar_expect_tx(&sm.kfull[st], kTileBytes);
 #pragma unroll
-        for (int kc = 0; kc < D / 64; ++kc)
-          tma_load_2d_hint(dst + kc * (kTileKeys * 128), kmap, kc * 64, row0 + i * kTileKeys,
-                           &sm.kfull[st], sweep == 0 ? keep : drop);
-      }
+      for (int kc = 0; kc < D / 64; ++kc)
+        tma_load_2d_hint(dst + kc * (kTileKeys * 128), kmap, kc * 64, row0 + i * kTileKeys,
+                         &sm.kfull[st], sw == 0 ? keep : drop);
     }
   }
-  (void)last_q_item;
   // Drain: make sure no copy is still landing in shared memory when the CTA
   // retires (only relevant after an abort; normally every load was consumed).
   if (!ok) {
@@ -201,8 +262,10 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
       const uint32_t last = ((tile - 1 - st) / S) * S + st;  // last tile issued into st
       wait_bar_drain(&sm.kfull[st], (last / S) & 1, 100000000ull);
     }
-    if (issued_q0 > 0) wait_bar_drain(&sm.qfull[0], ((issued_q0 - 1) >> 1) & 1, 100000000ull);
-    if (issued_q1 > 0) wait_bar_drain(&sm.qfull[1], ((issued_q1 - 1) >> 1) & 1, 100000000ull);
+    for (uint32_t b = 0; b < 2; ++b) {
+      const uint32_t nb = (q_issued + 1 - b) / 2;  // Q loads issued into buffer b
+      if (nb > 0) wait_bar_drain(&sm.qfull[b], (nb - 1) & 1, 100000000ull);
+    }
   }
 }
 
@@ -216,27 +279,25 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
   const int nh = p.R_pad > 128 ? 2 : 1;
   const uint32_t idesc1 = idesc_bf16_f32(128, kTileKeys);
-  // sweep 2: N = rows of the group (128, or what is left of R_pad in the last group)
-  const uint32_t idesc2a = idesc_bf16_f32(128, p.R_pad > 128 ? 128 : p.R_pad);
-  const uint32_t idesc2b = idesc_bf16_f32(128, p.R_pad > 128 ? p.R_pad - 128 : 128);
+  // sweep 2: one MMA chain with N = every window row (up to 256 = two slots side by side)
+  const uint32_t idesc2 = idesc_bf16_f32(128, p.R_pad);
   // descriptor steps (address / 16) between the 64-wide column blocks of Q and of a K tile
   const uint32_t qcol_step = static_cast<uint32_t>(p.q_rows) * 128 / 16;
   constexpr uint32_t kcol_step = kTileKeys * 128 / 16;
   uint32_t st = 0, kph = 0;  // K stage ring: position and phase of the next tile
   uint32_t sl = 0, tph = 0;  // TMEM slot ring: position and phase of the next slot
   bool ok = true;
-  for (int j = 0; j <= J && ok; ++j) {
-    prefetch_item(p, first, stride, j, J);
-    for (int sweep = 0; sweep < 2 && ok; ++sweep) {
-      const int jj = sweep == 0 ? j : j - 1;
-      if (sweep == 0 && j >= J) continue;
-      if (sweep == 1 && j == 0) continue;
+  EntryIter ei(J);
+  int jj, sw;
+  for (uint32_t e = 0; ok && ei.next(jj, sw); ++e) {
+    {
       const int t = first + jj * stride;
+      if (sw == 0) prefetch_item(p, first, stride, jj, J);
       const ItemInfo it = decode_item(p, t, load_item(p, t));
-      const int qb = jj & 1;
+      const uint32_t qb = e & 1;
       const uint64_t qdesc0 = sw128_desc(smem_u32(sm.qbuf) + qb * sm.qbytes);
-      if (sweep == 0 && !wait_bar_warp(&sm.qfull[qb], (jj >> 1) & 1, p)) { ok = false; break; }
-      const bool s1 = sweep == 0;
+      if (!wait_bar_warp(&sm.qfull[qb], (e >> 1) & 1, p)) { ok = false; break; }
+      const bool s1 = sw == 0;
       const uint32_t astep = s1 ? qcol_step : kcol_step, bstep = s1 ? kcol_step : qcol_step;
       for (int i = 0; i < it.ntiles; ++i) {
         if (!wait_bar_warp(&sm.kfull[st], kph, p)) { ok = false; break; }
@@ -244,28 +305,41 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
         // descriptor's low field is the address / 16, so the k-step offsets
         // (all inside shared memory, no carry out of the field) are plain adds.
         const uint64_t kdesc = sw128_desc(smem_u32(sm.kbuf) + st * kTileBytes);
-        // One 128-column TMEM slot per 128-row group of Q: sweep 1 writes
-        // S[rows of group h][keys], sweep 2 writes S^T[keys][rows of group h].
-        for (int h = 0; h < nh; ++h) {
-          if (!wait_bar_warp(&sm.tempty[sl], tph ^ 1, p)) { ok = false; break; }
-          tc_fence_after();
+        // One 128-column TMEM slot per 128-row group of Q.  Sweep 1 writes
+        // S[rows of group h][keys] into slot sl + h with one MMA chain per
+        // group; sweep 2 writes S^T[keys][all rows] with a single chain of
+        // N = R_pad across the tile's slots (sl is even when nh = 2), which
+        // reads the K tile once instead of once per group.
+        for (int h = 0; h < nh; ++h)
+          if (!wait_bar_warp(&sm.tempty[sl + h], tph ^ 1, p)) { ok = false; break; }
+        if (!ok) break;
+        tc_fence_after();
+        if (s1) {
+          for (int h = 0; h < nh; ++h) {
+            const uint32_t dcol = tmem_base + (sl + h) * kSlotCols;
+            const uint64_t qdesc = qdesc0 + static_cast<uint64_t>(h * (128 * 128 / 16));
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+              const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
+              umma_bf16_elect(dcol, qdesc + a, kdesc + b, idesc1, k > 0);
+            }
+            umma_commit_elect(&sm.tfull[sl + h]);
+          }
+        } else {
           const uint32_t dcol = tmem_base + sl * kSlotCols;
-          const uint64_t qdesc = qdesc0 + static_cast<uint64_t>(h * (128 * 128 / 16));
-          const uint32_t idesc = s1 ? idesc1 : (h == 0 ? idesc2a : idesc2b);
-          const uint64_t adesc = s1 ? qdesc : kdesc, bdesc = s1 ? kdesc : qdesc;
 #pragma unroll
           for (int k = 0; k < D / 16; ++k) {
             const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
-            umma_bf16_elect(dcol, adesc + a, bdesc + b, idesc, k > 0);
+            umma_bf16_elect(dcol, kdesc + a, qdesc0 + b, idesc2, k > 0);
           }
-          umma_commit_elect(&sm.tfull[sl]);
-          if (++sl == kSlots) { sl = 0; tph ^= 1; }
+          for (int h = 0; h < nh; ++h) umma_commit_elect(&sm.tfull[sl + h]);
         }
-        if (!ok) break;
+        sl += nh;
+        if (sl == kSlots) { sl = 0; tph ^= 1; }
         umma_commit_elect(&sm.kempty[st]);
         if (++st == static_cast<uint32_t>(p.stages)) { st = 0; kph ^= 1; }
       }
-      if (ok && sweep == 1) umma_commit_elect(&sm.qempty[qb]);
+      if (ok) umma_commit_elect(&sm.qempty[qb]);  // the entry's Q buffer is free once these finish
     }
   }
   // Every MMA issued so far has completed once `done` flips.
@@ -352,214 +426,232 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
 }
 
 // ---- TMEM slot hand-off --------------------------------------------------
-// A warpgroup waits for slot g to be filled, copies its part of the slot into
-// registers, and releases the slot before doing any arithmetic, so the MMA of
-// later tiles overlaps the exponentials.
+// Every fill is consumed by all four softmax warpgroups: warpgroup w copies
+// its 32-column slice [32w, 32w + 32) of the slot and releases the slot at
+// once (the slot's empty barrier counts all 512 softmax threads), so the
+// tensor core refills a slot as soon as the last slice is copied and no
+// warpgroup holds a slot while it computes.
 
-__device__ __forceinline__ bool slot_acquire(const ScoreParams& p, const Smem& sm, uint32_t g,
-                                             bool ok) {
-  if (ok && !wait_bar(&sm.tfull[g % kSlots], (g / kSlots) & 1, p)) ok = false;
-  ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld needs the whole warp
-  if (ok) tc_fence_after();
+__device__ __forceinline__ bool slot_wait(const ScoreParams& p, const Smem& sm, uint32_t g, bool ok) {
+  if (ok && !wait_bar(&sm.tfull[g & (kSlots - 1)], (g / kSlots) & 1, p)) ok = false;
   return ok;
 }
 
-__device__ __forceinline__ void slot_release(const Smem& sm, uint32_t g) {
+// Copy this warpgroup's 32 columns of slot (g mod 4) and release the slot.
+// Loaded even when the wait failed (the address is always inside this CTA's
+// TMEM allocation; the values are then discarded): a conditional load would
+// leave the array undefined on one path and spill it.
+__device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r)[32]) {
+  const uint32_t sl = g & (kSlots - 1);
+  tmem_ld32_async(lane_base + sl * kSlotCols, r);
+  tmem_wait32(r);
   tc_fence_before();
-  mbar_arrive(&sm.tempty[g % kSlots]);
+  mbar_arrive(&sm.tempty[sl]);
 }
 
-template <int NCH>
-__device__ __forceinline__ void load_slot(uint32_t taddr, uint32_t (&r)[NCH][32]) {
-#pragma unroll
-  for (int c = 0; c < NCH; ++c) tmem_ld32_async(taddr + c * 32, r[c]);
-#pragma unroll
-  for (int c = 0; c < NCH; ++c) tmem_wait32(r[c]);
-}
-
-// Sweep 1, slot g: this thread's row `row` against the tile's 128 keys, in two
-// 64-column pieces (copy, then arithmetic); the slot is released after the
-// second copy.
-__device__ __forceinline__ void s1_slot(const ScoreParams& p, const Smem& sm, uint32_t lane_addr,
-                                        uint32_t g, bool& ok, int row, int n, int kb, float& m,
-                                        float& z) {
-  ok = slot_acquire(p, sm, g, ok);
-  const int tr = row < p.R ? row_pos(p, row, n) : -1;
-  const bool full = (kb + kTileKeys - 1) <= (n - p.W);  // every key visible to every row
-#pragma unroll
-  for (int piece = 0; piece < 2; ++piece) {
-    // Loaded even when the wait failed (the address is always inside this
-    // CTA's TMEM allocation; the values are then discarded): a conditional
-    // load would leave the array undefined on one path and spill it.
-    uint32_t r[2][32];
-    load_slot<2>(lane_addr + piece * 64, r);
-    if (piece == 1) slot_release(sm, g);
-    if (ok && tr >= 0) {
-      s1_chunk(r[0], p.scale_log2, full, kb + piece * 64, tr, m, z);
-      s1_chunk(r[1], p.scale_log2, full, kb + piece * 64 + 32, tr, m, z);
-    }
-  }
-}
-
-// Sweep 2, slot g: this thread's key k against rows r0 .. r0 + 32*nch, in
-// pieces of up to 64 columns; partial sum into a[8].
-template <int NCH>
-__device__ __forceinline__ void s2_piece(const ScoreParams& p, uint32_t taddr, bool ok, bool full,
-                                         const float* nl, int r0, int k, int n, float (&a)[8]) {
-  uint32_t r[NCH][32];
-  load_slot<NCH>(taddr, r);
-  if (!ok || k >= n) return;
-#pragma unroll
-  for (int c = 0; c < NCH; ++c) s2_chunk(p, r[c], full, nl + c * 32, r0 + c * 32, k, n, a);
-}
-
-__device__ __forceinline__ void s2_slot(const ScoreParams& p, const Smem& sm, uint32_t lane_addr,
-                                        uint32_t g, bool& ok, int nch, int r0, int k, int n,
-                                        int kb, const float* nlam, float (&a)[8]) {
-  ok = slot_acquire(p, sm, g, ok);
-  const bool full = (kb + kTileKeys - 1 <= n - p.W) && (r0 + nch * 32 <= p.R);
-  for (int c = 0; c < nch; c += 2) {
-    if (c + 1 < nch)
-      s2_piece<2>(p, lane_addr + c * 32, ok, full, nlam + r0 + c * 32, r0 + c * 32, k, n, a);
-    else
-      s2_piece<1>(p, lane_addr + c * 32, ok, full, nlam + r0 + c * 32, r0 + c * 32, k, n, a);
-  }
-  slot_release(sm, g);
-}
-
-// Softmax warpgroup wg (0..3) owns TMEM slot wg.  Slot g of the tile stream
-// (tile t, 128-row group h -> g = t*nh + h) lands in slot g % 4, so with
-// nh = 2 warpgroup wg handles row group wg & 1 of the tiles t = wg >> 1 (mod 2)
-// and with nh = 1 the whole of tiles t = wg (mod 4).  No two warpgroups
-// share a slot or synchronise with each other; partial results go to global
-// memory (sweep 1: per-row (max, sum) per warpgroup; sweep 2: one partial sum
-// per 128-row group, added by the selection kernel).
 __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base,
                                            int wg, int first, int stride, int J) {
   const int warp = threadIdx.x >> 5;
-  const int quarter = warp & 3;                       // TMEM lane quarter of this warp
+  const int quarter = warp & 3;                        // TMEM lane quarter of this warp
   const int lrow = quarter * 32 + (threadIdx.x & 31);  // TMEM lane: row (sweep 1) / key (sweep 2)
-  const int wtid = threadIdx.x - (4 + 4 * wg) * 32;    // 0..127 within the warpgroup
-  const int bar_id = 1 + wg;
+  const int stid = threadIdx.x - 128;                  // 0..511 over the softmax warpgroups
   const int nh = p.R_pad > 128 ? 2 : 1;                // 128-row groups (slots) per tile
-  const int half = nh == 2 ? (wg & 1) : 0;             // row group of this warpgroup
-  const uint32_t tmask = nh == 2 ? 1 : 3, tres = nh == 2 ? (wg >> 1) : wg;  // own tiles: (t & tmask) == tres
-  const int row = half * 128 + lrow;                   // sweep-1 row of this thread
-  const int r0 = half * 128;                           // sweep-2 first row
-  const int nch = (nh == 2 ? (half == 0 ? 128 : p.R_pad - 128) : p.R_pad) / 32;
-  const int PR = nh == 2 ? 128 : p.R_pad;              // rows per sweep-1 partial record
-  float* raw_out = half == 0 ? p.raw : p.raw1;
-  const uint32_t lane_addr =
-      tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + wg * kSlotCols;
-  float* nlam = sm.lam + wg * p.R_pad;  // -lse2 of the current sweep-2 unit
-  uint32_t tile = 0;
+  // this warpgroup's column slice of every slot
+  const uint32_t lane_base =
+      tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(32 * wg);
+  // sweep 2: this warpgroup's rows [32wg, 32wg + 32) of group 0 and [128 + 32wg, ...) of group 1
+  const int r0a = 32 * wg, r0b = 128 + 32 * wg;
+  const bool has_a = r0a < (nh == 2 ? 128 : p.R_pad);
+  const bool has_b = nh == 2 && r0b < p.R_pad;
+  uint32_t g = 0;     // slot stream position (advances nh per tile)
+  uint32_t tc = 0;    // sweep-2 tiles done (reduction buffer parity, writer)
+  uint32_t q1 = 0, q2 = 0;  // sweep-1 / sweep-2 entries done
   bool ok = true;
 
-  for (int j = 0; j <= J; ++j) {
-    prefetch_item(p, first, stride, j, J);
-    // ---------------- sweep 1 of item j ----------------
-    if (j < J) {
-      const int t = first + j * stride;
+  EntryIter ei(J);
+  int jj, sw;
+  while (ei.next(jj, sw)) {
+    // ---------------- sweep 1 ----------------
+    if (sw == 0) {
+      prefetch_item(p, first, stride, jj, J);
+      const int t = first + jj * stride;
       const ItemInfo it = decode_item(p, t, load_item(p, t));
-      float m = -INFINITY, z = 0.f;
+      float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
+      const int tr0 = lrow < p.R ? row_pos(p, lrow, it.n) : -1;
+      const int tr1 = 128 + lrow < p.R ? row_pos(p, 128 + lrow, it.n) : -1;
       for (int i = 0; i < it.ntiles; ++i) {
-        const uint32_t gt = tile + i;
-        if ((gt & tmask) != tres) continue;
-        s1_slot(p, sm, lane_addr, gt * nh + half, ok, row, it.n, it.key0 + i * kTileKeys, m, z);
-      }
-      tile += it.ntiles;
-      // publish this warpgroup's (max, sum) partial of the chunk: entry
-      // [t][wg][lrow] of rows PR = 128 (two row groups) or R_pad (one)
-      if (row < p.R_pad)
-        p.part[(static_cast<size_t>(t) * kSoftmaxWGs + wg) * PR + lrow] = make_float2(m, z);
-      __threadfence();
-      named_bar_sync(bar_id, 128);
-      if (wtid == 0) {
-        const int old = atomicAdd(&p.cnt[it.u], 1);
-        __threadfence();
-        sm.flag[wg] = (old == kSoftmaxWGs * it.nchunks - 1);
-      }
-      named_bar_sync(bar_id, 128);
-      if (sm.flag[wg]) {
-        // Last arrival for this unit: merge every chunk's partials of each row
-        // into lse2 = M + log2(Z), one pass, eight independent loads in flight.
-        for (int r = wtid; r < p.R_pad; r += 128) {
-          // entries of row r: one per warpgroup and chunk, of which only the
-          // two warpgroups of r's row group wrote when nh = 2
-          const int per_chunk = nh == 2 ? 2 : kSoftmaxWGs;
-          const int nq = per_chunk * it.nchunks;
-          const float2* base =
-              p.part + static_cast<size_t>(it.cs) * kSoftmaxWGs * PR + (nh == 2 ? (r & 127) : r);
-          float M = -INFINITY, Z = 0.f;
-          for (int q0 = 0; q0 < nq; q0 += 8) {
-            float2 e[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int q = q0 + i;
-              // chunk q / per_chunk, warpgroup: nh=2 -> (r >> 7) + 2*(q & 1); nh=1 -> q & 3
-              const int w = nh == 2 ? ((r >> 7) + 2 * (q & 1)) : (q & 3);
-              e[i] = q < nq ? __ldcg(&base[(static_cast<size_t>(q / per_chunk) * kSoftmaxWGs + w) * PR])
-                            : make_float2(-INFINITY, 0.f);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              if (e[i].x == -INFINITY) continue;
-              if (e[i].x > M) {
-                Z = Z * ex2_approx(M - e[i].x) + e[i].y;
-                M = e[i].x;
-              } else {
-                Z += e[i].y * ex2_approx(e[i].x - M);
-              }
-            }
+        const int k0 = it.key0 + i * kTileKeys + 32 * wg;  // this warpgroup's 32 keys
+        const bool full = k0 + 31 <= it.n - p.W;          // every key visible to every row
+        for (int h = 0; h < nh; ++h) {
+          ok = slot_wait(p, sm, g + h, ok);
+          uint32_t r[32];
+          slot_take(sm, lane_base, g + h, r);
+          const int tr = h == 0 ? tr0 : tr1;
+          if (ok && tr >= 0) {
+            if (h == 0) s1_chunk(r, p.scale_log2, full, k0, tr, m0, z0);
+            else s1_chunk(r, p.scale_log2, full, k0, tr, m1, z1);
           }
-          p.lam[static_cast<size_t>(it.u) * p.R_pad + r] =
-              (M == -INFINITY || Z <= 0.f) ? INFINITY : M + lg2_approx(Z);
         }
-        __threadfence();
-        named_bar_sync(bar_id, 128);
-        if (wtid == 0 && it.u != p.stall_unit) st_release(&p.ready[it.u], 1);
+        g += nh;
       }
+      // hand the four warpgroups' (max, sum) of each row to the publisher warp
+      if (!wait_bar(&sm.pempty[0], (q1 & 1) ^ 1, p)) ok = false;
+      if (lrow < p.R_pad) sm.pc[wg * p.R_pad + lrow] = make_float2(m0, z0);
+      if (nh == 2 && 128 + lrow < p.R_pad) sm.pc[wg * p.R_pad + 128 + lrow] = make_float2(m1, z1);
+      mbar_arrive(&sm.pfull[0]);
+      ++q1;
     }
-    // ---------------- sweep 2 of item j-1 ----------------
-    if (j > 0) {
-      const int t = first + (j - 1) * stride;
+    // ---------------- sweep 2 ----------------
+    else {
+      const int t = first + jj * stride;
       const ItemInfo it = decode_item(p, t, load_item(p, t));
-      if (wtid == 0) {
-        int ready = ld_acquire(&p.ready[it.u]);
-        if (!ready) {
-          const uint64_t t0 = globaltimer_ns();
-          uint32_t spins = 0;
-          while (!(ready = ld_acquire(&p.ready[it.u]))) {
-            __nanosleep(64);
-            if ((++spins & 15u) == 0) {
-              if (ld_volatile(p.abort_flag)) break;
-              if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
-                atomicExch(p.abort_flag, 1);
-                atomicOr(p.status, kStatusTimeout);
-                break;
-              }
-            }
-          }
-        }
-        sm.flag[4 + wg] = ready;
-      }
-      named_bar_sync(bar_id, 128);
-      const bool have = sm.flag[4 + wg] != 0;
-      for (int r = r0 + wtid; r < r0 + nch * 32; r += 128)  // stored negated: exp2(s*c + (-lse2))
-        nlam[r] = have ? -__ldcg(&p.lam[static_cast<size_t>(it.u) * p.R_pad + r]) : -INFINITY;
-      named_bar_sync(bar_id, 128);
-      float* out = raw_out + static_cast<size_t>(it.u) * p.S_cap;
-      for (int i = 0; i < it.ntiles; ++i) {
-        const uint32_t gt = tile + i;
-        if ((gt & tmask) != tres) continue;
+      // -lse2 of the unit, loaded ahead by the normaliser warp
+      const uint32_t lb = q2 & 1;
+      if (!wait_bar(&sm.lfull[lb], (q2 >> 1) & 1, p)) ok = false;
+      const float* lam = sm.lam + lb * p.R_pad;
+      float* out = p.raw + static_cast<size_t>(it.u) * p.S_cap;
+      for (int i = 0; i < it.ntiles; ++i, ++tc) {
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
+        const bool key_full = kb + kTileKeys - 1 <= it.n - p.W;
         float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        s2_slot(p, sm, lane_addr, gt * nh + half, ok, nch, r0, k, it.n, kb, nlam, a);
-        if (ok && k < it.n) out[k] = sum8(a) * p.inv_G;
+        ok = slot_wait(p, sm, g, ok);
+        if (nh == 2) ok = slot_wait(p, sm, g + 1, ok);
+        {
+          uint32_t r[32];
+          slot_take(sm, lane_base, g, r);
+          if (ok && has_a && k < it.n)
+            s2_chunk(p, r, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
+        }
+        if (nh == 2) {
+          uint32_t r[32];
+          slot_take(sm, lane_base, g + 1, r);
+          if (ok && has_b && k < it.n)
+            s2_chunk(p, r, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
+        }
+        g += nh;
+        // sum the four warpgroups' partials of each key; warpgroup tc mod 4 writes
+        float* red = sm.red + (tc & 1) * (kSoftmaxWGs * 128);
+        red[wg * 128 + lrow] = sum8(a);
+        named_bar_sync(1, 128 * kSoftmaxWGs);
+        if (wg == static_cast<int>(tc % kSoftmaxWGs) && ok && k < it.n) {
+          float sum = 0.f;
+#pragma unroll
+          for (int w = 0; w < kSoftmaxWGs; ++w) sum += red[w * 128 + lrow];
+          out[k] = sum * p.inv_G;
+        }
       }
-      tile += it.ntiles;
+      // every thread has passed the last tile's barrier: nobody reads the buffer any more
+      if (stid == 0) mbar_arrive(&sm.lempty[lb]);
+      ++q2;
     }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Publisher warp: for each sweep-1 entry, merge the four warpgroups' (max,
+// sum) of every row into one record of the chunk, count the chunk in, and if
+// it is the unit's last, merge every chunk's record into the unit's lse2 and
+// release it.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 merge_ms(float2 a, float2 e) {  // (max, sum) in base 2
+  if (e.x == -INFINITY) return a;
+  if (e.x > a.x) return make_float2(e.x, a.y * ex2_approx(a.x - e.x) + e.y);
+  return make_float2(a.x, a.y + e.y * ex2_approx(e.x - a.x));
+}
+
+__device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
+  const int lane = threadIdx.x & 31;
+  uint32_t q1 = 0;
+  EntryIter ei(J);
+  int jj, sw;
+  while (ei.next(jj, sw)) {
+    if (sw != 0) continue;
+    const int t = first + jj * stride;
+    const ItemInfo it = decode_item(p, t, load_item(p, t));
+    if (!wait_bar_warp(&sm.pfull[0], q1 & 1, p)) return;
+    float2* rec = p.part + static_cast<size_t>(t) * p.R_pad;
+    for (int r = lane; r < p.R_pad; r += 32) {
+      float2 a = make_float2(-INFINITY, 0.f);
+#pragma unroll
+      for (int w = 0; w < kSoftmaxWGs; ++w) a = merge_ms(a, sm.pc[w * p.R_pad + r]);
+      rec[r] = a;
+    }
+    __syncwarp();
+    mbar_arrive_elect(&sm.pempty[0]);  // pc may be overwritten
+    ++q1;
+    __threadfence();
+    __syncwarp();
+    int last = 0;
+    if (lane == 0) {
+      last = atomicAdd(&p.cnt[it.u], 1) == it.nchunks - 1;
+      __threadfence();
+    }
+    last = __shfl_sync(0xffffffffu, last, 0);
+    if (!last) continue;
+    // Last chunk of the unit: lse2 = M + log2(Z) over every chunk's record,
+    // eight independent loads in flight per lane.
+    const float2* base = p.part + static_cast<size_t>(it.cs) * p.R_pad;
+    for (int r = lane; r < p.R_pad; r += 32) {
+      float2 a = make_float2(-INFINITY, 0.f);
+      for (int q0 = 0; q0 < it.nchunks; q0 += 8) {
+        float2 e[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          e[i] = q0 + i < it.nchunks ? __ldcg(&base[static_cast<size_t>(q0 + i) * p.R_pad + r])
+                                     : make_float2(-INFINITY, 0.f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a = merge_ms(a, e[i]);
+      }
+      p.lam[static_cast<size_t>(it.u) * p.R_pad + r] =
+          (a.x == -INFINITY || a.y <= 0.f) ? INFINITY : a.x + lg2_approx(a.y);
+    }
+    __threadfence();
+    __syncwarp();
+    if (lane == 0 && it.u != p.stall_unit) st_release(&p.ready[it.u], 1);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Normaliser warp: for each sweep-2 entry, wait for the unit's lse2 (bounded)
+// and copy -lse2 into the entry's lam buffer ahead of the softmax warpgroups.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void lam_loader(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
+  const int lane = threadIdx.x & 31;
+  uint32_t q2 = 0;
+  EntryIter ei(J);
+  int jj, sw;
+  while (ei.next(jj, sw)) {
+    if (sw != 1) continue;
+    const int t = first + jj * stride;
+    const ItemInfo it = decode_item(p, t, load_item(p, t));
+    const uint32_t lb = q2 & 1;
+    if (!wait_bar_warp(&sm.lempty[lb], ((q2 >> 1) & 1) ^ 1, p)) return;
+    int ready = 0;
+    if (lane == 0) {
+      const uint64_t t0 = globaltimer_ns();
+      uint32_t spins = 0;
+      while (!(ready = ld_acquire(&p.ready[it.u]))) {
+        __nanosleep(64);
+        if ((++spins & 15u) == 0) {
+          if (ld_volatile(p.abort_flag)) break;
+          if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
+            atomicExch(p.abort_flag, 1);
+            atomicOr(p.status, kStatusTimeout);
+            break;
+          }
+        }
+      }
+    }
+    ready = __shfl_sync(0xffffffffu, ready, 0);
+    __syncwarp();  // the other lanes read lse2 after lane 0's acquire
+    float* lam = sm.lam + lb * p.R_pad;
+    for (int r = lane; r < p.R_pad; r += 32)  // stored negated: exp2(s*c + (-lse2))
+      lam[r] = ready ? -__ldcg(&p.lam[static_cast<size_t>(it.u) * p.R_pad + r]) : -INFINITY;
+    __syncwarp();
+    mbar_arrive_elect(&sm.lfull[lb]);
+    ++q2;
+    if (!ready) return;
   }
 }
 
@@ -583,9 +675,15 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     }
     for (int i = 0; i < kSlots; ++i) {
       mbar_init(&sm.tfull[i], 1);
-      mbar_init(&sm.tempty[i], 128);  // the 128 threads of the warpgroup that owns the tile
+      mbar_init(&sm.tempty[i], 128 * kSoftmaxWGs);  // every softmax thread copies its slice
     }
     mbar_init(sm.done, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.lfull[i], 1);
+      mbar_init(&sm.lempty[i], 1);
+    }
+    mbar_init(sm.pfull, 128 * kSoftmaxWGs);
+    mbar_init(sm.pempty, 1);
     fence_barrier_init();
     fence_proxy_async();
   }
@@ -606,6 +704,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     regs_dealloc<kRegsControl>();
     if (warp == 0 && (threadIdx.x & 31) == 0) producer<D>(p, sm, first, stride, J);
     if (warp == 1) mma_issuer<D>(p, sm, tmem_base, first, stride, J);  // whole warp
+    if (warp == 2) publisher(p, sm, first, stride, J);                 // whole warp
+    if (warp == 3) lam_loader(p, sm, first, stride, J);                // whole warp
   } else {
     regs_alloc<kRegsSoftmax>();
     softmax_wg(p, sm, tmem_base, (warp - 4) >> 2, first, stride, J);  // warpgroups 0..3
@@ -692,13 +792,8 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
 }  // namespace
 
 int score_smem_bytes(int d, int q_rows, int R_pad, int stages) {
-  size_t off = 0;
-  off += 2 * static_cast<size_t>(q_rows) * d * 2;
-  off += static_cast<size_t>(stages) * kTileKeys * d * 2;
-  off += kSoftmaxWGs * sizeof(float) * R_pad;
-  off = (off + 7) & ~size_t(7);
-  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1);
-  off += sizeof(uint32_t) + 8 * sizeof(int);
+  size_t koff, loff, roff, poff, boff;
+  const size_t off = smem_size(d, q_rows, R_pad, stages, &koff, &loff, &roff, &poff, &boff);
   return static_cast<int>((off + 127) & ~size_t(127));
 }
 

@@ -182,25 +182,13 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
     for (int j = threadIdx.x; j < n; j += blockDim.x) idx[j] = j;
   for (int j = count + threadIdx.x; j < b; j += blockDim.x) idx[j] = -1;
   if (threadIdx.x == 0) *cnt = count;
-  float* raw = ld.score_slot < 0 ? nullptr
-                                 : p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) *
-                                               static_cast<size_t>(p.S_cap);
-  // Units the score kernel visited (every H2O unit, SnapKV units it must cut)
-  // hold each score as two partial sums when the window has two 128-row
-  // groups: add them in place, so the scores seen below, the H2O state and
-  // the scores view are complete.
-  const bool scored = ld.method == KVEV_H2O ? n > 0 : (ld.method == KVEV_SNAPKV && n > b);
-  if (scored && p.raw1 != nullptr) {
-    const float* raw1 =
-        p.raw1 + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
-    for (int j = threadIdx.x; j < n; j += blockDim.x) raw[j] += __ldcs(raw1 + j);
-    __syncthreads();  // pooling below reads neighbours written by other threads
-  }
   if (identity || ld.method == KVEV_STREAMING) return;
 
   // protected tail [E, n) occupies slots k .. count-1
   for (int j = threadIdx.x; j < n - E; j += blockDim.x) idx[k + j] = E + j;
   if (k == 0) return;
+  const float* raw =
+      p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
   build_keys(keys, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV);
   __syncthreads();
   if (k >= E) {
