@@ -449,6 +449,20 @@ __device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, ui
   mbar_arrive(&sm.tempty[sl]);
 }
 
+// Both slots of a tile (g, g + 1) in one round trip: two loads in flight, one
+// wait, both released before any arithmetic.
+__device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r0)[32],
+                                           uint32_t (&r1)[32]) {
+  const uint32_t s0 = g & (kSlots - 1), s1 = (g + 1) & (kSlots - 1);
+  tmem_ld32_async(lane_base + s0 * kSlotCols, r0);
+  tmem_ld32_async(lane_base + s1 * kSlotCols, r1);
+  tmem_wait32(r0);
+  tmem_wait32(r1);
+  tc_fence_before();
+  mbar_arrive(&sm.tempty[s0]);
+  mbar_arrive(&sm.tempty[s1]);
+}
+
 __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base,
                                            int wg, int first, int stride, int J) {
   const int warp = threadIdx.x >> 5;
@@ -482,15 +496,18 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int i = 0; i < it.ntiles; ++i) {
         const int k0 = it.key0 + i * kTileKeys + 32 * wg;  // this warpgroup's 32 keys
         const bool full = k0 + 31 <= it.n - p.W;          // every key visible to every row
-        for (int h = 0; h < nh; ++h) {
-          ok = slot_wait(p, sm, g + h, ok);
-          uint32_t r[32];
-          slot_take(sm, lane_base, g + h, r);
-          const int tr = h == 0 ? tr0 : tr1;
-          if (ok && tr >= 0) {
-            if (h == 0) s1_chunk(r, p.scale_log2, full, k0, tr, m0, z0);
-            else s1_chunk(r, p.scale_log2, full, k0, tr, m1, z1);
-          }
+        if (nh == 2) {
+          ok = slot_wait(p, sm, g, ok);
+          ok = slot_wait(p, sm, g + 1, ok);
+          uint32_t r0[32], r1[32];
+          slot_take2(sm, lane_base, g, r0, r1);
+          if (ok && tr0 >= 0) s1_chunk(r0, p.scale_log2, full, k0, tr0, m0, z0);
+          if (ok && tr1 >= 0) s1_chunk(r1, p.scale_log2, full, k0, tr1, m1, z1);
+        } else {
+          ok = slot_wait(p, sm, g, ok);
+          uint32_t r0[32];
+          slot_take(sm, lane_base, g, r0);
+          if (ok && tr0 >= 0) s1_chunk(r0, p.scale_log2, full, k0, tr0, m0, z0);
         }
         g += nh;
       }
@@ -517,17 +534,18 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         ok = slot_wait(p, sm, g, ok);
         if (nh == 2) ok = slot_wait(p, sm, g + 1, ok);
-        {
-          uint32_t r[32];
-          slot_take(sm, lane_base, g, r);
-          if (ok && has_a && k < it.n)
-            s2_chunk(p, r, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
-        }
         if (nh == 2) {
-          uint32_t r[32];
-          slot_take(sm, lane_base, g + 1, r);
+          uint32_t ra[32], rb[32];
+          slot_take2(sm, lane_base, g, ra, rb);
+          if (ok && has_a && k < it.n)
+            s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
           if (ok && has_b && k < it.n)
-            s2_chunk(p, r, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
+            s2_chunk(p, rb, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
+        } else {
+          uint32_t ra[32];
+          slot_take(sm, lane_base, g, ra);
+          if (ok && has_a && k < it.n)
+            s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
         }
         g += nh;
         // sum the four warpgroups' partials of each key; warpgroup tc mod 4 writes
