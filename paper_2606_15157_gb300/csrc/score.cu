@@ -50,6 +50,8 @@ struct Smem {
   uint64_t* lempty;  // [2] lam buffer read by the softmax warpgroups
   uint64_t* pfull;   // partials of a sweep-1 entry written to pc by the softmax threads
   uint64_t* pempty;  // pc read by the publisher warp
+  uint64_t* rfull;   // [2] red buffer holds the four warpgroups' partials of a tile
+  uint64_t* rempty;  // [2] red buffer read by the tile's writer warpgroup
   uint64_t* kfull;
   uint64_t* kempty;
   uint64_t* qfull;
@@ -75,7 +77,7 @@ __host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int R_pa
   *poff = off;
   off += sizeof(float2) * kSoftmaxWGs * R_pad;
   *boff = off;
-  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6);
+  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6 + 4);
   off += sizeof(uint32_t) + 2 * sizeof(int);
   return off;
 }
@@ -102,7 +104,9 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   s.lempty = s.lfull + 2;
   s.pfull = s.lempty + 2;
   s.pempty = s.pfull + 1;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.pempty + 1);
+  s.rfull = s.pempty + 1;
+  s.rempty = s.rfull + 2;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.rempty + 2);
   s.flag = reinterpret_cast<int*>(s.tmem_slot + 1);
   return s;
 }
@@ -548,18 +552,27 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
         }
         g += nh;
-        // sum the four warpgroups' partials of each key; warpgroup tc mod 4 writes
-        float* red = sm.red + (tc & 1) * (kSoftmaxWGs * 128);
+        // Sum the four warpgroups' partials of each key: every warpgroup
+        // deposits its partial in buffer tc mod 2 and moves on; warpgroup
+        // tc mod 4 waits for the other three, writes the sum and frees the buffer.
+        const uint32_t rb = tc & 1, rph = (tc >> 1) & 1;
+        float* red = sm.red + rb * (kSoftmaxWGs * 128);
+        if (!wait_bar(&sm.rempty[rb], rph ^ 1, p)) ok = false;
         red[wg * 128 + lrow] = sum8(a);
-        named_bar_sync(1, 128 * kSoftmaxWGs);
-        if (wg == static_cast<int>(tc % kSoftmaxWGs) && ok && k < it.n) {
-          float sum = 0.f;
+        mbar_arrive(&sm.rfull[rb]);
+        if (wg == static_cast<int>(tc % kSoftmaxWGs)) {
+          if (!wait_bar(&sm.rfull[rb], rph, p)) ok = false;
+          if (ok && k < it.n) {
+            float sum = 0.f;
 #pragma unroll
-          for (int w = 0; w < kSoftmaxWGs; ++w) sum += red[w * 128 + lrow];
-          out[k] = sum * p.inv_G;
+            for (int w = 0; w < kSoftmaxWGs; ++w) sum += red[w * 128 + lrow];
+            out[k] = sum * p.inv_G;
+          }
+          mbar_arrive(&sm.rempty[rb]);
         }
       }
-      // every thread has passed the last tile's barrier: nobody reads the buffer any more
+      // every warpgroup is done reading lam once all have passed this barrier
+      named_bar_sync(1, 128 * kSoftmaxWGs);
       if (stid == 0) mbar_arrive(&sm.lempty[lb]);
       ++q2;
     }
@@ -702,6 +715,10 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     }
     mbar_init(sm.pfull, 128 * kSoftmaxWGs);
     mbar_init(sm.pempty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.rfull[i], 128 * kSoftmaxWGs);
+      mbar_init(&sm.rempty[i], 128);  // the writer warpgroup
+    }
     fence_barrier_init();
     fence_proxy_async();
   }
