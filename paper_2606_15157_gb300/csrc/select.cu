@@ -21,23 +21,64 @@ namespace kvev {
 
 namespace {
 
-// Per-unit scores (or pooled scores) into order-preserving keys in shared memory.
+// Per-unit scores (or pooled scores) into order-preserving keys in shared
+// memory.  Every load of a key's window is issued before any is used, four
+// keys per thread at a time (the window reads of neighbouring keys overlap
+// and are served by L1), so the latency of the score reads is paid once per
+// group of keys rather than once per window element.
+template <int P>
+__device__ __forceinline__ void build_keys_pooled(uint32_t* keys, const float* raw, int E, bool is_max) {
+  constexpr int h = P / 2;
+  constexpr int U = 4;
+  for (int i0 = threadIdx.x; i0 < E; i0 += U * blockDim.x) {
+    float w[U][P];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+#pragma unroll
+      for (int j = 0; j < P; ++j) {
+        const int q = i - h + j;
+        w[u][j] = (i < E && q >= 0 && q < E) ? raw[q] : (is_max ? -INFINITY : 0.f);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i >= E) break;
+      float v = w[u][0];
+#pragma unroll
+      for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[u][j]) : v + w[u][j];
+      keys[i] = float_key(is_max ? v : v / static_cast<float>(P));
+    }
+  }
+}
+
 __device__ void build_keys(uint32_t* keys, const float* raw, int E, int pool, int pool_type,
                            bool do_pool) {
+  const bool is_max = pool_type == KVEV_POOL_MAX;
+  if (do_pool) {
+    switch (pool) {  // common widths with fully unrolled windows
+      case 3: build_keys_pooled<3>(keys, raw, E, is_max); return;
+      case 5: build_keys_pooled<5>(keys, raw, E, is_max); return;
+      case 7: build_keys_pooled<7>(keys, raw, E, is_max); return;
+      case 9: build_keys_pooled<9>(keys, raw, E, is_max); return;
+      default: break;
+    }
+  }
   const int h = pool / 2;
   for (int i = threadIdx.x; i < E; i += blockDim.x) {
     float v;
     if (!do_pool) {
       v = raw[i];
-    } else if (pool_type == KVEV_POOL_MAX) {
+    } else if (is_max) {
       v = -INFINITY;
       const int lo = max(i - h, 0), hi = min(i + h, E - 1);
       for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
     } else {
-      float s = 0.f;
+      float sum = 0.f;
       const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-      for (int j = lo; j <= hi; ++j) s += raw[j];
-      v = s / static_cast<float>(pool);
+      for (int j = lo; j <= hi; ++j) sum += raw[j];
+      v = sum / static_cast<float>(pool);
     }
     keys[i] = float_key(v);
   }
