@@ -31,7 +31,7 @@ constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 51
 constexpr int kRegsControl = 64;
 constexpr int kRegsSoftmax = 104;
 constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
-constexpr int kSelectThreads = 512;
+constexpr int kSelectThreads = 1024;
 constexpr int kWsAlign = 256;
 
 // Bits of the device status word.
