@@ -58,7 +58,7 @@ bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 
 struct WsLayout {
   int n_units = 0, R = 0, R_pad = 0, max_items = 0;
-  size_t lens = 0, abort_flag = 0, cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
+  size_t lens = 0, abort_flag = 0, node_cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
          lam = 0, raw = 0, total = 0;
 };
 
@@ -77,7 +77,7 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   };
   w.lens = take(sizeof(int) * std::max(B, 1));
   w.abort_flag = take(sizeof(int));
-  w.cnt = take(sizeof(int) * std::max(w.n_units, 1));
+  w.node_cnt = take(sizeof(int) * static_cast<size_t>(std::max(w.max_items, 1)) * kTreeLevels);
   w.ready = take(sizeof(int) * std::max(w.n_units, 1));
   w.chunk_start = take(sizeof(int) * (w.n_units + 1));
   w.item = take(sizeof(int4) * std::max(w.max_items, 1));
@@ -501,6 +501,10 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   const int tiles_max = (S_cap + kTileKeys - 1) / kTileKeys;
   const int chunk_tiles = std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid);
   if (chunk_tiles > 0xFFFF) return KVEV_ENOTSUP;  // tiles per item are packed in 16 bits
+  // the normaliser's merge tree has kTreeLevels internal levels of fan-in kTreeFanIn
+  int leaves = 1;
+  for (int i = 0; i < kTreeLevels; ++i) leaves *= kTreeFanIn;
+  if ((tiles_max + chunk_tiles - 1) / chunk_tiles > leaves) return KVEV_ENOTSUP;
   PrologueParams pp = {};
   pp.n_units = ws.n_units;
   pp.B = B;
@@ -514,7 +518,8 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   pp.lens = lens_ok;
   pp.S_cap = S_cap;
   pp.status = D.status;
-  pp.cnt = reinterpret_cast<int*>(wsb + ws.cnt);
+  pp.node_cnt = reinterpret_cast<int*>(wsb + ws.node_cnt);
+  pp.n_node_cnt = std::max(ws.max_items, 1) * kTreeLevels;
   pp.ready = reinterpret_cast<int*>(wsb + ws.ready);
   pp.abort_flag = reinterpret_cast<int*>(wsb + ws.abort_flag);
   pp.chunk_start = reinterpret_cast<int*>(wsb + ws.chunk_start);
@@ -578,7 +583,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.lens = lens_ok;
     sp.chunk_start = pp.chunk_start;
     sp.item = pp.item;
-    sp.cnt = pp.cnt;
+    sp.node_cnt = pp.node_cnt;
     sp.ready = pp.ready;
     sp.abort_flag = pp.abort_flag;
     sp.status = D.status;

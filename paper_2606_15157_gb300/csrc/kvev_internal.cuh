@@ -19,8 +19,13 @@ constexpr int kTileKeys = 128;        // keys per tensor-core tile (MMA M or N)
 // merge; the cost is reuse distance (grid * chunk bytes between a tile's two
 // reads, ~78 MB at 16 tiles on 152 SMs, inside the 126 MB L2).
 constexpr int kMinChunkTiles = 16;
-constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel (one per TMEM slot)
-constexpr int kScoreThreads = 128 * (1 + kSoftmaxWGs);  // + warpgroup 0: TMA warp, MMA warp, 2 idle
+// The per-row (max, sum) records of a unit's chunks are merged up a tree of
+// fan-in kTreeFanIn (the last child to arrive merges its siblings), so the
+// normaliser is ready a few load round trips after the unit's last chunk.
+constexpr int kTreeFanIn = 4;
+constexpr int kTreeLevels = 5;        // internal levels: up to 4^5 = 1024 chunks per unit
+constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel
+constexpr int kScoreThreads = 128 * (1 + kSoftmaxWGs);  // + warpgroup 0: TMA, MMA, publisher, normaliser warps
 constexpr int kSlots = 4;             // TMEM accumulator slots of the score kernel
 constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 512 columns)
 // Register split of the score kernel (setmaxnreg): warpgroup 0 shrinks to 64,
@@ -57,7 +62,8 @@ struct PrologueParams {
   const int* lens_in; // caller's lengths
   int* lens;          // validated copy (out-of-range lengths become 0, flagged)
   int* status;
-  int* cnt;
+  int* node_cnt;      // [items][kTreeLevels] arrival counters of the merge tree (zeroed here)
+  int n_node_cnt;     // counters in node_cnt (workspace capacity)
   int* ready;
   int* abort_flag;
   int* chunk_start;   // [n_units + 1]
@@ -76,11 +82,12 @@ struct ScoreParams {
   const int* lens;
   const int* chunk_start;
   const int4* item;   // [items] {unit, n, first key, tiles | chunks of the unit << 16}
-  int* cnt;
+  int* node_cnt;      // [items][kTreeLevels]: counter of the tree node whose first leaf is the item
   int* ready;
   int* abort_flag;
   int* status;
-  float2* part;       // [items][R_pad] per-row (max, sum) of each chunk, base-2 units
+  float2* part;       // [items][R_pad] per-row (max, sum) of a chunk, or of the tree node
+                      // whose first leaf is that chunk, base-2 units
   float* lam;         // [n_units][R_pad] per-row log2-sum-exp
   float* raw;         // [n_units][S_cap] window scores
   long long wait_ns;
@@ -363,6 +370,17 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
   asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
   asm("mov.b64 %0, {%1, %2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
+  float2 d;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+
+// Two-lane packed fp32 add.
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  uint64_t ra, rb, rd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
   float2 d;
   asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
   return d;

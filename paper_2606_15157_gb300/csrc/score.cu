@@ -369,41 +369,42 @@ __device__ __forceinline__ float max32(const float (&v)[32]) {
   return fmax3(b, c, e);
 }
 
-__device__ __forceinline__ float sum8(const float (&a)[8]) {
-  return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+__device__ __forceinline__ float sum4x2(const float2 (&a)[4]) {
+  const float2 s = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
+  return s.x + s.y;
+}
+
+// Keys of a 32-key chunk that row position tr cannot see are set to -inf.
+__device__ __forceinline__ void mask_chunk(float (&v)[32], int k0, int tr) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    if (k0 + i > tr) v[i] = -INFINITY;
 }
 
 // One 32-key chunk of sweep 1 for one row: online base-2 (max, sum) update.
-__device__ __forceinline__ void s1_chunk(const uint32_t (&rr)[32], float c, bool full, int k0,
-                                         int tr, float& m, float& z) {
-  float v[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(rr[i]);
-  if (!full) {
-#pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if (k0 + i > tr) v[i] = -INFINITY;
-  }
-  const float mx = max32(v);
-  if (mx == -INFINITY) return;
-  const float mnew = fmaxf(m, mx * c);
-  const float zs = z * ex2_approx(m - mnew);  // m = -inf -> 0
-  const float2 cc = make_float2(c, c), nm = make_float2(-mnew, -mnew);
-  float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+// Branch-free, so the two rows a thread holds interleave: a row with no
+// visible key yet (m = -inf) offsets its exponents by 0 instead, where every
+// term is exp2(-inf) = 0.
+__device__ __forceinline__ void s1_chunk(const float (&v)[32], float c, float& m, float& z) {
+  const float mnew = fmaxf(m, max32(v) * c);
+  const float base = mnew == -INFINITY ? 0.f : mnew;
+  const float zs = z * ex2_approx(m - base);  // m = -inf -> 0
+  const float2 cc = make_float2(c, c), nb = make_float2(-base, -base);
+  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
 #pragma unroll
   for (int i = 0; i < 32; i += 2) {
-    const float2 t = ffma2(make_float2(v[i], v[i + 1]), cc, nm);
-    a[i & 7] += ex2_approx(t.x);
-    a[(i + 1) & 7] += ex2_approx(t.y);
+    const float2 t = ffma2(make_float2(v[i], v[i + 1]), cc, nb);
+    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t.x), ex2_approx(t.y)));
   }
-  z = zs + sum8(a);
+  z = zs + sum4x2(a);
   m = mnew;
 }
 
 // One 32-row chunk of sweep 2 for this thread's key: sum of exp2(s*c - lse2_r)
-// into eight accumulators; nl = -lse2 of the chunk's rows (shared memory).
+// into four packed accumulators; nl = -lse2 of the chunk's rows (shared memory).
 __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&rr)[32], bool full,
-                                         const float* nl, int r0, int k, int n, float (&a)[8]) {
+                                         const float* nl, int r0, int k, int n, float2 (&a)[4]) {
   const float c = p.scale_log2;
   const float2 cc = make_float2(c, c);
   if (full) {
@@ -414,17 +415,18 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
                               make_float2(l4.x, l4.y));
       const float2 t1 = ffma2(make_float2(__uint_as_float(rr[i + 2]), __uint_as_float(rr[i + 3])),
                               cc, make_float2(l4.z, l4.w));
-      a[i & 7] += ex2_approx(t0.x);
-      a[(i + 1) & 7] += ex2_approx(t0.y);
-      a[(i + 2) & 7] += ex2_approx(t1.x);
-      a[(i + 3) & 7] += ex2_approx(t1.y);
+      a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+      a[((i >> 1) + 1) & 3] =
+          fadd2(a[((i >> 1) + 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
     }
   } else {
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       const int r = r0 + i;
-      if (r < p.R && k <= row_pos(p, r, n))
-        a[i & 7] += ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
+      if (r < p.R && k <= row_pos(p, r, n)) {
+        const float e = ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
+        if (i & 1) a[(i >> 1) & 3].y += e; else a[(i >> 1) & 3].x += e;
+      }
     }
   }
 }
@@ -432,9 +434,10 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
 // ---- TMEM slot hand-off --------------------------------------------------
 // Every fill is consumed by all four softmax warpgroups: warpgroup w copies
 // its 32-column slice [32w, 32w + 32) of the slot and releases the slot at
-// once (the slot's empty barrier counts all 512 softmax threads), so the
-// tensor core refills a slot as soon as the last slice is copied and no
-// warpgroup holds a slot while it computes.
+// once (the slot's empty barrier counts the 16 softmax warps: one elected lane
+// arrives for its warp, as a shared-memory barrier takes its arrivals one at a
+// time), so the tensor core refills a slot as soon as the last slice is copied
+// and no warpgroup holds a slot while it computes.
 
 __device__ __forceinline__ bool slot_wait(const ScoreParams& p, const Smem& sm, uint32_t g, bool ok) {
   if (ok && !wait_bar(&sm.tfull[g & (kSlots - 1)], (g / kSlots) & 1, p)) ok = false;
@@ -450,7 +453,8 @@ __device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, ui
   tmem_ld32_async(lane_base + sl * kSlotCols, r);
   tmem_wait32(r);
   tc_fence_before();
-  mbar_arrive(&sm.tempty[sl]);
+  __syncwarp();
+  mbar_arrive_elect(&sm.tempty[sl]);
 }
 
 // Both slots of a tile (g, g + 1) in one round trip: two loads in flight, one
@@ -463,8 +467,9 @@ __device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, u
   tmem_wait32(r0);
   tmem_wait32(r1);
   tc_fence_before();
-  mbar_arrive(&sm.tempty[s0]);
-  mbar_arrive(&sm.tempty[s1]);
+  __syncwarp();
+  mbar_arrive_elect(&sm.tempty[s0]);
+  mbar_arrive_elect(&sm.tempty[s1]);
 }
 
 __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base,
@@ -500,26 +505,45 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int i = 0; i < it.ntiles; ++i) {
         const int k0 = it.key0 + i * kTileKeys + 32 * wg;  // this warpgroup's 32 keys
         const bool full = k0 + 31 <= it.n - p.W;          // every key visible to every row
+        // Rows of a slot that do not exist (tr < 0) are computed like the
+        // others and dropped when the warpgroup publishes.
         if (nh == 2) {
           ok = slot_wait(p, sm, g, ok);
           ok = slot_wait(p, sm, g + 1, ok);
           uint32_t r0[32], r1[32];
           slot_take2(sm, lane_base, g, r0, r1);
-          if (ok && tr0 >= 0) s1_chunk(r0, p.scale_log2, full, k0, tr0, m0, z0);
-          if (ok && tr1 >= 0) s1_chunk(r1, p.scale_log2, full, k0, tr1, m1, z1);
+          float v0[32], v1[32];
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            v0[q] = __uint_as_float(r0[q]);
+            v1[q] = __uint_as_float(r1[q]);
+          }
+          if (!full) {
+            mask_chunk(v0, k0, tr0);
+            mask_chunk(v1, k0, tr1);
+          }
+          s1_chunk(v0, p.scale_log2, m0, z0);
+          s1_chunk(v1, p.scale_log2, m1, z1);
         } else {
           ok = slot_wait(p, sm, g, ok);
           uint32_t r0[32];
           slot_take(sm, lane_base, g, r0);
-          if (ok && tr0 >= 0) s1_chunk(r0, p.scale_log2, full, k0, tr0, m0, z0);
+          float v0[32];
+#pragma unroll
+          for (int q = 0; q < 32; ++q) v0[q] = __uint_as_float(r0[q]);
+          if (!full) mask_chunk(v0, k0, tr0);
+          s1_chunk(v0, p.scale_log2, m0, z0);
         }
         g += nh;
       }
       // hand the four warpgroups' (max, sum) of each row to the publisher warp
       if (!wait_bar(&sm.pempty[0], (q1 & 1) ^ 1, p)) ok = false;
-      if (lrow < p.R_pad) sm.pc[wg * p.R_pad + lrow] = make_float2(m0, z0);
-      if (nh == 2 && 128 + lrow < p.R_pad) sm.pc[wg * p.R_pad + 128 + lrow] = make_float2(m1, z1);
-      mbar_arrive(&sm.pfull[0]);
+      const float2 none = make_float2(-INFINITY, 0.f);
+      if (lrow < p.R_pad) sm.pc[wg * p.R_pad + lrow] = tr0 >= 0 && ok ? make_float2(m0, z0) : none;
+      if (nh == 2 && 128 + lrow < p.R_pad)
+        sm.pc[wg * p.R_pad + 128 + lrow] = tr1 >= 0 && ok ? make_float2(m1, z1) : none;
+      __syncwarp();
+      mbar_arrive_elect(&sm.pfull[0]);
       ++q1;
     }
     // ---------------- sweep 2 ----------------
@@ -535,7 +559,8 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
         const bool key_full = kb + kTileKeys - 1 <= it.n - p.W;
-        float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                       make_float2(0.f, 0.f)};
         ok = slot_wait(p, sm, g, ok);
         if (nh == 2) ok = slot_wait(p, sm, g + 1, ok);
         if (nh == 2) {
@@ -558,8 +583,9 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         const uint32_t rb = tc & 1, rph = (tc >> 1) & 1;
         float* red = sm.red + rb * (kSoftmaxWGs * 128);
         if (!wait_bar(&sm.rempty[rb], rph ^ 1, p)) ok = false;
-        red[wg * 128 + lrow] = sum8(a);
-        mbar_arrive(&sm.rfull[rb]);
+        red[wg * 128 + lrow] = sum4x2(a);
+        __syncwarp();
+        mbar_arrive_elect(&sm.rfull[rb]);
         if (wg == static_cast<int>(tc % kSoftmaxWGs)) {
           if (!wait_bar(&sm.rfull[rb], rph, p)) ok = false;
           if (ok && k < it.n) {
@@ -568,7 +594,8 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             for (int w = 0; w < kSoftmaxWGs; ++w) sum += red[w * 128 + lrow];
             out[k] = sum * p.inv_G;
           }
-          mbar_arrive(&sm.rempty[rb]);
+          __syncwarp();
+          mbar_arrive_elect(&sm.rempty[rb]);
         }
       }
       // every warpgroup is done reading lam once all have passed this barrier
@@ -581,18 +608,23 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
 
 // ---------------------------------------------------------------------------
 // Publisher warp: for each sweep-1 entry, merge the four warpgroups' (max,
-// sum) of every row into one record of the chunk, count the chunk in, and if
-// it is the unit's last, merge every chunk's record into the unit's lse2 and
-// release it.
+// sum) of every row into the chunk's record, then climb the unit's merge tree:
+// a node's record lives in the slot of its first leaf chunk; the last of a
+// node's (up to kTreeFanIn) children to arrive merges its siblings' records
+// into its own and carries the result one level up.  Whoever completes the
+// root turns it into the unit's lse2 and releases it.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float2 merge_ms(float2 a, float2 e) {  // (max, sum) in base 2
   if (e.x == -INFINITY) return a;
-  if (e.x > a.x) return make_float2(e.x, a.y * ex2_approx(a.x - e.x) + e.y);
-  return make_float2(a.x, a.y + e.y * ex2_approx(e.x - a.x));
+  if (a.x == -INFINITY) return e;
+  const float m = fmaxf(a.x, e.x);
+  return make_float2(m, a.y * ex2_approx(a.x - m) + e.y * ex2_approx(e.x - m));
 }
 
 __device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
+  constexpr int kRowsPerLane = 8;  // R_pad <= 256
   const int lane = threadIdx.x & 31;
+  const int nr = p.R_pad >> 5;
   uint32_t q1 = 0;
   EntryIter ei(J);
   int jj, sw;
@@ -601,41 +633,66 @@ __device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, 
     const int t = first + jj * stride;
     const ItemInfo it = decode_item(p, t, load_item(p, t));
     if (!wait_bar_warp(&sm.pfull[0], q1 & 1, p)) return;
-    float2* rec = p.part + static_cast<size_t>(t) * p.R_pad;
-    for (int r = lane; r < p.R_pad; r += 32) {
-      float2 a = make_float2(-INFINITY, 0.f);
+    float2 acc[kRowsPerLane];  // rows lane + 32 i of the current tree node
 #pragma unroll
-      for (int w = 0; w < kSoftmaxWGs; ++w) a = merge_ms(a, sm.pc[w * p.R_pad + r]);
-      rec[r] = a;
+    for (int i = 0; i < kRowsPerLane; ++i) {
+      acc[i] = make_float2(-INFINITY, 0.f);
+      if (i < nr) {
+#pragma unroll
+        for (int w = 0; w < kSoftmaxWGs; ++w) acc[i] = merge_ms(acc[i], sm.pc[w * p.R_pad + lane + 32 * i]);
+      }
     }
     __syncwarp();
     mbar_arrive_elect(&sm.pempty[0]);  // pc may be overwritten
     ++q1;
-    __threadfence();
-    __syncwarp();
-    int last = 0;
-    if (lane == 0) {
-      last = atomicAdd(&p.cnt[it.u], 1) == it.nchunks - 1;
+    int c = t - it.cs;         // index of the current node within its level (a leaf: the chunk)
+    int nodes = it.nchunks;    // nodes of the current level
+    int span = 1;              // leaf chunks under a node of the current level
+    int level = 0;
+    bool root = nodes == 1;
+    while (!root) {
+      float2* rec = p.part + static_cast<size_t>(it.cs + c * span) * p.R_pad;
+#pragma unroll
+      for (int i = 0; i < kRowsPerLane; ++i)
+        if (i < nr) rec[lane + 32 * i] = acc[i];
       __threadfence();
-    }
-    last = __shfl_sync(0xffffffffu, last, 0);
-    if (!last) continue;
-    // Last chunk of the unit: lse2 = M + log2(Z) over every chunk's record,
-    // eight independent loads in flight per lane.
-    const float2* base = p.part + static_cast<size_t>(it.cs) * p.R_pad;
-    for (int r = lane; r < p.R_pad; r += 32) {
-      float2 a = make_float2(-INFINITY, 0.f);
-      for (int q0 = 0; q0 < it.nchunks; q0 += 8) {
-        float2 e[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          e[i] = q0 + i < it.nchunks ? __ldcg(&base[static_cast<size_t>(q0 + i) * p.R_pad + r])
-                                     : make_float2(-INFINITY, 0.f);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) a = merge_ms(a, e[i]);
+      __syncwarp();
+      const int c0 = c / kTreeFanIn * kTreeFanIn;  // first sibling
+      const int nchild = min(kTreeFanIn, nodes - c0);
+      int last = 0;
+      if (lane == 0) {
+        int* cnt = p.node_cnt + static_cast<size_t>(it.cs + c0 * span) * kTreeLevels + level;
+        last = atomicAdd(cnt, 1) == nchild - 1;
+        __threadfence();
       }
-      p.lam[static_cast<size_t>(it.u) * p.R_pad + r] =
-          (a.x == -INFINITY || a.y <= 0.f) ? INFINITY : a.x + lg2_approx(a.y);
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (!last) break;
+      for (int k = 0; k < nchild; ++k) {
+        if (c0 + k == c) continue;
+        const float2* sib = p.part + static_cast<size_t>(it.cs + (c0 + k) * span) * p.R_pad;
+#pragma unroll
+        for (int h = 0; h < kRowsPerLane; h += 4) {  // four loads in flight (64 registers)
+          float2 e[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            e[i] = h + i < nr ? __ldcg(&sib[lane + 32 * (h + i)]) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) acc[h + i] = merge_ms(acc[h + i], e[i]);
+        }
+      }
+      c /= kTreeFanIn;
+      nodes = (nodes + kTreeFanIn - 1) / kTreeFanIn;
+      span *= kTreeFanIn;
+      ++level;
+      root = nodes == 1;
+    }
+    if (!root) continue;
+    // The root: lse2 = M + log2(Z) per row.
+#pragma unroll
+    for (int i = 0; i < kRowsPerLane; ++i) {
+      if (i < nr)
+        p.lam[static_cast<size_t>(it.u) * p.R_pad + lane + 32 * i] =
+            (acc[i].x == -INFINITY || acc[i].y <= 0.f) ? INFINITY : acc[i].x + lg2_approx(acc[i].y);
     }
     __threadfence();
     __syncwarp();
@@ -660,11 +717,16 @@ __device__ __forceinline__ void lam_loader(const ScoreParams& p, const Smem& sm,
     if (!wait_bar_warp(&sm.lempty[lb], ((q2 >> 1) & 1) ^ 1, p)) return;
     int ready = 0;
     if (lane == 0) {
+      // Polled with a growing sleep: this warp shares an issue port with one
+      // warp of every softmax warpgroup, and a tight poll takes most of its
+      // issue slots.  The normaliser is needed two entries later, so a poll
+      // interval of a microsecond or two costs nothing.
       const uint64_t t0 = globaltimer_ns();
-      uint32_t spins = 0;
+      uint32_t spins = 0, sleep_ns = 128;
       while (!(ready = ld_acquire(&p.ready[it.u]))) {
-        __nanosleep(64);
-        if ((++spins & 15u) == 0) {
+        __nanosleep(sleep_ns);
+        if (sleep_ns < 2048) sleep_ns <<= 1;
+        if ((++spins & 7u) == 0) {
           if (ld_volatile(p.abort_flag)) break;
           if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
             atomicExch(p.abort_flag, 1);
@@ -706,18 +768,18 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     }
     for (int i = 0; i < kSlots; ++i) {
       mbar_init(&sm.tfull[i], 1);
-      mbar_init(&sm.tempty[i], 128 * kSoftmaxWGs);  // every softmax thread copies its slice
+      mbar_init(&sm.tempty[i], 4 * kSoftmaxWGs);  // every softmax warp copies its slice
     }
     mbar_init(sm.done, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sm.lfull[i], 1);
       mbar_init(&sm.lempty[i], 1);
     }
-    mbar_init(sm.pfull, 128 * kSoftmaxWGs);
+    mbar_init(sm.pfull, 4 * kSoftmaxWGs);
     mbar_init(sm.pempty, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.rfull[i], 128 * kSoftmaxWGs);
-      mbar_init(&sm.rempty[i], 128);  // the writer warpgroup
+      mbar_init(&sm.rfull[i], 4 * kSoftmaxWGs);
+      mbar_init(&sm.rempty[i], 4);  // the writer warpgroup's warps
     }
     fence_barrier_init();
     fence_proxy_async();
@@ -764,6 +826,7 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     carry = 0;
     *p.abort_flag = 0;
   }
+  for (int i = tid; i < p.n_node_cnt; i += blockDim.x) p.node_cnt[i] = 0;
   for (int s = tid; s < p.B; s += blockDim.x) {
     int n = p.lens_in[s];
     if (n < 0 || n > p.S_cap) {
@@ -783,7 +846,6 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
       const int n = p.lens[s];
       const bool need = n > 0 && (p.slayer_method[ls] == KVEV_H2O || n > p.slayer_budget[ls]);
       c = need ? (n + p.chunk_keys - 1) / p.chunk_keys : 0;
-      p.cnt[u] = 0;
       p.ready[u] = 0;
     }
     // block-wide exclusive scan of c
