@@ -313,10 +313,11 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
         // S[rows of group h][keys] into slot sl + h with one MMA chain per
         // group; sweep 2 writes S^T[keys][all rows] with a single chain of
         // N = R_pad across the tile's slots (sl is even when nh = 2), which
-        // reads the K tile once instead of once per group.
-        for (int h = 0; h < nh; ++h)
-          if (!wait_bar_warp(&sm.tempty[sl + h], tph ^ 1, p)) { ok = false; break; }
-        if (!ok) break;
+        // reads the K tile once instead of once per group.  The slots of a
+        // tile are filled, announced and released together: one full and one
+        // empty barrier per tile (those of its first slot), as every barrier
+        // operation costs the issuing warp a few hundred cycles here.
+        if (!wait_bar_warp(&sm.tempty[sl], tph ^ 1, p)) { ok = false; break; }
         tc_fence_after();
         if (s1) {
           for (int h = 0; h < nh; ++h) {
@@ -327,7 +328,6 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
               const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
               umma_bf16_elect(dcol, qdesc + a, kdesc + b, idesc1, k > 0);
             }
-            umma_commit_elect(&sm.tfull[sl + h]);
           }
         } else {
           const uint32_t dcol = tmem_base + sl * kSlotCols;
@@ -336,8 +336,8 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
             const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
             umma_bf16_elect(dcol, kdesc + a, qdesc0 + b, idesc2, k > 0);
           }
-          for (int h = 0; h < nh; ++h) umma_commit_elect(&sm.tfull[sl + h]);
         }
+        umma_commit_elect(&sm.tfull[sl]);
         sl += nh;
         if (sl == kSlots) { sl = 0; tph ^= 1; }
         umma_commit_elect(&sm.kempty[st]);
@@ -458,10 +458,10 @@ __device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, ui
 }
 
 // Both slots of a tile (g, g + 1) in one round trip: two loads in flight, one
-// wait, both released before any arithmetic.
+// wait, both released (through the first slot's barrier) before any arithmetic.
 __device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r0)[32],
                                            uint32_t (&r1)[32]) {
-  const uint32_t s0 = g & (kSlots - 1), s1 = (g + 1) & (kSlots - 1);
+  const uint32_t s0 = g & (kSlots - 1), s1 = s0 + 1;
   tmem_ld32_async(lane_base + s0 * kSlotCols, r0);
   tmem_ld32_async(lane_base + s1 * kSlotCols, r1);
   tmem_wait32(r0);
@@ -469,7 +469,6 @@ __device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, u
   tc_fence_before();
   __syncwarp();
   mbar_arrive_elect(&sm.tempty[s0]);
-  mbar_arrive_elect(&sm.tempty[s1]);
 }
 
 __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm, uint32_t tmem_base,
@@ -509,7 +508,6 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         // others and dropped when the warpgroup publishes.
         if (nh == 2) {
           ok = slot_wait(p, sm, g, ok);
-          ok = slot_wait(p, sm, g + 1, ok);
           uint32_t r0[32], r1[32];
           slot_take2(sm, lane_base, g, r0, r1);
           float v0[32], v1[32];
@@ -562,7 +560,6 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
         ok = slot_wait(p, sm, g, ok);
-        if (nh == 2) ok = slot_wait(p, sm, g + 1, ok);
         if (nh == 2) {
           uint32_t ra[32], rb[32];
           slot_take2(sm, lane_base, g, ra, rb);
