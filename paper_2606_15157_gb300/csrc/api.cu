@@ -578,6 +578,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.chunk_keys = pp.chunk_keys;
     sp.q_rows = q_rows;
     sp.stages = stages;
+    sp.stage_per_tile = stages == kSlots / (ws.R_pad > 128 ? 2 : 1);
     sp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));
     sp.inv_G = 1.0f / static_cast<float>(P.G);
     sp.lens = lens_ok;

@@ -77,6 +77,8 @@ struct ScoreParams {
   int chunk_keys;     // keys per work item (multiple of 128)
   int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
   int stages;         // K tile ring depth
+  int stage_per_tile; // stages == tiles held in TMEM: a K stage is free when its tile's
+                      // accumulator is full (the producer waits on that barrier)
   float scale_log2;   // log2(e) / sqrt(d)
   float inv_G;
   const int* lens;

@@ -217,6 +217,7 @@ __device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uin
 template <int D>
 __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   constexpr uint32_t kTileBytes = kTileKeys * D * 2;
+  const uint32_t nh = p.R_pad > 128 ? 2 : 1;  // TMEM slots per tile
   const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
   const uint64_t drop = policy_evict_first();  // second read: its last use
   uint32_t tile = 0;            // tiles issued (for the drain after an abort)
@@ -249,7 +250,9 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
       }
       const uint32_t st = pst, ph = pph;
       if (++pst == static_cast<uint32_t>(p.stages)) { pst = 0; pph ^= 1; }
-      if (!wait_bar(&sm.kempty[st], ph ^ 1, p)) { ok = false; break; }
+      // the stage's previous tile is done with it once its MMAs complete
+      uint64_t* freed = p.stage_per_tile ? &sm.tfull[st * nh] : &sm.kempty[st];
+      if (!wait_bar(freed, ph ^ 1, p)) { ok = false; break; }
       uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kTileBytes;
       mbar_expect_tx(&sm.kfull[st], kTileBytes);
 #pragma unroll
@@ -340,7 +343,7 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
         umma_commit_elect(&sm.tfull[sl]);
         sl += nh;
         if (sl == kSlots) { sl = 0; tph ^= 1; }
-        umma_commit_elect(&sm.kempty[st]);
+        if (!p.stage_per_tile) umma_commit_elect(&sm.kempty[st]);
         if (++st == static_cast<uint32_t>(p.stages)) { st = 0; kph ^= 1; }
       }
       if (ok) umma_commit_elect(&sm.qempty[qb]);  // the entry's Q buffer is free once these finish
