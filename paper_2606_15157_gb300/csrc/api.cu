@@ -549,9 +549,20 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
                       ws.R_pad))
         return KVEV_ECUDA;
     }
-    int stages = 6;
-    while (stages >= 2 && score_smem_bytes(P.d, q_rows, ws.R_pad, stages) + 1024 > D.smem_optin)
-      --stages;
+    // K stages that fit next to q_bufs Q buffers.  A second Q buffer hides the
+    // next entry's Q load; when it costs the K ring its depth (fewer than four
+    // stages), one buffer and a deeper ring are the better trade.
+    auto fit = [&](int q_bufs) {
+      int st = 6;
+      while (st >= 2 && score_smem_bytes(P.d, q_rows, q_bufs, ws.R_pad, st) + 1024 > D.smem_optin)
+        --st;
+      return st;
+    };
+    int q_bufs = 2, stages = fit(2);
+    if (stages < 4 && fit(1) > stages) {
+      q_bufs = 1;
+      stages = fit(1);
+    }
     if (stages < 2) return KVEV_ENOTSUP;
     // The softmax warpgroups raise their register count with setmaxnreg,
     // drawing on the registers the CTA was launched with; refuse to launch a
@@ -560,7 +571,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     if (score_regs_ok(P.d) != 1) return KVEV_ENOTSUP;
     // Request more than half of the SM's shared memory so exactly one CTA is
     // resident per SM: its TMEM allocation then never waits on another CTA.
-    const size_t smem = std::max<size_t>(score_smem_bytes(P.d, q_rows, ws.R_pad, stages),
+    const size_t smem = std::max<size_t>(score_smem_bytes(P.d, q_rows, q_bufs, ws.R_pad, stages),
                                          static_cast<size_t>(D.smem_optin) / 2 + 1024);
     if (D.score_smem_set != smem) {
       if (score_set_smem(P.d, smem) != cudaSuccess) return KVEV_ECUDA;
@@ -577,6 +588,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.S_cap = S_cap;
     sp.chunk_keys = pp.chunk_keys;
     sp.q_rows = q_rows;
+    sp.q_bufs = q_bufs;
     sp.stages = stages;
     sp.stage_per_tile = stages == kSlots / (ws.R_pad > 128 ? 2 : 1);
     sp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));

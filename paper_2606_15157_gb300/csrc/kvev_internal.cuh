@@ -25,6 +25,7 @@ constexpr int kMinChunkTiles = 16;
 constexpr int kTreeFanIn = 4;
 constexpr int kTreeLevels = 5;        // internal levels: up to 4^5 = 1024 chunks per unit
 constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel
+constexpr int kRedTiles = 8;          // sweep-2 tiles whose key sums are combined at once
 constexpr int kScoreThreads = 128 * (1 + kSoftmaxWGs);  // + warpgroup 0: TMA, MMA, publisher, normaliser warps
 constexpr int kSlots = 4;             // TMEM accumulator slots of the score kernel
 constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 512 columns)
@@ -76,6 +77,8 @@ struct ScoreParams {
   int n_units, B, H_kv, H_q, G, W, R, R_pad, S_cap;
   int chunk_keys;     // keys per work item (multiple of 128)
   int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
+  int q_bufs;         // Q buffers (2: the next entry's Q loads during this entry; 1: it
+                      // loads once this entry is done, leaving room for more K stages)
   int stages;         // K tile ring depth
   int stage_per_tile; // stages == tiles held in TMEM: a K stage is free when its tile's
                       // accumulator is full (the producer waits on that barrier)
@@ -511,7 +514,7 @@ __device__ __forceinline__ uint32_t float_key(float f) {
 namespace kvev {
 cudaError_t launch_prologue(const PrologueParams& p, cudaStream_t s);
 cudaError_t launch_score(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
-int score_smem_bytes(int d, int q_rows, int R_pad, int stages);
+int score_smem_bytes(int d, int q_rows, int q_bufs, int R_pad, int stages);
 bool decode_supported(int d, int G);
 cudaError_t launch_decode_init(const DecodeParams& p, cudaStream_t s);
 cudaError_t launch_decode_step(const DecodeParams& p, size_t smem, cudaStream_t s);

@@ -40,18 +40,17 @@ namespace kvev {
 namespace {
 
 struct Smem {
-  uint8_t* qbuf;     // two Q buffers of qbytes each, indexed arithmetically (a dynamically
+  uint8_t* qbuf;     // q_bufs Q buffers of qbytes each, indexed arithmetically (a dynamically
   uint32_t qbytes;   // indexed member array would push the whole struct to local memory)
   uint8_t* kbuf;     // stages * tile bytes
   float* lam;        // [2][R_pad]: -lse2 of the units of the next two sweep-2 entries
-  float* red;        // [2][kSoftmaxWGs][128]: per-warpgroup partial key sums of a sweep-2 tile
+  float* red;        // [kSoftmaxWGs][kRedTiles][128]: per-warpgroup partial key sums of a batch
+                     // of sweep-2 tiles
   float2* pc;        // [kSoftmaxWGs][R_pad]: per-warpgroup (max, sum) of a sweep-1 item
   uint64_t* lfull;   // [2] lam buffer written by the normaliser warp
   uint64_t* lempty;  // [2] lam buffer read by the softmax warpgroups
   uint64_t* pfull;   // partials of a sweep-1 entry written to pc by the softmax threads
   uint64_t* pempty;  // pc read by the publisher warp
-  uint64_t* rfull;   // [2] red buffer holds the four warpgroups' partials of a tile
-  uint64_t* rempty;  // [2] red buffer read by the tile's writer warpgroup
   uint64_t* kfull;
   uint64_t* kempty;
   uint64_t* qfull;
@@ -63,21 +62,21 @@ struct Smem {
   int* flag;         // [2]: scratch of the publisher warp
 };
 
-__host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int R_pad, int stages,
+__host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int q_bufs, int R_pad, int stages,
                                                       size_t* koff, size_t* loff, size_t* roff,
                                                       size_t* poff, size_t* boff) {
-  size_t off = 2 * static_cast<size_t>(q_rows) * D * 2;
+  size_t off = static_cast<size_t>(q_bufs) * q_rows * D * 2;
   *koff = off;
   off += static_cast<size_t>(stages) * kTileKeys * D * 2;
   *loff = off;
   off += sizeof(float) * 2 * R_pad;
   *roff = off;
-  off += sizeof(float) * 2 * kSoftmaxWGs * 128;
+  off += sizeof(float) * kSoftmaxWGs * kRedTiles * 128;
   off = (off + 7) & ~size_t(7);
   *poff = off;
   off += sizeof(float2) * kSoftmaxWGs * R_pad;
   *boff = off;
-  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6 + 4);
+  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6);
   off += sizeof(uint32_t) + 2 * sizeof(int);
   return off;
 }
@@ -85,7 +84,7 @@ __host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int R_pa
 __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D) {
   Smem s;
   size_t koff, loff, roff, poff, boff;
-  smem_size(D, p.q_rows, p.R_pad, p.stages, &koff, &loff, &roff, &poff, &boff);
+  smem_size(D, p.q_rows, p.q_bufs, p.R_pad, p.stages, &koff, &loff, &roff, &poff, &boff);
   s.qbuf = base;
   s.qbytes = static_cast<uint32_t>(p.q_rows) * D * 2;
   s.kbuf = base + koff;
@@ -104,9 +103,7 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   s.lempty = s.lfull + 2;
   s.pfull = s.lempty + 2;
   s.pempty = s.pfull + 1;
-  s.rfull = s.pempty + 1;
-  s.rempty = s.rfull + 2;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.rempty + 2);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.pempty + 1);
   s.flag = reinterpret_cast<int*>(s.tmem_slot + 1);
   return s;
 }
@@ -205,7 +202,7 @@ __device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, u
 // ---------------------------------------------------------------------------
 template <int D>
 __device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uint32_t e, const ItemInfo& it) {
-  const uint32_t qb = e & 1;
+  const uint32_t qb = e % p.q_bufs;
   mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R_pad) * D * 2);
   const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
 #pragma unroll
@@ -223,6 +220,9 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
   uint32_t tile = 0;            // tiles issued (for the drain after an abort)
   uint32_t pst = 0, pph = 0;    // K stage ring: position and phase of the next tile
   uint32_t q_issued = 0;        // entries whose Q load has been issued
+  const uint32_t nq = p.q_bufs;
+  // Q of entry x goes into buffer x mod nq once entry x - nq has released it
+  auto q_free = [&](uint32_t x) { return mbar_try_wait(&sm.qempty[x % nq], ((x / nq) & 1) ^ 1); };
   bool ok = true;
   EntryIter ei(J);
   int jj, sw;
@@ -230,20 +230,23 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
     const int t = first + jj * stride;
     if (sw == 0) prefetch_item(p, first, stride, jj, J);
     const ItemInfo it = decode_item(p, t, load_item(p, t));
-    if (q_issued == e) {
-      if (!wait_bar(&sm.qempty[e & 1], ((e >> 1) & 1) ^ 1, p)) { ok = false; break; }
-      load_q<D>(p, sm, e, it);
-      ++q_issued;
-    }
-    // the next entry's Q goes out as soon as its buffer is released
     EntryIter la = ei;
     int jn, swn;
     const bool has_next = la.next(jn, swn);
     const CUtensorMap* kmap = &p.kmap[it.ls];
     const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
+    // This entry's Q goes out as soon as its buffer is free, and at the
+    // latest before the K tile that fills the last stage (the K tiles before
+    // it do not depend on Q, so they stream in meanwhile); with two buffers
+    // the next entry's Q goes out during this entry.
+    const int q_by = min(p.stages, it.ntiles) - 1;
     for (int i = 0; i < it.ntiles; ++i, ++tile) {
-      if (has_next && q_issued == e + 1 &&
-          mbar_try_wait(&sm.qempty[(e + 1) & 1], (((e + 1) >> 1) & 1) ^ 1)) {
+      if (q_issued == e && (i >= q_by || q_free(e))) {
+        if (!wait_bar(&sm.qempty[e % nq], ((e / nq) & 1) ^ 1, p)) { ok = false; break; }
+        load_q<D>(p, sm, e, it);
+        ++q_issued;
+      }
+      if (nq > 1 && has_next && q_issued == e + 1 && q_free(e + 1)) {
         const int tn = first + jn * stride;
         load_q<D>(p, sm, e + 1, decode_item(p, tn, load_item(p, tn)));
         ++q_issued;
@@ -269,9 +272,9 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
       const uint32_t last = ((tile - 1 - st) / S) * S + st;  // last tile issued into st
       wait_bar_drain(&sm.kfull[st], (last / S) & 1, 100000000ull);
     }
-    for (uint32_t b = 0; b < 2; ++b) {
-      const uint32_t nb = (q_issued + 1 - b) / 2;  // Q loads issued into buffer b
-      if (nb > 0) wait_bar_drain(&sm.qfull[b], (nb - 1) & 1, 100000000ull);
+    for (uint32_t b = 0; b < nq && b < q_issued; ++b) {
+      const uint32_t last = ((q_issued - 1 - b) / nq) * nq + b;  // last Q load into buffer b
+      wait_bar_drain(&sm.qfull[b], (last / nq) & 1, 100000000ull);
     }
   }
 }
@@ -301,9 +304,9 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
       const int t = first + jj * stride;
       if (sw == 0) prefetch_item(p, first, stride, jj, J);
       const ItemInfo it = decode_item(p, t, load_item(p, t));
-      const uint32_t qb = e & 1;
+      const uint32_t qb = e % p.q_bufs;
       const uint64_t qdesc0 = sw128_desc(smem_u32(sm.qbuf) + qb * sm.qbytes);
-      if (!wait_bar_warp(&sm.qfull[qb], (e >> 1) & 1, p)) { ok = false; break; }
+      if (!wait_bar_warp(&sm.qfull[qb], (e / p.q_bufs) & 1, p)) { ok = false; break; }
       const bool s1 = sw == 0;
       const uint32_t astep = s1 ? qcol_step : kcol_step, bstep = s1 ? kcol_step : qcol_step;
       for (int i = 0; i < it.ntiles; ++i) {
@@ -489,7 +492,6 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   const bool has_a = r0a < (nh == 2 ? 128 : p.R_pad);
   const bool has_b = nh == 2 && r0b < p.R_pad;
   uint32_t g = 0;     // slot stream position (advances nh per tile)
-  uint32_t tc = 0;    // sweep-2 tiles done (reduction buffer parity, writer)
   uint32_t q1 = 0, q2 = 0;  // sweep-1 / sweep-2 entries done
   bool ok = true;
 
@@ -556,7 +558,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       if (!wait_bar(&sm.lfull[lb], (q2 >> 1) & 1, p)) ok = false;
       const float* lam = sm.lam + lb * p.R_pad;
       float* out = p.raw + static_cast<size_t>(it.u) * p.S_cap;
-      for (int i = 0; i < it.ntiles; ++i, ++tc) {
+      for (int i = 0; i < it.ntiles; ++i) {
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
         const bool key_full = kb + kTileKeys - 1 <= it.n - p.W;
@@ -577,29 +579,26 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
         }
         g += nh;
-        // Sum the four warpgroups' partials of each key: every warpgroup
-        // deposits its partial in buffer tc mod 2 and moves on; warpgroup
-        // tc mod 4 waits for the other three, writes the sum and frees the buffer.
-        const uint32_t rb = tc & 1, rph = (tc >> 1) & 1;
-        float* red = sm.red + rb * (kSoftmaxWGs * 128);
-        if (!wait_bar(&sm.rempty[rb], rph ^ 1, p)) ok = false;
-        red[wg * 128 + lrow] = sum4x2(a);
-        __syncwarp();
-        mbar_arrive_elect(&sm.rfull[rb]);
-        if (wg == static_cast<int>(tc % kSoftmaxWGs)) {
-          if (!wait_bar(&sm.rfull[rb], rph, p)) ok = false;
-          if (ok && k < it.n) {
+        // Each warpgroup keeps its partial sum of every key of a batch of
+        // kRedTiles tiles in its own shared-memory rows; at the end of the
+        // batch all four are added (in warpgroup order) and stored, with one
+        // barrier on either side instead of a hand-off per tile.
+        const int bt = i % kRedTiles;
+        sm.red[(wg * kRedTiles + bt) * 128 + lrow] = sum4x2(a);
+        if (bt == kRedTiles - 1 || i == it.ntiles - 1) {
+          named_bar_sync(1, 128 * kSoftmaxWGs);
+          const int key0 = it.key0 + (i - bt) * kTileKeys;
+          for (int q = stid; q < (bt + 1) * 128; q += 128 * kSoftmaxWGs) {
             float sum = 0.f;
 #pragma unroll
-            for (int w = 0; w < kSoftmaxWGs; ++w) sum += red[w * 128 + lrow];
-            out[k] = sum * p.inv_G;
+            for (int w = 0; w < kSoftmaxWGs; ++w) sum += sm.red[w * kRedTiles * 128 + q];
+            if (ok && key0 + q < it.n) out[key0 + q] = sum * p.inv_G;
           }
-          __syncwarp();
-          mbar_arrive_elect(&sm.rempty[rb]);
+          // the batch's rows may be overwritten, and after the entry's last
+          // batch every warpgroup is done reading lam
+          named_bar_sync(1, 128 * kSoftmaxWGs);
         }
       }
-      // every warpgroup is done reading lam once all have passed this barrier
-      named_bar_sync(1, 128 * kSoftmaxWGs);
       if (stid == 0) mbar_arrive(&sm.lempty[lb]);
       ++q2;
     }
@@ -777,10 +776,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     }
     mbar_init(sm.pfull, 4 * kSoftmaxWGs);
     mbar_init(sm.pempty, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.rfull[i], 4 * kSoftmaxWGs);
-      mbar_init(&sm.rempty[i], 4);  // the writer warpgroup's warps
-    }
     fence_barrier_init();
     fence_proxy_async();
   }
@@ -888,9 +883,9 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
 
 }  // namespace
 
-int score_smem_bytes(int d, int q_rows, int R_pad, int stages) {
+int score_smem_bytes(int d, int q_rows, int q_bufs, int R_pad, int stages) {
   size_t koff, loff, roff, poff, boff;
-  const size_t off = smem_size(d, q_rows, R_pad, stages, &koff, &loff, &roff, &poff, &boff);
+  const size_t off = smem_size(d, q_rows, q_bufs, R_pad, stages, &koff, &loff, &roff, &poff, &boff);
   return static_cast<int>((off + 127) & ~size_t(127));
 }
 
