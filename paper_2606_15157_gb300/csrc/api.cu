@@ -499,7 +499,8 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   // that a unit never spans more than two rounds of the persistent grid
   const int grid = D.num_sms;
   const int tiles_max = (S_cap + kTileKeys - 1) / kTileKeys;
-  const int chunk_tiles = std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid);
+  // (an even number of tiles: chunks are swept in 256-key super-tiles)
+  const int chunk_tiles = (std::max(kMinChunkTiles, (tiles_max + grid - 1) / grid) + 1) & ~1;
   if (chunk_tiles > 0xFFFF) return KVEV_ENOTSUP;  // tiles per item are packed in 16 bits
   // the normaliser's merge tree has kTreeLevels internal levels of fan-in kTreeFanIn
   int leaves = 1;
@@ -544,22 +545,22 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     for (int i = 0; i < n_slayers; ++i) {
       const int l = P.score_layers[i];
       if (!encode_map(&sp.kmap[i], K[l], P.d, static_cast<uint64_t>(B) * P.H_kv * S_cap,
-                      kTileKeys) ||
+                      kSuperKeys) ||
           !encode_map(&sp.qmap[i], Q_win[l], P.d, static_cast<uint64_t>(B) * P.H_q * P.W,
                       ws.R_pad))
         return KVEV_ECUDA;
     }
-    // K stages that fit next to q_bufs Q buffers.  A second Q buffer hides the
-    // next entry's Q load; when it costs the K ring its depth (fewer than four
-    // stages), one buffer and a deeper ring are the better trade.
+    // K stages (256-key super-tiles) that fit next to q_bufs Q buffers.  A
+    // second Q buffer hides the next entry's Q load, but the ring needs two
+    // stages; with one buffer the next entry's Q loads once this one is done.
     auto fit = [&](int q_bufs) {
-      int st = 6;
+      int st = 4;
       while (st >= 2 && score_smem_bytes(P.d, q_rows, q_bufs, ws.R_pad, st) + 1024 > D.smem_optin)
         --st;
       return st;
     };
     int q_bufs = 2, stages = fit(2);
-    if (stages < 4 && fit(1) > stages) {
+    if (stages < 2) {
       q_bufs = 1;
       stages = fit(1);
     }
@@ -590,7 +591,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.q_rows = q_rows;
     sp.q_bufs = q_bufs;
     sp.stages = stages;
-    sp.stage_per_tile = stages == kSlots / (ws.R_pad > 128 ? 2 : 1);
     sp.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(P.d)));
     sp.inv_G = 1.0f / static_cast<float>(P.G);
     sp.lens = lens_ok;

@@ -14,6 +14,7 @@ namespace kvev {
 constexpr int kMaxLayers = 128;       // layers in one plan
 constexpr int kMaxScoreLayers = 64;   // SnapKV/H2O layers (tensor maps travel as kernel params)
 constexpr int kTileKeys = 128;        // keys per tensor-core tile (MMA M or N)
+constexpr int kSuperKeys = 256;       // keys per K stage (sweep 1 MMAs take N = 256 keys)
 // Tiles per scoring work item (chunk), at least.  Larger chunks give each CTA
 // more slack before it needs a unit's normaliser and halve the partials to
 // merge; the cost is reuse distance (grid * chunk bytes between a tile's two
@@ -80,8 +81,6 @@ struct ScoreParams {
   int q_bufs;         // Q buffers (2: the next entry's Q loads during this entry; 1: it
                       // loads once this entry is done, leaving room for more K stages)
   int stages;         // K tile ring depth
-  int stage_per_tile; // stages == tiles held in TMEM: a K stage is free when its tile's
-                      // accumulator is full (the producer waits on that barrier)
   float scale_log2;   // log2(e) / sqrt(d)
   float inv_G;
   const int* lens;

@@ -67,7 +67,7 @@ __host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int q_bu
                                                       size_t* poff, size_t* boff) {
   size_t off = static_cast<size_t>(q_bufs) * q_rows * D * 2;
   *koff = off;
-  off += static_cast<size_t>(stages) * kTileKeys * D * 2;
+  off += static_cast<size_t>(stages) * kSuperKeys * D * 2;
   *loff = off;
   off += sizeof(float) * 2 * R_pad;
   *roff = off;
@@ -213,11 +213,10 @@ __device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uin
 
 template <int D>
 __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
-  constexpr uint32_t kTileBytes = kTileKeys * D * 2;
-  const uint32_t nh = p.R_pad > 128 ? 2 : 1;  // TMEM slots per tile
+  constexpr uint32_t kStageBytes = kSuperKeys * D * 2;
   const uint64_t keep = policy_evict_last();   // first read of a K tile: keep it for the re-read
   const uint64_t drop = policy_evict_first();  // second read: its last use
-  uint32_t tile = 0;            // tiles issued (for the drain after an abort)
+  uint32_t tile = 0;            // super-tiles issued (for the drain after an abort)
   uint32_t pst = 0, pph = 0;    // K stage ring: position and phase of the next tile
   uint32_t q_issued = 0;        // entries whose Q load has been issued
   const uint32_t nq = p.q_bufs;
@@ -235,12 +234,13 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
     const bool has_next = la.next(jn, swn);
     const CUtensorMap* kmap = &p.kmap[it.ls];
     const int row0 = (it.s * p.H_kv + it.h) * p.S_cap + it.key0;
+    const int nst = (it.ntiles + 1) / 2;  // 256-key super-tiles of the item
     // This entry's Q goes out as soon as its buffer is free, and at the
-    // latest before the K tile that fills the last stage (the K tiles before
-    // it do not depend on Q, so they stream in meanwhile); with two buffers
-    // the next entry's Q goes out during this entry.
-    const int q_by = min(p.stages, it.ntiles) - 1;
-    for (int i = 0; i < it.ntiles; ++i, ++tile) {
+    // latest before the super-tile that fills the last stage (the K loads
+    // before it do not depend on Q, so they stream in meanwhile); with two
+    // buffers the next entry's Q goes out during this entry.
+    const int q_by = min(p.stages, nst) - 1;
+    for (int i = 0; i < nst; ++i, ++tile) {
       if (q_issued == e && (i >= q_by || q_free(e))) {
         if (!wait_bar(&sm.qempty[e % nq], ((e / nq) & 1) ^ 1, p)) { ok = false; break; }
         load_q<D>(p, sm, e, it);
@@ -253,14 +253,12 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
       }
       const uint32_t st = pst, ph = pph;
       if (++pst == static_cast<uint32_t>(p.stages)) { pst = 0; pph ^= 1; }
-      // the stage's previous tile is done with it once its MMAs complete
-      uint64_t* freed = p.stage_per_tile ? &sm.tfull[st * nh] : &sm.kempty[st];
-      if (!wait_bar(freed, ph ^ 1, p)) { ok = false; break; }
-      uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kTileBytes;
-      mbar_expect_tx(&sm.kfull[st], kTileBytes);
+      if (!wait_bar(&sm.kempty[st], ph ^ 1, p)) { ok = false; break; }
+      uint8_t* dst = sm.kbuf + static_cast<size_t>(st) * kStageBytes;
+      mbar_expect_tx(&sm.kfull[st], kStageBytes);
 #pragma unroll
       for (int kc = 0; kc < D / 64; ++kc)
-        tma_load_2d_hint(dst + kc * (kTileKeys * 128), kmap, kc * 64, row0 + i * kTileKeys,
+        tma_load_2d_hint(dst + kc * (kSuperKeys * 128), kmap, kc * 64, row0 + i * kSuperKeys,
                          &sm.kfull[st], sw == 0 ? keep : drop);
     }
   }
@@ -286,71 +284,70 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
 template <int D>
 __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm, uint32_t tmem_base, int first,
                            int stride, int J) {
-  constexpr uint32_t kTileBytes = kTileKeys * D * 2;
+  constexpr uint32_t kStageBytes = kSuperKeys * D * 2;
   const int nh = p.R_pad > 128 ? 2 : 1;
-  const uint32_t idesc1 = idesc_bf16_f32(128, kTileKeys);
-  // sweep 2: one MMA chain with N = every window row (up to 256 = two slots side by side)
+  // sweep 1: S[128 rows of a group][256 keys of a super-tile]
+  const uint32_t idesc1 = idesc_bf16_f32(128, kSuperKeys);
+  // sweep 2: S^T[128 keys][every window row] (up to 256)
   const uint32_t idesc2 = idesc_bf16_f32(128, p.R_pad);
-  // descriptor steps (address / 16) between the 64-wide column blocks of Q and of a K tile
+  // descriptor steps (address / 16) between the 64-wide column blocks of Q and of a K stage
   const uint32_t qcol_step = static_cast<uint32_t>(p.q_rows) * 128 / 16;
-  constexpr uint32_t kcol_step = kTileKeys * 128 / 16;
-  uint32_t st = 0, kph = 0;  // K stage ring: position and phase of the next tile
-  uint32_t sl = 0, tph = 0;  // TMEM slot ring: position and phase of the next slot
+  constexpr uint32_t kcol_step = kSuperKeys * 128 / 16;
+  constexpr uint32_t khalf = kTileKeys * 128 / 16;   // second 128-key half of a super-tile
+  constexpr uint32_t qgroup = 128 * 128 / 16;         // second 128-row group of Q
+  uint32_t st = 0, kph = 0;  // K stage ring: position and phase of the next super-tile
+  uint32_t sl = 0, tph = 0;  // TMEM ring of two 256-column units: first slot and phase
   bool ok = true;
   EntryIter ei(J);
   int jj, sw;
   for (uint32_t e = 0; ok && ei.next(jj, sw); ++e) {
-    {
-      const int t = first + jj * stride;
-      if (sw == 0) prefetch_item(p, first, stride, jj, J);
-      const ItemInfo it = decode_item(p, t, load_item(p, t));
-      const uint32_t qb = e % p.q_bufs;
-      const uint64_t qdesc0 = sw128_desc(smem_u32(sm.qbuf) + qb * sm.qbytes);
-      if (!wait_bar_warp(&sm.qfull[qb], (e / p.q_bufs) & 1, p)) { ok = false; break; }
-      const bool s1 = sw == 0;
-      const uint32_t astep = s1 ? qcol_step : kcol_step, bstep = s1 ? kcol_step : qcol_step;
-      for (int i = 0; i < it.ntiles; ++i) {
-        if (!wait_bar_warp(&sm.kfull[st], kph, p)) { ok = false; break; }
-        // Descriptors of the tile and of the Q row group, built once: a
-        // descriptor's low field is the address / 16, so the k-step offsets
-        // (all inside shared memory, no carry out of the field) are plain adds.
-        const uint64_t kdesc = sw128_desc(smem_u32(sm.kbuf) + st * kTileBytes);
-        // One 128-column TMEM slot per 128-row group of Q.  Sweep 1 writes
-        // S[rows of group h][keys] into slot sl + h with one MMA chain per
-        // group; sweep 2 writes S^T[keys][all rows] with a single chain of
-        // N = R_pad across the tile's slots (sl is even when nh = 2), which
-        // reads the K tile once instead of once per group.  The slots of a
-        // tile are filled, announced and released together: one full and one
-        // empty barrier per tile (those of its first slot), as every barrier
-        // operation costs the issuing warp a few hundred cycles here.
+    const int t = first + jj * stride;
+    if (sw == 0) prefetch_item(p, first, stride, jj, J);
+    const ItemInfo it = decode_item(p, t, load_item(p, t));
+    const uint32_t qb = e % p.q_bufs;
+    const uint64_t qdesc0 = sw128_desc(smem_u32(sm.qbuf) + qb * sm.qbytes);
+    if (!wait_bar_warp(&sm.qfull[qb], (e / p.q_bufs) & 1, p)) { ok = false; break; }
+    const bool s1 = sw == 0;
+    const int nst = (it.ntiles + 1) / 2;
+    for (int j = 0; ok && j < nst; ++j) {
+      if (!wait_bar_warp(&sm.kfull[st], kph, p)) { ok = false; break; }
+      // Descriptors built once per super-tile: a descriptor's low field is
+      // the address / 16, so the k-step offsets (all inside shared memory, no
+      // carry out of the field) are plain adds.
+      const uint64_t kdesc = sw128_desc(smem_u32(sm.kbuf) + st * kStageBytes);
+      // Work units of one super-tile, each a 256-column TMEM unit (two
+      // slots) with one full and one empty barrier (those of its first
+      // slot): sweep 1 -> one unit per 128-row group of Q, N = 256 keys;
+      // sweep 2 -> one unit per 128-key half, N = every window row.
+      const int nu = s1 ? nh : min(2, it.ntiles - 2 * j);
+      for (int u = 0; u < nu; ++u) {
         if (!wait_bar_warp(&sm.tempty[sl], tph ^ 1, p)) { ok = false; break; }
         tc_fence_after();
+        const uint32_t dcol = tmem_base + sl * kSlotCols;
         if (s1) {
-          for (int h = 0; h < nh; ++h) {
-            const uint32_t dcol = tmem_base + (sl + h) * kSlotCols;
-            const uint64_t qdesc = qdesc0 + static_cast<uint64_t>(h * (128 * 128 / 16));
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-              const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
-              umma_bf16_elect(dcol, qdesc + a, kdesc + b, idesc1, k > 0);
-            }
-          }
-        } else {
-          const uint32_t dcol = tmem_base + sl * kSlotCols;
+          const uint64_t qdesc = qdesc0 + static_cast<uint64_t>(u * qgroup);
 #pragma unroll
           for (int k = 0; k < D / 16; ++k) {
-            const uint32_t a = (k >> 2) * astep + (k & 3) * 2, b = (k >> 2) * bstep + (k & 3) * 2;
-            umma_bf16_elect(dcol, kdesc + a, qdesc0 + b, idesc2, k > 0);
+            const uint32_t a = (k >> 2) * qcol_step + (k & 3) * 2, b = (k >> 2) * kcol_step + (k & 3) * 2;
+            umma_bf16_elect(dcol, qdesc + a, kdesc + b, idesc1, k > 0);
+          }
+        } else {
+          const uint64_t adesc = kdesc + static_cast<uint64_t>(u * khalf);
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint32_t a = (k >> 2) * kcol_step + (k & 3) * 2, b = (k >> 2) * qcol_step + (k & 3) * 2;
+            umma_bf16_elect(dcol, adesc + a, qdesc0 + b, idesc2, k > 0);
           }
         }
         umma_commit_elect(&sm.tfull[sl]);
-        sl += nh;
+        sl += 2;
         if (sl == kSlots) { sl = 0; tph ^= 1; }
-        if (!p.stage_per_tile) umma_commit_elect(&sm.kempty[st]);
-        if (++st == static_cast<uint32_t>(p.stages)) { st = 0; kph ^= 1; }
       }
-      if (ok) umma_commit_elect(&sm.qempty[qb]);  // the entry's Q buffer is free once these finish
+      if (!ok) break;
+      umma_commit_elect(&sm.kempty[st]);
+      if (++st == static_cast<uint32_t>(p.stages)) { st = 0; kph ^= 1; }
     }
+    if (ok) umma_commit_elect(&sm.qempty[qb]);  // the entry's Q buffer is free once these finish
   }
   // Every MMA issued so far has completed once `done` flips.
   umma_commit_elect(sm.done);
@@ -387,12 +384,11 @@ __device__ __forceinline__ void mask_chunk(float (&v)[32], int k0, int tr) {
     if (k0 + i > tr) v[i] = -INFINITY;
 }
 
-// One 32-key chunk of sweep 1 for one row: online base-2 (max, sum) update.
-// Branch-free, so the two rows a thread holds interleave: a row with no
-// visible key yet (m = -inf) offsets its exponents by 0 instead, where every
-// term is exp2(-inf) = 0.
-__device__ __forceinline__ void s1_chunk(const float (&v)[32], float c, float& m, float& z) {
-  const float mnew = fmaxf(m, max32(v) * c);
+// One sweep-1 unit for one row: online base-2 (max, sum) update over the
+// thread's 64 keys (two 32-key halves), with one rescale of the running sum.
+__device__ __forceinline__ void s1_chunk64(const float (&v0)[32], const float (&v1)[32], float c, float& m,
+                                           float& z) {
+  const float mnew = fmaxf(m, fmaxf(max32(v0), max32(v1)) * c);
   const float base = mnew == -INFINITY ? 0.f : mnew;
   const float zs = z * ex2_approx(m - base);  // m = -inf -> 0
   const float2 cc = make_float2(c, c), nb = make_float2(-base, -base);
@@ -400,8 +396,10 @@ __device__ __forceinline__ void s1_chunk(const float (&v)[32], float c, float& m
                  make_float2(0.f, 0.f)};
 #pragma unroll
   for (int i = 0; i < 32; i += 2) {
-    const float2 t = ffma2(make_float2(v[i], v[i + 1]), cc, nb);
-    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t.x), ex2_approx(t.y)));
+    const float2 t0 = ffma2(make_float2(v0[i], v0[i + 1]), cc, nb);
+    const float2 t1 = ffma2(make_float2(v1[i], v1[i + 1]), cc, nb);
+    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
   }
   z = zs + sum4x2(a);
   m = mnew;
@@ -463,7 +461,7 @@ __device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, ui
   mbar_arrive_elect(&sm.tempty[sl]);
 }
 
-// Both slots of a tile (g, g + 1) in one round trip: two loads in flight, one
+// Both slots of a unit (g, g + 1) in one round trip: two loads in flight, one
 // wait, both released (through the first slot's barrier) before any arithmetic.
 __device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r0)[32],
                                            uint32_t (&r1)[32]) {
@@ -491,7 +489,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   const int r0a = 32 * wg, r0b = 128 + 32 * wg;
   const bool has_a = r0a < (nh == 2 ? 128 : p.R_pad);
   const bool has_b = nh == 2 && r0b < p.R_pad;
-  uint32_t g = 0;     // slot stream position (advances nh per tile)
+  uint32_t g = 0;     // slot stream position (advances 2 per 256-column unit)
   uint32_t q1 = 0, q2 = 0;  // sweep-1 / sweep-2 entries done
   bool ok = true;
 
@@ -506,12 +504,16 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
       const int tr0 = lrow < p.R ? row_pos(p, lrow, it.n) : -1;
       const int tr1 = 128 + lrow < p.R ? row_pos(p, 128 + lrow, it.n) : -1;
-      for (int i = 0; i < it.ntiles; ++i) {
-        const int k0 = it.key0 + i * kTileKeys + 32 * wg;  // this warpgroup's 32 keys
-        const bool full = k0 + 31 <= it.n - p.W;          // every key visible to every row
-        // Rows of a slot that do not exist (tr < 0) are computed like the
-        // others and dropped when the warpgroup publishes.
-        if (nh == 2) {
+      // One unit per (256-key super-tile, 128-row group): this warpgroup's 32
+      // keys of each 128-key half, for the thread's row of the group.  Rows
+      // that do not exist (tr < 0) are computed like the others and dropped
+      // when the warpgroup publishes.
+      const int nst = (it.ntiles + 1) / 2;
+      for (int j = 0; j < nst; ++j) {
+        const int kb = it.key0 + j * kSuperKeys;
+        const int k0 = kb + 32 * wg;                       // keys k0.. and k0 + 128..
+        const bool full = kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
+        for (int h = 0; h < nh; ++h) {
           ok = slot_wait(p, sm, g, ok);
           uint32_t r0[32], r1[32];
           slot_take2(sm, lane_base, g, r0, r1);
@@ -521,23 +523,17 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             v0[q] = __uint_as_float(r0[q]);
             v1[q] = __uint_as_float(r1[q]);
           }
+          const int tr = h == 0 ? tr0 : tr1;
           if (!full) {
-            mask_chunk(v0, k0, tr0);
-            mask_chunk(v1, k0, tr1);
+            mask_chunk(v0, k0, tr);
+            mask_chunk(v1, k0 + kTileKeys, tr);
           }
-          s1_chunk(v0, p.scale_log2, m0, z0);
-          s1_chunk(v1, p.scale_log2, m1, z1);
-        } else {
-          ok = slot_wait(p, sm, g, ok);
-          uint32_t r0[32];
-          slot_take(sm, lane_base, g, r0);
-          float v0[32];
-#pragma unroll
-          for (int q = 0; q < 32; ++q) v0[q] = __uint_as_float(r0[q]);
-          if (!full) mask_chunk(v0, k0, tr0);
-          s1_chunk(v0, p.scale_log2, m0, z0);
+          if (h == 0)
+            s1_chunk64(v0, v1, p.scale_log2, m0, z0);
+          else
+            s1_chunk64(v0, v1, p.scale_log2, m1, z1);
+          g += 2;
         }
-        g += nh;
       }
       // hand the four warpgroups' (max, sum) of each row to the publisher warp
       if (!wait_bar(&sm.pempty[0], (q1 & 1) ^ 1, p)) ok = false;
@@ -578,7 +574,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
           if (ok && has_a && k < it.n)
             s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
         }
-        g += nh;
+        g += 2;
         // Each warpgroup keeps its partial sum of every key of a batch of
         // kRedTiles tiles in its own shared-memory rows; at the end of the
         // batch all four are added (in warpgroup order) and stored, with one
