@@ -435,41 +435,28 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
   }
 }
 
-// ---- TMEM slot hand-off --------------------------------------------------
-// Every fill is consumed by all four softmax warpgroups: warpgroup w copies
-// its 32-column slice [32w, 32w + 32) of the slot and releases the slot at
-// once (the slot's empty barrier counts the 16 softmax warps: one elected lane
-// arrives for its warp, as a shared-memory barrier takes its arrivals one at a
-// time), so the tensor core refills a slot as soon as the last slice is copied
-// and no warpgroup holds a slot while it computes.
+// ---- TMEM unit hand-off ----------------------------------------------------
+// Every 256-column unit is consumed by all four softmax warpgroups:
+// warpgroup w copies its 64 columns and releases the unit at once (the
+// unit's empty barrier counts the 16 softmax warps: one elected lane arrives
+// for its warp, as a shared-memory barrier takes its arrivals one at a time),
+// so the tensor core refills it as soon as the last slice is copied and no
+// warpgroup holds TMEM while it computes.
 
 __device__ __forceinline__ bool slot_wait(const ScoreParams& p, const Smem& sm, uint32_t g, bool ok) {
   if (ok && !wait_bar(&sm.tfull[g & (kSlots - 1)], (g / kSlots) & 1, p)) ok = false;
   return ok;
 }
 
-// Copy this warpgroup's 32 columns of slot (g mod 4) and release the slot.
-// Loaded even when the wait failed (the address is always inside this CTA's
-// TMEM allocation; the values are then discarded): a conditional load would
-// leave the array undefined on one path and spill it.
-__device__ __forceinline__ void slot_take(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r)[32]) {
-  const uint32_t sl = g & (kSlots - 1);
-  tmem_ld32_async(lane_base + sl * kSlotCols, r);
-  tmem_wait32(r);
-  tc_fence_before();
-  __syncwarp();
-  mbar_arrive_elect(&sm.tempty[sl]);
-}
 
-// Both slots of a unit (g, g + 1) in one round trip: two loads in flight, one
-// wait, both released (through the first slot's barrier) before any arithmetic.
-__device__ __forceinline__ void slot_take2(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r0)[32],
-                                           uint32_t (&r1)[32]) {
-  const uint32_t s0 = g & (kSlots - 1), s1 = s0 + 1;
-  tmem_ld32_async(lane_base + s0 * kSlotCols, r0);
-  tmem_ld32_async(lane_base + s1 * kSlotCols, r1);
-  tmem_wait32(r0);
-  tmem_wait32(r1);
+// This warpgroup's 64 columns of a unit (the unit's two slots are 256
+// adjacent columns; warpgroup w takes [64w, 64w + 64)) in one load, released
+// (through the first slot's barrier) before any arithmetic.
+__device__ __forceinline__ void unit_take(const Smem& sm, uint32_t lane_base, uint32_t g, uint32_t (&r0)[32],
+                                          uint32_t (&r1)[32]) {
+  const uint32_t s0 = g & (kSlots - 1);
+  tmem_ld64_async(lane_base + s0 * kSlotCols, r0, r1);
+  tmem_wait64(r0, r1);
   tc_fence_before();
   __syncwarp();
   mbar_arrive_elect(&sm.tempty[s0]);
@@ -482,13 +469,13 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   const int lrow = quarter * 32 + (threadIdx.x & 31);  // TMEM lane: row (sweep 1) / key (sweep 2)
   const int stid = threadIdx.x - 128;                  // 0..511 over the softmax warpgroups
   const int nh = p.R_pad > 128 ? 2 : 1;                // 128-row groups (slots) per tile
-  // this warpgroup's column slice of every slot
+  // this warpgroup's 64 columns of every 256-column unit
   const uint32_t lane_base =
-      tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(32 * wg);
-  // sweep 2: this warpgroup's rows [32wg, 32wg + 32) of group 0 and [128 + 32wg, ...) of group 1
-  const int r0a = 32 * wg, r0b = 128 + 32 * wg;
-  const bool has_a = r0a < (nh == 2 ? 128 : p.R_pad);
-  const bool has_b = nh == 2 && r0b < p.R_pad;
+      tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(64 * wg);
+  // sweep 2: this warpgroup's rows [64wg, 64wg + 32) and [64wg + 32, 64wg + 64)
+  const int r0a = 64 * wg, r0b = 64 * wg + 32;
+  const bool has_a = r0a < p.R_pad;
+  const bool has_b = r0b < p.R_pad;
   uint32_t g = 0;     // slot stream position (advances 2 per 256-column unit)
   uint32_t q1 = 0, q2 = 0;  // sweep-1 / sweep-2 entries done
   bool ok = true;
@@ -511,12 +498,12 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       const int nst = (it.ntiles + 1) / 2;
       for (int j = 0; j < nst; ++j) {
         const int kb = it.key0 + j * kSuperKeys;
-        const int k0 = kb + 32 * wg;                       // keys k0.. and k0 + 128..
+        const int k0 = kb + 64 * wg;                       // keys k0 .. k0 + 63
         const bool full = kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
         for (int h = 0; h < nh; ++h) {
           ok = slot_wait(p, sm, g, ok);
           uint32_t r0[32], r1[32];
-          slot_take2(sm, lane_base, g, r0, r1);
+          unit_take(sm, lane_base, g, r0, r1);
           float v0[32], v1[32];
 #pragma unroll
           for (int q = 0; q < 32; ++q) {
@@ -526,7 +513,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
           const int tr = h == 0 ? tr0 : tr1;
           if (!full) {
             mask_chunk(v0, k0, tr);
-            mask_chunk(v1, k0 + kTileKeys, tr);
+            mask_chunk(v1, k0 + 32, tr);
           }
           if (h == 0)
             s1_chunk64(v0, v1, p.scale_log2, m0, z0);
@@ -561,18 +548,13 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
         ok = slot_wait(p, sm, g, ok);
-        if (nh == 2) {
+        {
           uint32_t ra[32], rb[32];
-          slot_take2(sm, lane_base, g, ra, rb);
+          unit_take(sm, lane_base, g, ra, rb);
           if (ok && has_a && k < it.n)
             s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
           if (ok && has_b && k < it.n)
             s2_chunk(p, rb, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
-        } else {
-          uint32_t ra[32];
-          slot_take(sm, lane_base, g, ra);
-          if (ok && has_a && k < it.n)
-            s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
         }
         g += 2;
         // Each warpgroup keeps its partial sum of every key of a batch of
