@@ -59,7 +59,7 @@ struct Smem {
   uint64_t* tempty;
   uint64_t* done;
   uint32_t* tmem_slot;
-  int* flag;         // [2]: scratch of the publisher warp
+  uint64_t* nap;     // never completed: the normaliser warp sleeps on it between polls
 };
 
 __host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int q_bufs, int R_pad, int stages,
@@ -76,8 +76,8 @@ __host__ __device__ __forceinline__ size_t smem_size(int D, int q_rows, int q_bu
   *poff = off;
   off += sizeof(float2) * kSoftmaxWGs * R_pad;
   *boff = off;
-  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 6);
-  off += sizeof(uint32_t) + 2 * sizeof(int);
+  off += sizeof(uint64_t) * (2 * stages + 4 + 2 * kSlots + 1 + 7);
+  off += sizeof(uint32_t);
   return off;
 }
 
@@ -103,8 +103,8 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const ScoreParams& p, int D
   s.lempty = s.lfull + 2;
   s.pfull = s.lempty + 2;
   s.pempty = s.pfull + 1;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.pempty + 1);
-  s.flag = reinterpret_cast<int*>(s.tmem_slot + 1);
+  s.nap = s.pempty + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.nap + 1);
   return s;
 }
 
@@ -692,28 +692,28 @@ __device__ __forceinline__ void lam_loader(const ScoreParams& p, const Smem& sm,
     const ItemInfo it = decode_item(p, t, load_item(p, t));
     const uint32_t lb = q2 & 1;
     if (!wait_bar_warp(&sm.lempty[lb], ((q2 >> 1) & 1) ^ 1, p)) return;
+    // The whole warp polls the unit's flag; between polls it sleeps on a
+    // shared-memory barrier that never completes (a suspended wait, which
+    // unlike a spin leaves this warp's issue port to the softmax warps that
+    // share it).  The normaliser is needed one entry later at the earliest,
+    // so a microsecond between polls costs nothing.
     int ready = 0;
-    if (lane == 0) {
-      // Polled with a growing sleep: this warp shares an issue port with one
-      // warp of every softmax warpgroup, and a tight poll takes most of its
-      // issue slots.  The normaliser is needed two entries later, so a poll
-      // interval of a microsecond or two costs nothing.
-      const uint64_t t0 = globaltimer_ns();
-      uint32_t spins = 0, sleep_ns = 128;
-      while (!(ready = ld_acquire(&p.ready[it.u]))) {
-        __nanosleep(sleep_ns);
-        if (sleep_ns < 2048) sleep_ns <<= 1;
-        if ((++spins & 7u) == 0) {
-          if (ld_volatile(p.abort_flag)) break;
-          if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
-            atomicExch(p.abort_flag, 1);
-            atomicOr(p.status, kStatusTimeout);
-            break;
-          }
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+      int v = 0, stop = 0;
+      if (lane == 0) {
+        v = ld_acquire(&p.ready[it.u]);
+        if (!v && ld_volatile(p.abort_flag)) stop = 1;
+        if (!v && !stop && globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
+          atomicExch(p.abort_flag, 1);
+          atomicOr(p.status, kStatusTimeout);
+          stop = 1;
         }
       }
+      ready = __shfl_sync(0xffffffffu, v, 0);
+      if (ready || __shfl_sync(0xffffffffu, stop, 0)) break;
+      mbar_try_wait_sleep(sm.nap, 0, 1000);
     }
-    ready = __shfl_sync(0xffffffffu, ready, 0);
     __syncwarp();  // the other lanes read lse2 after lane 0's acquire
     float* lam = sm.lam + lb * p.R_pad;
     for (int r = lane; r < p.R_pad; r += 32)  // stored negated: exp2(s*c + (-lse2))
@@ -754,6 +754,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
     }
     mbar_init(sm.pfull, 4 * kSoftmaxWGs);
     mbar_init(sm.pempty, 1);
+    mbar_init(sm.nap, 1);
     fence_barrier_init();
     fence_proxy_async();
   }
