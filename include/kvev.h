@@ -140,9 +140,14 @@ KVEV_API int kvev_plan_scores_offset(const kvev_plan *plan, int B, int S_cap, in
                                      size_t *byte_offset);
 
 /* Prefill eviction of every layer of the plan in grouped launches.
- *   K[L], V[L]     host arrays of device pointers; layer l's cache is bf16
+ *   K[L], V[L]     host arrays of pointers; layer l's cache is bf16
  *                  [B][H_kv][S_cap][d] (16-byte aligned).  Entries of FULL
- *                  layers may be NULL.
+ *                  layers may be NULL.  K of a SnapKV / H2O layer must be
+ *                  device memory (it is streamed by the tensor-memory
+ *                  accelerator); V of every layer and K of a StreamingLLM layer
+ *                  are only read row by row at the kept positions and may also
+ *                  be pinned host memory that the device addresses directly
+ *                  (unified addressing), which is then read in place.
  *   Q_win[L]       host array of device pointers to the observation-window
  *                  queries, bf16 [B][H_q][W][d] (16-byte aligned); query i of
  *                  the window sits at position lens[s] - W + i.  Needed for
