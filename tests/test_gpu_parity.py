@@ -209,6 +209,34 @@ def test_repeat_calls_identical(torch):
         assert torch.equal(first[k], bufs[k])
 
 
+def test_host_resident_gathered_tensors(torch):
+    # V of every layer and K of the StreamingLLM layers are only gathered at
+    # the kept positions: passed as pinned host memory they are read in place,
+    # with outputs identical to the all-device call.
+    from paper_2606_15157_gb300 import kvev
+    wl = gen.config_tiny(2)
+    dev = host_to_dev(torch, gen.host_tensors(wl))
+    plan = kvev.Plan.from_workload(wl)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    pin = lambda t: None if t is None else t.cpu().pin_memory()
+    scoring = [int(wl.route[l]) in (gen.SNAPKV, gen.H2O) for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    runs = []
+    for host in (False, True):
+        for b in bufs.values():
+            if hasattr(b, "zero_"):
+                b.zero_()
+        K = [dev[l][0] if (scoring[l] or not host) else pin(dev[l][0]) for l in range(wl.L)]
+        V = [pin(dev[l][1]) if host else dev[l][1] for l in range(wl.L)]
+        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+        torch.cuda.synchronize()
+        assert plan.status() == kvev.OK
+        runs.append({k: bufs[k].clone() for k in ("out_K", "out_V", "out_idx", "out_count", "h2o_state")})
+    for k in runs[0]:
+        assert torch.equal(runs[0][k], runs[1][k]), k
+
+
 def test_wait_timeout_reports_status(torch):
     # A unit whose normaliser is never published: every wait on it runs out
     # after the (short) limit, the kernel finishes, the status word says
