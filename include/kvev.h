@@ -84,6 +84,56 @@ KVEV_API int kvev_alloc_from_scores(int32_t *budget_out, const double *s, int L,
  * remainder; no b_min is re-applied.  EINVAL if the input sum is <= 0. */
 KVEV_API int kvev_alloc_rescale(int32_t *budget_out, const int32_t *budget_in, int L, int64_t B_target);
 
+/* ---- plan constructor: route profiles, TopRank, allocation scores -------- */
+/* Host only (no GPU needed); every statistic is computed in fp64. */
+
+#define KVEV_SCOPE_PREFILL 1 /* a route active in the prefill phase only (Sec. 3.1) */
+#define KVEV_SCOPE_DECODE 2  /* ... in the decode phase only */
+#define KVEV_SCOPE_BOTH 3    /* the tied both-phase candidate */
+
+/* Sec. 3.2, representation-similarity profile: C[l][r] = cos(h_full_l, h_r_l).
+ *   h_full   host fp32 [L][D]: FullKV's pooled attention-module output of layer l.
+ *   h_cand   host fp32 [R][L][D]: the same with candidate operator r applied.
+ *   C_out    host fp64 [L][R]; larger is closer to FullKV.
+ * EINVAL: sizes <= 0, a NULL pointer, or a zero or non-finite norm. */
+KVEV_API int kvev_profile_cosine(double *C_out, const float *h_full, const float *h_cand, int L, int R,
+                                 int64_t D);
+
+/* Sec. 3.3, PPL allocation score: s_l = max_r (ppl[l][r] - ppl_full), the
+ * largest perplexity degradation of layer l over the profiled operators.
+ *   ppl      host fp64 [L][R]: perplexity with operator r at layer l only.
+ * EINVAL: sizes <= 0, a NULL pointer, or a non-finite value. */
+KVEV_API int kvev_score_ppl(double *s_out, const double *ppl, double ppl_full, int L, int R);
+
+/* Sec. 3.3, entropy allocation score: H_l = mean over the `rows` attention
+ * rows of layer l (calibration sequences x heads x queries, flattened) of the
+ * Shannon entropy in nats, -sum_k p log p (terms with p = 0 contribute 0).
+ *   A        host fp32 [L][rows][K]: FullKV attention probabilities; masked
+ *            keys are 0 and every row sums to 1 (within 1e-3).
+ * EINVAL: sizes <= 0, a NULL pointer, a negative or non-finite entry, or a
+ * row that is not a distribution. */
+KVEV_API int kvev_score_entropy(double *H_out, const float *A, int L, int64_t rows, int K);
+
+/* Sec. 3.2, Eq. (policy_routing): per layer, the operator with the best
+ * profile statistic.
+ *   g        host fp64 [L][R]: statistic of operator ops[r] at layer l.
+ *   ops[R]   the operator ids (KVEV_*) of the profile's columns.
+ *   covered  host uint8 [L][R] or NULL: 0 excludes an entry (the operator is
+ *            not covered by the profile, or not compatible with the scope).
+ *   higher_is_better  1 for the cosine profile, 0 for the PPL profile.
+ * route_out[l] is ops of the best covered column; equal statistics keep the
+ * column listed first; a layer with no covered column gets KVEV_FULL.
+ * EINVAL: sizes <= 0, a NULL pointer, an unknown operator id, or a
+ * non-finite covered entry. */
+KVEV_API int kvev_route_toprank(int32_t *route_out, const double *g, int L, int R, const int32_t *ops,
+                                const uint8_t *covered, int higher_is_better);
+
+/* Sec. 3.2: install a route in the phases of a scope (KVEV_SCOPE_*): active
+ * phases take route[l], inactive ones KVEV_FULL.  EINVAL if an operator is
+ * not valid in an active phase (SnapKV is prefill only, TOVA decode only). */
+KVEV_API int kvev_route_install(int32_t *route_prefill, int32_t *route_decode, const int32_t *route,
+                                int L, int scope);
+
 /* ---- plan ---------------------------------------------------------------- */
 
 /* Create the static plan of Eq. 1 (host memory only; no device work).
@@ -109,6 +159,19 @@ KVEV_API int kvev_plan_create(kvev_plan **out, int L, int H_q, int H_kv, int d,
                      const int32_t *route_prefill, const int32_t *route_decode,
                      const int32_t *budget, int window, int pool_kernel, int pool_type,
                      int sink, int recent, int h2o_recent);
+
+/* Sec. 3.4: a completed plan is serialised once and loaded at run time.
+ * kvev_plan_save writes the plan's definition (geometry, routes, budgets,
+ * rule parameters) to buf; with buf NULL it only stores the size in *bytes,
+ * otherwise *bytes is the buffer's capacity on entry and the size written on
+ * return.  The format is little-endian: the 8 bytes "KVEVPLN1", then 32-bit
+ * words, then a 64-bit FNV-1a checksum of everything before it.
+ * kvev_plan_load validates the magic, size and checksum and recreates the
+ * plan through kvev_plan_create (same checks, same errors).
+ * EINVAL: NULL pointers, a buffer too small (save), or a corrupt or
+ * truncated buffer (load). */
+KVEV_API int kvev_plan_save(const kvev_plan *plan, void *buf, size_t *bytes);
+KVEV_API int kvev_plan_load(kvev_plan **out, const void *buf, size_t bytes);
 
 /* Release the plan and the small device status buffer it may hold. */
 KVEV_API void kvev_plan_destroy(kvev_plan *plan);

@@ -320,6 +320,79 @@ extern "C" int kvev_plan_create(kvev_plan** out, int L, int H_q, int H_kv, int d
   return KVEV_OK;
 }
 
+// ---- plan serialisation (Sec. 3.4) ------------------------------------------
+namespace {
+
+constexpr char kPlanMagic[8] = {'K', 'V', 'E', 'V', 'P', 'L', 'N', '1'};
+constexpr int kPlanHead = 10;  // words after the magic: L, H_q, H_kv, d, W, pool, type, sink, recent, h2o
+
+uint64_t fnv1a(const uint8_t* p, size_t n) {
+  uint64_t h = 1469598103934665603ULL;
+  for (size_t i = 0; i < n; ++i) {
+    h ^= p[i];
+    h *= 1099511628211ULL;
+  }
+  return h;
+}
+
+size_t plan_bytes(int L) { return 8 + 4 * static_cast<size_t>(kPlanHead + 3 * L) + 8; }
+
+void put32(uint8_t* p, uint32_t v) {
+  for (int i = 0; i < 4; ++i) p[i] = static_cast<uint8_t>(v >> (8 * i));
+}
+uint32_t get32(const uint8_t* p) {
+  uint32_t v = 0;
+  for (int i = 0; i < 4; ++i) v |= static_cast<uint32_t>(p[i]) << (8 * i);
+  return v;
+}
+
+}  // namespace
+
+extern "C" int kvev_plan_save(const kvev_plan* plan, void* buf, size_t* bytes) {
+  if (!plan || !bytes) return KVEV_EINVAL;
+  const kvev_plan& P = *plan;
+  const size_t need = plan_bytes(P.L);
+  if (!buf) {
+    *bytes = need;
+    return KVEV_OK;
+  }
+  if (*bytes < need) return KVEV_EINVAL;
+  uint8_t* o = static_cast<uint8_t*>(buf);
+  std::memcpy(o, kPlanMagic, 8);
+  size_t at = 8;
+  const int32_t head[kPlanHead] = {P.L, P.H_q, P.H_kv, P.d, P.W, P.pool_kernel, P.pool_type,
+                                   P.sink, P.recent, P.h2o_recent};
+  for (int i = 0; i < kPlanHead; ++i, at += 4) put32(o + at, static_cast<uint32_t>(head[i]));
+  for (const std::vector<int>* v : {&P.route_pre, &P.route_dec, &P.budget})
+    for (int l = 0; l < P.L; ++l, at += 4) put32(o + at, static_cast<uint32_t>((*v)[l]));
+  const uint64_t h = fnv1a(o, at);
+  put32(o + at, static_cast<uint32_t>(h));
+  put32(o + at + 4, static_cast<uint32_t>(h >> 32));
+  *bytes = need;
+  return KVEV_OK;
+}
+
+extern "C" int kvev_plan_load(kvev_plan** out, const void* buf, size_t bytes) {
+  if (!out) return KVEV_EINVAL;
+  *out = nullptr;
+  if (!buf || bytes < 8 + 4 * kPlanHead + 8) return KVEV_EINVAL;
+  const uint8_t* in = static_cast<const uint8_t*>(buf);
+  if (std::memcmp(in, kPlanMagic, 8) != 0) return KVEV_EINVAL;
+  const int32_t L = static_cast<int32_t>(get32(in + 8));
+  if (L <= 0 || L > kMaxLayers || bytes != plan_bytes(L)) return KVEV_EINVAL;
+  const size_t body = bytes - 8;
+  const uint64_t h = static_cast<uint64_t>(get32(in + body)) | (static_cast<uint64_t>(get32(in + body + 4)) << 32);
+  if (h != fnv1a(in, body)) return KVEV_EINVAL;
+  int32_t head[kPlanHead];
+  for (int i = 0; i < kPlanHead; ++i) head[i] = static_cast<int32_t>(get32(in + 8 + 4 * i));
+  std::vector<int32_t> pre(L), dec(L), bud(L);
+  size_t at = 8 + 4 * kPlanHead;
+  for (std::vector<int32_t>* v : {&pre, &dec, &bud})
+    for (int l = 0; l < L; ++l, at += 4) (*v)[l] = static_cast<int32_t>(get32(in + at));
+  return kvev_plan_create(out, L, head[1], head[2], head[3], pre.data(), dec.data(), bud.data(), head[4],
+                          head[5], head[6], head[7], head[8], head[9]);
+}
+
 extern "C" void kvev_plan_destroy(kvev_plan* plan) {
   if (!plan) return;
   if (plan->ctx.status) cudaFree(plan->ctx.status);

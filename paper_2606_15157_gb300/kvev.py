@@ -20,6 +20,7 @@ OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE, ENOTSUP = range(7)
 FULL, SNAPKV, H2O, STREAMING, TOVA = 0, 1, 2, 3, 4
 POOL_MAX, POOL_AVG = 0, 1
 T_IDENTITY, T_CAP_Q95 = 0, 1
+SCOPE_PREFILL, SCOPE_DECODE, SCOPE_BOTH = 1, 2, 3
 
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA",
                 ETIMEOUT: "ETIMEOUT", EDEVICE: "EDEVICE", ENOTSUP: "ENOTSUP"}
@@ -30,7 +31,8 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
            "kvev_plan_last_timings", "kvev_evict_prefill_noalloc", "kvev_decode_query",
            "kvev_decode_layer", "kvev_decode_state_offsets", "kvev_decode_init",
-           "kvev_decode_step"]
+           "kvev_decode_step", "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
+           "kvev_route_toprank", "kvev_route_install", "kvev_plan_save", "kvev_plan_load"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
 
 
@@ -79,6 +81,13 @@ def load(path: str = LIB_PATH):
         L.kvev_decode_state_offsets.argtypes = [vp, C.c_int, C.c_int, P(sz)]
         L.kvev_decode_init.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
         L.kvev_decode_step.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
+        L.kvev_profile_cosine.argtypes = [vp, vp, vp, C.c_int, C.c_int, i64]
+        L.kvev_score_ppl.argtypes = [vp, vp, C.c_double, C.c_int, C.c_int]
+        L.kvev_score_entropy.argtypes = [vp, vp, C.c_int, i64, C.c_int]
+        L.kvev_route_toprank.argtypes = [vp, vp, C.c_int, C.c_int, vp, vp, C.c_int]
+        L.kvev_route_install.argtypes = [vp, vp, vp, C.c_int, C.c_int]
+        L.kvev_plan_save.argtypes = [vp, vp, P(sz)]
+        L.kvev_plan_load.argtypes = [P(vp), vp, sz]
         for name in EXPORTS:
             if name != "kvev_plan_destroy":
                 getattr(L, name).restype = C.c_int
@@ -238,6 +247,74 @@ def kvev_plan_debug_stall_unit(handle: int, unit: int):
     _check(load().kvev_plan_debug_stall_unit(handle, int(unit)), "kvev_plan_debug_stall_unit")
 
 
+def kvev_profile_cosine(h_full, h_cand) -> np.ndarray:
+    """Sec. 3.2 cosine profile: h_full [L, D], h_cand [R, L, D] -> C [L, R] (fp64)."""
+    hf = np.ascontiguousarray(h_full, np.float32)
+    hc = np.ascontiguousarray(h_cand, np.float32)
+    L, D = hf.shape
+    R = hc.shape[0]
+    assert hc.shape == (R, L, D)
+    out = np.zeros((L, R), np.float64)
+    _check(load().kvev_profile_cosine(out.ctypes.data, hf.ctypes.data, hc.ctypes.data, L, R, D),
+           "kvev_profile_cosine")
+    return out
+
+
+def kvev_score_ppl(ppl, ppl_full: float) -> np.ndarray:
+    """Sec. 3.3 PPL allocation score: max_r (ppl[l, r] - ppl_full)."""
+    p = np.ascontiguousarray(ppl, np.float64)
+    L, R = p.shape
+    out = np.zeros(L, np.float64)
+    _check(load().kvev_score_ppl(out.ctypes.data, p.ctypes.data, float(ppl_full), L, R), "kvev_score_ppl")
+    return out
+
+
+def kvev_score_entropy(A) -> np.ndarray:
+    """Sec. 3.3 entropy allocation score of attention rows A [L, rows, K] (nats)."""
+    a = np.ascontiguousarray(A, np.float32)
+    L, rows, K = a.shape
+    out = np.zeros(L, np.float64)
+    _check(load().kvev_score_entropy(out.ctypes.data, a.ctypes.data, L, rows, K), "kvev_score_entropy")
+    return out
+
+
+def kvev_route_toprank(g, ops, higher_is_better: bool, covered=None) -> np.ndarray:
+    """Eq. (policy_routing): per layer, the operator of the best covered column of g [L, R]."""
+    gg = np.ascontiguousarray(g, np.float64)
+    L, R = gg.shape
+    o = np.ascontiguousarray(ops, np.int32)
+    cv = None if covered is None else np.ascontiguousarray(covered, np.uint8)
+    out = np.zeros(L, np.int32)
+    _check(load().kvev_route_toprank(out.ctypes.data, gg.ctypes.data, L, R, o.ctypes.data,
+                                     None if cv is None else cv.ctypes.data, int(bool(higher_is_better))),
+           "kvev_route_toprank")
+    return out
+
+
+def kvev_route_install(route, scope: int):
+    """Active phases of the scope take route[l], the others FULL: (route_prefill, route_decode)."""
+    r = np.ascontiguousarray(route, np.int32)
+    pre, dec = np.zeros(len(r), np.int32), np.zeros(len(r), np.int32)
+    _check(load().kvev_route_install(pre.ctypes.data, dec.ctypes.data, r.ctypes.data, len(r), int(scope)),
+           "kvev_route_install")
+    return pre, dec
+
+
+def kvev_plan_save(handle: int) -> bytes:
+    n = C.c_size_t(0)
+    _check(load().kvev_plan_save(handle, None, C.byref(n)), "kvev_plan_save")
+    buf = C.create_string_buffer(n.value)
+    _check(load().kvev_plan_save(handle, buf, C.byref(n)), "kvev_plan_save")
+    return buf.raw[:n.value]
+
+
+def kvev_plan_load(data: bytes) -> int:
+    h = C.c_void_p()
+    buf = C.create_string_buffer(bytes(data), len(data))
+    _check(load().kvev_plan_load(C.byref(h), buf, len(data)), "kvev_plan_load")
+    return h.value
+
+
 def alloc_pyramid(L: int, B_total: int, b_min: int) -> np.ndarray:
     """Pyramidal schedule: weights decreasing linearly with depth (1.5 -> 0.5) fed to Eq. 3."""
     w = np.ones(1) if L == 1 else 1.5 - np.arange(L) / (L - 1)
@@ -278,6 +355,22 @@ class Plan:
 
     def query(self, B, S_cap):
         return kvev_plan_query(self.handle, B, S_cap)
+
+    def save(self) -> bytes:
+        """The plan's serialised definition (Sec. 3.4)."""
+        return kvev_plan_save(self.handle)
+
+    @classmethod
+    def load(cls, data: bytes) -> "Plan":
+        """A plan recreated from kvev_plan_save bytes."""
+        obj = cls.__new__(cls)
+        obj.handle = kvev_plan_load(data)
+        words = np.frombuffer(bytes(data)[8:-8], dtype="<i4")
+        L = int(words[0])
+        obj.L, obj.H_q, obj.H_kv, obj.d, obj.window = L, int(words[1]), int(words[2]), int(words[3]), int(words[4])
+        obj.route = words[10:10 + L].astype(np.int32)
+        obj.budget = words[10 + 2 * L:10 + 3 * L].astype(np.int32)
+        return obj
 
     def layer_offset(self, B, layer):
         return kvev_plan_layer_offset(self.handle, B, layer)
