@@ -407,22 +407,28 @@ __device__ __forceinline__ void s1_chunk64(const float (&v0)[32], const float (&
 
 // One 32-row chunk of sweep 2 for this thread's key: sum of exp2(s*c - lse2_r)
 // into four packed accumulators; nl = -lse2 of the chunk's rows (shared memory).
+// Every row of the chunk counts for this key: no per-element checks.
+__device__ __forceinline__ void s2_chunk_full(const uint32_t (&rr)[32], float c, const float* nl,
+                                              float2 (&a)[4]) {
+  const float2 cc = make_float2(c, c);
+#pragma unroll
+  for (int i = 0; i < 32; i += 4) {
+    const float4 l4 = lds4(nl + i);
+    const float2 t0 = ffma2(make_float2(__uint_as_float(rr[i]), __uint_as_float(rr[i + 1])), cc,
+                            make_float2(l4.x, l4.y));
+    const float2 t1 = ffma2(make_float2(__uint_as_float(rr[i + 2]), __uint_as_float(rr[i + 3])),
+                            cc, make_float2(l4.z, l4.w));
+    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+    a[((i >> 1) + 1) & 3] =
+        fadd2(a[((i >> 1) + 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
+  }
+}
+
 __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&rr)[32], bool full,
                                          const float* nl, int r0, int k, int n, float2 (&a)[4]) {
   const float c = p.scale_log2;
-  const float2 cc = make_float2(c, c);
   if (full) {
-#pragma unroll
-    for (int i = 0; i < 32; i += 4) {
-      const float4 l4 = lds4(nl + i);
-      const float2 t0 = ffma2(make_float2(__uint_as_float(rr[i]), __uint_as_float(rr[i + 1])), cc,
-                              make_float2(l4.x, l4.y));
-      const float2 t1 = ffma2(make_float2(__uint_as_float(rr[i + 2]), __uint_as_float(rr[i + 3])),
-                              cc, make_float2(l4.z, l4.w));
-      a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
-      a[((i >> 1) + 1) & 3] =
-          fadd2(a[((i >> 1) + 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
-    }
+    s2_chunk_full(rr, c, nl, a);
   } else {
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
@@ -551,10 +557,15 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
         {
           uint32_t ra[32], rb[32];
           unit_take(sm, lane_base, g, ra, rb);
-          if (ok && has_a && k < it.n)
-            s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
-          if (ok && has_b && k < it.n)
-            s2_chunk(p, rb, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
+          if (ok && key_full && r0b + 32 <= p.R) {  // the common case: every key and row counts
+            s2_chunk_full(ra, p.scale_log2, lam + r0a, a);
+            s2_chunk_full(rb, p.scale_log2, lam + r0b, a);
+          } else {
+            if (ok && has_a && k < it.n)
+              s2_chunk(p, ra, key_full && r0a + 32 <= p.R, lam + r0a, r0a, k, it.n, a);
+            if (ok && has_b && k < it.n)
+              s2_chunk(p, rb, key_full && r0b + 32 <= p.R, lam + r0b, r0b, k, it.n, a);
+          }
         }
         g += 2;
         // Each warpgroup keeps its partial sum of every key of a batch of
