@@ -40,6 +40,7 @@ struct kvev_plan {
   std::vector<int> score_layers;
   int64_t wait_ns = 2000000000LL;
   int stall_unit = -1;
+  bool h2o_full = false;  // H2O prefill scores accumulate over every prompt query row
   // device-side state, created on first use (status word allocated lazily)
   DevCtx ctx;
   cudaStream_t last_stream = nullptr;
@@ -115,6 +116,22 @@ bool encode_map(CUtensorMap* m, const void* base, int d, uint64_t rows, int box_
   cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// Whole-prompt queries bf16 [B*H_q][S_cap][d] as a 3-D map whose box is G
+// heads x W positions x 64 columns: it lands as the G*W rows of 128 bytes of
+// a window (head-major), the layout of the 2-D window map.
+bool encode_map_prompt(CUtensorMap* m, const void* base, int d, int S_cap, uint64_t heads, int W, int G) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(S_cap), heads};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(S_cap) * d * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(W), static_cast<cuuint32_t>(G)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -460,6 +477,12 @@ extern "C" int kvev_plan_scores_offset(const kvev_plan* plan, int B, int S_cap, 
   return KVEV_OK;
 }
 
+extern "C" int kvev_plan_set_h2o_full_prompt(kvev_plan* plan, int on) {
+  if (!plan || (on != 0 && on != 1)) return KVEV_EINVAL;
+  plan->h2o_full = on == 1;
+  return KVEV_OK;
+}
+
 extern "C" int kvev_plan_set_wait_limit(kvev_plan* plan, int64_t ns) {
   if (!plan || ns <= 0) return KVEV_EINVAL;
   plan->wait_ns = ns;
@@ -606,21 +629,29 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
       if (which == 1) P.launched[k] = true;
     }
   };
-  mark(KVEV_K_PROLOGUE, 0);
-  if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
-  mark(KVEV_K_PROLOGUE, 1);
+  pp.W = P.W;
+  bool any_h2o = false;
+  for (int i = 0; i < n_slayers; ++i) any_h2o |= P.route_pre[P.score_layers[i]] == KVEV_H2O;
+  // H2O prefill scores over every prompt query row: scored by row blocks of W
+  // positions (blocks of one launch each), accumulated in the score array
+  const bool blocks = P.h2o_full && any_h2o;
 
   // ---- window scores ----------------------------------------------------
+  ScoreParams sp;
+  std::memset(&sp, 0, sizeof(sp));
+  int score_grid = 0;
+  size_t score_smem = 0;
   if (ws.n_units > 0) {
-    ScoreParams sp;
-    std::memset(&sp, 0, sizeof(sp));
     const int q_rows = ws.R_pad > 128 ? 256 : 128;
     for (int i = 0; i < n_slayers; ++i) {
       const int l = P.score_layers[i];
       if (!encode_map(&sp.kmap[i], K[l], P.d, static_cast<uint64_t>(B) * P.H_kv * S_cap,
                       kSuperKeys) ||
-          !encode_map(&sp.qmap[i], Q_win[l], P.d, static_cast<uint64_t>(B) * P.H_q * P.W,
-                      ws.R_pad))
+          !(blocks && P.route_pre[l] == KVEV_H2O
+                ? encode_map_prompt(&sp.qmap[i], Q_win[l], P.d, S_cap, static_cast<uint64_t>(B) * P.H_q,
+                                    P.W, P.G)
+                : encode_map(&sp.qmap[i], Q_win[l], P.d, static_cast<uint64_t>(B) * P.H_q * P.W,
+                             ws.R_pad)))
         return KVEV_ECUDA;
     }
     // K stages (256-key super-tiles) that fit next to q_bufs Q buffers.  A
@@ -678,8 +709,52 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
     sp.wait_ns = P.wait_ns;
     sp.stall_unit = P.stall_unit;
+    score_grid = grid;
+    score_smem = smem;
+  }
+  // one prologue + score pass; the first prologue also validates the lengths
+  auto pass = [&](int mode, int win0) -> int {
+    pp.mode = mode;
+    pp.win0 = win0;
+    if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+    if (ws.n_units == 0) return KVEV_OK;
+    sp.row_min = mode == kScoreH2OBlock ? win0 : 0;
+    sp.q_full = mode == kScoreH2OBlock;
+    sp.accumulate = mode == kScoreH2OBlock;
+    return launch_score(sp, P.d, score_grid, score_smem, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
+  };
+  if (!blocks) {
+    mark(KVEV_K_PROLOGUE, 0);
+    pp.mode = kScoreAll;
+    pp.win0 = 0;
+    if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+    mark(KVEV_K_PROLOGUE, 1);
+    if (ws.n_units > 0) {
+      mark(KVEV_K_SCORE, 0);
+      sp.row_min = 0;
+      sp.q_full = 0;
+      sp.accumulate = 0;
+      if (launch_score(sp, P.d, score_grid, score_smem, s) != cudaSuccess) return KVEV_ECUDA;
+      mark(KVEV_K_SCORE, 1);
+    }
+  } else {
+    // H2O score arrays start from zero; each block adds its rows' attention
+    const size_t per_slot = static_cast<size_t>(B) * P.H_kv * S_cap;
+    float* raw = reinterpret_cast<float*>(wsb + ws.raw);
+    for (int i = 0; i < n_slayers; ++i)
+      if (P.route_pre[P.score_layers[i]] == KVEV_H2O &&
+          cudaMemsetAsync(raw + static_cast<size_t>(i) * per_slot, 0, per_slot * sizeof(float), s) !=
+              cudaSuccess)
+        return KVEV_ECUDA;
+    mark(KVEV_K_PROLOGUE, 0);
+    mark(KVEV_K_PROLOGUE, 1);
     mark(KVEV_K_SCORE, 0);
-    if (launch_score(sp, P.d, grid, smem, s) != cudaSuccess) return KVEV_ECUDA;
+    for (int win0 = 0; win0 < S_cap; win0 += P.W) {
+      const int rc = pass(kScoreH2OBlock, win0);
+      if (rc != KVEV_OK) return rc;
+    }
+    const int rc = pass(kScoreNoH2O, 0);  // SnapKV layers, and the lengths the selection reads
+    if (rc != KVEV_OK) return rc;
     mark(KVEV_K_SCORE, 1);
   }
 

@@ -23,6 +23,10 @@ constexpr int kMinChunkTiles = 16;
 // The per-row (max, sum) records of a unit's chunks are merged up a tree of
 // fan-in kTreeFanIn (the last child to arrive merges its siblings), so the
 // normaliser is ready a few load round trips after the unit's last chunk.
+// What a prologue + score launch covers (PrologueParams::mode).
+constexpr int kScoreAll = 0;       // every scoring layer, rows = the observation window
+constexpr int kScoreNoH2O = 1;     // SnapKV layers only (H2O layers are scored by row blocks)
+constexpr int kScoreH2OBlock = 2;  // H2O layers, rows = one block of W prompt positions
 constexpr int kTreeFanIn = 4;
 constexpr int kTreeLevels = 5;        // internal levels: up to 4^5 = 1024 chunks per unit
 constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel
@@ -66,6 +70,9 @@ struct PrologueParams {
   int* status;
   int* node_cnt;      // [items][kTreeLevels] arrival counters of the merge tree (zeroed here)
   int n_node_cnt;     // counters in node_cnt (workspace capacity)
+  int W;              // observation window (the row block of kScoreH2OBlock)
+  int mode;           // kScoreAll, kScoreNoH2O, or kScoreH2OBlock (H2O rows [win0, win0 + W))
+  int win0;           // first query position of the row block (kScoreH2OBlock)
   int* ready;
   int* abort_flag;
   int* chunk_start;   // [n_units + 1]
@@ -78,6 +85,10 @@ struct ScoreParams {
   int n_units, B, H_kv, H_q, G, W, R, R_pad, S_cap;
   int chunk_keys;     // keys per work item (multiple of 128)
   int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
+  int row_min;        // window rows at positions below this do not exist (a partial row block)
+  int q_full;         // Q maps cover the whole prompt, bf16 [B*H_q][S_cap][d] (3-D, one box of
+                      // G heads x W positions ending at the unit's length)
+  int accumulate;     // add the scores to raw instead of storing them (row blocks of a prompt)
   int q_bufs;         // Q buffers (2: the next entry's Q loads during this entry; 1: it
                       // loads once this entry is done, leaving room for more K stages)
   int stages;         // K tile ring depth
@@ -242,6 +253,15 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
 }
 
 // Same, with an L2 cache-eviction policy (from createpolicy).
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d_hint(void* dst, const CUtensorMap* map, int x, int y,
                                                  uint64_t* bar, uint64_t policy) {
   asm volatile(

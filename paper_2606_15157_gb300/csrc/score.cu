@@ -203,6 +203,16 @@ __device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, u
 template <int D>
 __device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uint32_t e, const ItemInfo& it) {
   const uint32_t qb = e % p.q_bufs;
+  if (p.q_full) {
+    // G heads x the last W positions of the (truncated) prompt, one 3-D box per
+    // 64-column block; it lands as the same G*W rows of 128 bytes
+    mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R) * D * 2);
+#pragma unroll
+    for (int kc = 0; kc < D / 64; ++kc)
+      tma_load_3d(sm.qbuf + qb * sm.qbytes + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
+                  kc * 64, it.n - p.W, it.s * p.H_q + it.h * p.G, &sm.qfull[qb]);
+    return;
+  }
   mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R_pad) * D * 2);
   const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
 #pragma unroll
@@ -362,6 +372,13 @@ __device__ __forceinline__ int row_pos(const ScoreParams& p, int r, int n) {
   return n - p.W + (r % p.W);
 }
 
+// Position of row r if the row exists, else -1: rows before the sequence
+// start, and rows of a partial row block that belong to the previous block.
+__device__ __forceinline__ int row_live(const ScoreParams& p, int r, int n) {
+  const int t = row_pos(p, r, n);
+  return t >= p.row_min ? t : -1;
+}
+
 __device__ __forceinline__ float max32(const float (&v)[32]) {
   float t[11];
 #pragma unroll
@@ -433,7 +450,7 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       const int r = r0 + i;
-      if (r < p.R && k <= row_pos(p, r, n)) {
+      if (r < p.R && k <= row_live(p, r, n)) {
         const float e = ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
         if (i & 1) a[(i >> 1) & 3].y += e; else a[(i >> 1) & 3].x += e;
       }
@@ -495,8 +512,10 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       const int t = first + jj * stride;
       const ItemInfo it = decode_item(p, t, load_item(p, t));
       float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
-      const int tr0 = lrow < p.R ? row_pos(p, lrow, it.n) : -1;
-      const int tr1 = 128 + lrow < p.R ? row_pos(p, 128 + lrow, it.n) : -1;
+      const int tr0 = lrow < p.R ? row_live(p, lrow, it.n) : -1;
+      const int tr1 = 128 + lrow < p.R ? row_live(p, 128 + lrow, it.n) : -1;
+      // every row of the window exists (no row before the sequence or the block)
+      const bool rows_all = it.n - p.W >= p.row_min;
       // One unit per (256-key super-tile, 128-row group): this warpgroup's 32
       // keys of each 128-key half, for the thread's row of the group.  Rows
       // that do not exist (tr < 0) are computed like the others and dropped
@@ -505,7 +524,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int j = 0; j < nst; ++j) {
         const int kb = it.key0 + j * kSuperKeys;
         const int k0 = kb + 64 * wg;                       // keys k0 .. k0 + 63
-        const bool full = kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
+        const bool full = rows_all && kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
         for (int h = 0; h < nh; ++h) {
           ok = slot_wait(p, sm, g, ok);
           uint32_t r0[32], r1[32];
@@ -550,7 +569,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int i = 0; i < it.ntiles; ++i) {
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
-        const bool key_full = kb + kTileKeys - 1 <= it.n - p.W;
+        const bool key_full = it.n - p.W >= p.row_min && kb + kTileKeys - 1 <= it.n - p.W;
         float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
         ok = slot_wait(p, sm, g, ok);
@@ -581,7 +600,12 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             float sum = 0.f;
 #pragma unroll
             for (int w = 0; w < kSoftmaxWGs; ++w) sum += sm.red[w * kRedTiles * 128 + q];
-            if (ok && key0 + q < it.n) out[key0 + q] = sum * p.inv_G;
+            if (ok && key0 + q < it.n) {
+              if (p.accumulate)
+                out[key0 + q] += sum * p.inv_G;
+              else
+                out[key0 + q] = sum * p.inv_G;
+            }
           }
           // the batch's rows may be overwritten, and after the entry's last
           // batch every warpgroup is done reading lam
@@ -806,6 +830,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
 __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ PrologueParams p) {
   __shared__ int warp_sums[32];
   __shared__ int carry;
+  __shared__ int unit_len[1024];  // length each unit is scored over
   const int tid = threadIdx.x;
   if (tid == 0) {
     carry = 0;
@@ -828,9 +853,17 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     if (u < p.n_units) {
       const int ls = u / per_layer;
       const int s = (u - ls * per_layer) / p.H_kv;
-      const int n = p.lens[s];
-      const bool need = n > 0 && (p.slayer_method[ls] == KVEV_H2O || n > p.slayer_budget[ls]);
+      int n = p.lens[s];
+      const bool h2o = p.slayer_method[ls] == KVEV_H2O;
+      bool need = n > 0 && (h2o || n > p.slayer_budget[ls]);
+      if (p.mode == kScoreNoH2O && h2o) need = false;
+      if (p.mode == kScoreH2OBlock) {
+        // the prompt truncated after the block: its last W positions are the rows
+        n = min(n, p.win0 + p.W);
+        need = h2o && n > p.win0;
+      }
       c = need ? (n + p.chunk_keys - 1) / p.chunk_keys : 0;
+      unit_len[tid] = n;
       p.ready[u] = 0;
     }
     // block-wide exclusive scan of c
@@ -856,7 +889,7 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     const int excl = carry + (w > 0 ? warp_sums[w - 1] : 0) + x - c;
     if (u < p.n_units) {
       p.chunk_start[u] = excl;
-      const int n = p.lens[(u % per_layer) / p.H_kv];
+      const int n = unit_len[tid];
       for (int q = 0; q < c; ++q) {
         const int key0 = q * p.chunk_keys;
         const int nk = min(p.chunk_keys, n - key0);

@@ -32,7 +32,8 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_last_timings", "kvev_evict_prefill_noalloc", "kvev_decode_query",
            "kvev_decode_layer", "kvev_decode_state_offsets", "kvev_decode_init",
            "kvev_decode_step", "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
-           "kvev_route_toprank", "kvev_route_install", "kvev_plan_save", "kvev_plan_load"]
+           "kvev_route_toprank", "kvev_route_install", "kvev_plan_save", "kvev_plan_load",
+           "kvev_plan_set_h2o_full_prompt"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
 
 
@@ -88,6 +89,7 @@ def load(path: str = LIB_PATH):
         L.kvev_route_install.argtypes = [vp, vp, vp, C.c_int, C.c_int]
         L.kvev_plan_save.argtypes = [vp, vp, P(sz)]
         L.kvev_plan_load.argtypes = [P(vp), vp, sz]
+        L.kvev_plan_set_h2o_full_prompt.argtypes = [vp, C.c_int]
         for name in EXPORTS:
             if name != "kvev_plan_destroy":
                 getattr(L, name).restype = C.c_int
@@ -329,13 +331,15 @@ class Plan:
     """Owns a kvev plan; allocates outputs/workspace as torch CUDA tensors."""
 
     def __init__(self, L, H_q, H_kv, d, route, budget, window, pool_kernel=7, pool_type=POOL_AVG,
-                 sink=4, recent=-1, h2o_recent=-1, route_decode=None):
+                 sink=4, recent=-1, h2o_recent=-1, route_decode=None, h2o_full_prompt=False):
         self.L, self.H_q, self.H_kv, self.d = L, H_q, H_kv, d
         self.route = np.asarray(route, np.int32)
         self.budget = np.asarray(budget, np.int32)
         self.window = window
         self.handle = kvev_plan_create(L, H_q, H_kv, d, self.route, route_decode, self.budget,
                                        window, pool_kernel, pool_type, sink, recent, h2o_recent)
+        if h2o_full_prompt:
+            _check(load().kvev_plan_set_h2o_full_prompt(self.handle, 1), "kvev_plan_set_h2o_full_prompt")
 
     @classmethod
     def from_workload(cls, wl):

@@ -140,6 +140,39 @@ def test_scores_total_mass_equals_window_rows(orc, n, W, G, d):
     assert (raw >= 0).all()
 
 
+@pytest.mark.parametrize("n", [1, 37, 300])
+def test_full_prompt_scores_closed_form_and_mass(orc, n):
+    # H2O's full-prompt accumulation is the window score with every prompt
+    # position as a query row (W = n).  Equal logits: query t puts 1/(t+1) on
+    # keys 0..t, so raw[k] = sum_{t=k}^{n-1} 1/(t+1) = H_n - H_k (harmonic
+    # numbers); and every row's distribution sums to 1, so sum_k raw[k] = n.
+    rng = np.random.default_rng(9)
+    d, G = 64, 3
+    K = rand_bf16(rng, (n, d))
+    raw = orc.window_scores(K, np.zeros((G, n, d), np.uint16), n, n)
+    tail = np.cumsum((1.0 / np.arange(1, n + 1))[::-1])[::-1]  # H_n - H_k without cancellation
+    assert np.allclose(raw, tail, rtol=1e-13, atol=0)
+    Q = rand_bf16(rng, (G, n, d))
+    raw = orc.window_scores(K, Q, n, n)
+    assert abs(raw.sum() - n) <= 1e-9 * n
+
+
+def test_full_prompt_scores_are_sums_of_row_blocks(orc):
+    # The accumulation over all rows splits into blocks of W consecutive
+    # positions, block j scored as the window of the prompt truncated after it
+    # (the row-block decomposition the GPU path uses).
+    rng = np.random.default_rng(10)
+    n, W, d, G = 96, 16, 64, 2
+    K = rand_bf16(rng, (n, d))
+    Q = rand_bf16(rng, (G, n, d))
+    full = orc.window_scores(K, Q, n, n)
+    acc = np.zeros(n)
+    for j in range(n // W):
+        m = (j + 1) * W
+        acc[:m] += orc.window_scores(K[:m], np.ascontiguousarray(Q[:, j * W:m]), m, W)
+    assert np.allclose(acc, full, rtol=1e-12, atol=1e-15)
+
+
 @pytest.mark.parametrize("n,W", [(50, 8), (6, 8), (9, 9)])
 def test_scores_uniform_logits_closed_form(orc, n, W):
     # Q = 0 gives equal logits: row i (position t_i = n-W+i) puts 1/(t_i+1) on
