@@ -246,7 +246,7 @@ KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const voi
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
                        float *h2o_state, void *workspace, size_t workspace_bytes, void *stream);
 
-/* SURVEY N2 / Sec. 2.1 (H2O's original scoring): with on = 1, the prefill
+/* Sec. 2.1 (H2O's original scoring): with on = 1, the prefill
  * scores of the plan's H2O layers accumulate the attention of every prompt
  * query row, raw[k] = (1/G) sum_g sum_{t=k}^{n-1} p_{g,t}(k), instead of the
  * observation window's.  Q_win[l] of an H2O layer is then the whole prompt's
