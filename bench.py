@@ -61,6 +61,20 @@ def unit_bytes(wl, l: int, n: int) -> tuple[int, int]:
     return 0, 0
 
 
+def score_flops(wl) -> int:
+    """Tensor-core work of the window-score kernel: Q_win K^T (2 R n d flops
+    for R = G W rows and n keys) once per sweep, two sweeps per unit (the row
+    normaliser needs every key before any score is final)."""
+    tot = 0
+    for l in range(wl.L):
+        m, b = int(wl.route[l]), int(wl.budget[l])
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            if m == gen.H2O or (m == gen.SNAPKV and n > b):
+                tot += 2 * (2 * wl.G * wl.W * n * wl.d) * wl.H_kv
+    return tot
+
+
 def workload_bytes(wl):
     tot = sc = ev = 0
     for l in range(wl.L):
@@ -320,6 +334,8 @@ def run_ours(args, rank, world, local_rank):
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
     score_ms = statistics.mean(per_kernel["score"]) if per_kernel["score"] else float("nan")
     achieved = score_bytes / (score_ms / 1e3) / 1e9
+    tc_peak = float(peaks.get("bf16_tflops", 1900.0))
+    tc_achieved = score_flops(wl) / (score_ms / 1e3) / 1e12
     kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
     traffic = None
     tf = os.path.join(ROOT, "profiles", "score_traffic.json")
@@ -365,7 +381,12 @@ def run_ours(args, rank, world, local_rank):
             "kernel_ms": kernel_ms,
             "roofline": {"kernel": "score_kernel", "bound": "hbm", "achieved": achieved,
                          "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
-                         "traffic": traffic, "peak_source": peak_src},
+                         "traffic": traffic, "peak_source": peak_src,
+                         "tensor_pipe": {"achieved": tc_achieved, "peak": tc_peak, "unit": "TFLOP/s",
+                                         "frac": tc_achieved / tc_peak,
+                                         "work": "two sweeps of Q_win K^T (bf16 in, fp32 accumulate)",
+                                         "peak_source": "measured" if "bf16_tflops" in peaks
+                                         else "fallback"}},
             "clocks": clocks,
             "gpu_launches": kernels_launched,
             "e2e": e2e,

@@ -790,8 +790,16 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.raw = reinterpret_cast<float*>(wsb + ws.raw);
   sel.out_idx = out_idx;
   sel.out_count = out_count;
-  const size_t sel_smem = ws.n_units > 0 ? sizeof(uint32_t) * static_cast<size_t>(S_cap) : 0;
-  if (sel_smem + 4096 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
+  // dynamic shared memory of the selection: the unit's keys, then as many
+  // candidate positions (at most S_cap) as fit next to the static part
+  size_t sel_smem = 0;
+  if (ws.n_units > 0) {
+    const size_t keys_b = sizeof(uint32_t) * static_cast<size_t>(S_cap);
+    if (keys_b + kSelectStaticSmem + 1024 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
+    const size_t room = static_cast<size_t>(D.smem_optin) - kSelectStaticSmem - 1024 - keys_b;
+    sel.cand_cap = static_cast<int>(std::min<size_t>(room / sizeof(int), static_cast<size_t>(S_cap)));
+    sel_smem = keys_b + sizeof(int) * static_cast<size_t>(sel.cand_cap);
+  }
   if (sel_smem > 48 * 1024 && D.select_smem_set < sel_smem) {
     if (select_set_smem(sel_smem) != cudaSuccess) return KVEV_ECUDA;
     D.select_smem_set = sel_smem;

@@ -43,6 +43,7 @@ constexpr int kRegsControl = 64;
 constexpr int kRegsSoftmax = 104;
 constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
 constexpr int kSelectThreads = 1024;
+constexpr int kSelectStaticSmem = 17 * 1024;  // bound on the select kernel's static shared memory
 constexpr int kWsAlign = 256;
 
 // Bits of the device status word.
@@ -116,6 +117,7 @@ struct SelectParams {
   const float* raw;   // [n_units][S_cap]
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
+  int cand_cap;       // candidate positions that fit after the keys in dynamic shared memory
 };
 
 // Per-layer description of the decode arena.

@@ -12,29 +12,61 @@
 // Top-k order: larger score first, equal scores keep the lower position.
 // Output indices are ascending; unused slots hold -1.
 //
-// The k-th largest key is found by a 4-pass 8-bit radix select over an
-// order-preserving uint32 image of the fp32 scores held in shared memory,
-// then one ordered pass (ballot/popc prefix counts) writes the kept positions.
+// The k-th largest key is found over an order-preserving uint32 image of the
+// fp32 scores held in shared memory.  The pass that builds the keys also
+// histograms their top 12 bits; the bin holding the k-th key is then the only
+// one that matters: one pass gathers its positions (and counts, per warp
+// segment, the keys above it), two 10-bit radix passes over those candidates
+// alone fix the threshold key, and one ordered pass (ballot/popc prefix
+// counts) writes the kept positions.  Three passes over the unit's keys in
+// all; a first bin too crowded for the candidate buffer takes four 8-bit
+// radix passes over every key instead.
 #include "kvev_internal.cuh"
 
 namespace kvev {
 
 namespace {
 
+constexpr int kHistBits = 12;              // first radix digit: the top 12 bits of a key
+constexpr int kHistBins = 1 << kHistBits;
+constexpr int kSelWarps = kSelectThreads / 32;
+
+static_assert(kSelWarps == 32, "find_bin scans the warp totals with one warp");
+
+struct SelShared {
+  int hist[kHistBins];
+  int wsum[kSelWarps];
+  int wcnt[2][kSelWarps];  // per warp segment: keys above T, keys equal to T
+  int bcast[2];
+  int ncand;
+};
+
+// Adds each valid lane's digit to the histogram, one shared-memory atomic per
+// distinct digit of the warp (the scores of a unit crowd into few bins).
+// Every lane of the warp must call it.
+__device__ __forceinline__ void hist_add(int* hist, bool valid, uint32_t digit) {
+  const uint32_t d = valid ? digit : 0xFFFFFFFFu;
+  const uint32_t peers = __match_any_sync(0xffffffffu, d);
+  if (valid && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
+}
+
 // Per-unit scores (or pooled scores) into order-preserving keys in shared
-// memory.  Every load of a key's window is issued before any is used, four
-// keys per thread at a time (the window reads of neighbouring keys overlap
-// and are served by L1), so the latency of the score reads is paid once per
-// group of keys rather than once per window element.
+// memory, and the histogram of their top kHistBits bits.  Every load of a
+// key's window is issued before any is used, four keys per thread at a time
+// (the window reads of neighbouring keys overlap and are served by L1), so the
+// latency of the score reads is paid once per group of keys rather than once
+// per window element.  The loop bounds are uniform over the block so that all
+// lanes reach the warp-wide match in hist_add.
 template <int P>
-__device__ __forceinline__ void build_keys_pooled(uint32_t* keys, const float* raw, int E, bool is_max) {
+__device__ __forceinline__ void build_keys_pooled(uint32_t* keys, int* hist, const float* raw, int E,
+                                                  bool is_max) {
   constexpr int h = P / 2;
   constexpr int U = 4;
-  for (int i0 = threadIdx.x; i0 < E; i0 += U * blockDim.x) {
+  for (int b0 = 0; b0 < E; b0 += U * kSelectThreads) {
     float w[U][P];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
+      const int i = b0 + u * kSelectThreads + threadIdx.x;
 #pragma unroll
       for (int j = 0; j < P; ++j) {
         const int q = i - h + j;
@@ -43,122 +75,132 @@ __device__ __forceinline__ void build_keys_pooled(uint32_t* keys, const float* r
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i >= E) break;
+      const int i = b0 + u * kSelectThreads + threadIdx.x;
       float v = w[u][0];
 #pragma unroll
       for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[u][j]) : v + w[u][j];
-      keys[i] = float_key(is_max ? v : v / static_cast<float>(P));
+      const uint32_t key = float_key(is_max ? v : v / static_cast<float>(P));
+      if (i < E) keys[i] = key;
+      hist_add(hist, i < E, key >> (32 - kHistBits));
     }
   }
 }
 
-__device__ void build_keys(uint32_t* keys, const float* raw, int E, int pool, int pool_type,
+__device__ void build_keys(uint32_t* keys, int* hist, const float* raw, int E, int pool, int pool_type,
                            bool do_pool) {
   const bool is_max = pool_type == KVEV_POOL_MAX;
   if (do_pool) {
     switch (pool) {  // common widths with fully unrolled windows
-      case 3: build_keys_pooled<3>(keys, raw, E, is_max); return;
-      case 5: build_keys_pooled<5>(keys, raw, E, is_max); return;
-      case 7: build_keys_pooled<7>(keys, raw, E, is_max); return;
-      case 9: build_keys_pooled<9>(keys, raw, E, is_max); return;
+      case 3: build_keys_pooled<3>(keys, hist, raw, E, is_max); return;
+      case 5: build_keys_pooled<5>(keys, hist, raw, E, is_max); return;
+      case 7: build_keys_pooled<7>(keys, hist, raw, E, is_max); return;
+      case 9: build_keys_pooled<9>(keys, hist, raw, E, is_max); return;
       default: break;
     }
   }
   const int h = pool / 2;
-  for (int i = threadIdx.x; i < E; i += blockDim.x) {
-    float v;
-    if (!do_pool) {
-      v = raw[i];
-    } else if (is_max) {
-      v = -INFINITY;
-      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-      for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
-    } else {
-      float sum = 0.f;
-      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-      for (int j = lo; j <= hi; ++j) sum += raw[j];
-      v = sum / static_cast<float>(pool);
+  for (int b0 = 0; b0 < E; b0 += kSelectThreads) {
+    const int i = b0 + threadIdx.x;
+    float v = 0.f;
+    if (i < E) {
+      if (!do_pool) {
+        v = raw[i];
+      } else if (is_max) {
+        v = -INFINITY;
+        const int lo = max(i - h, 0), hi = min(i + h, E - 1);
+        for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
+      } else {
+        float sum = 0.f;
+        const int lo = max(i - h, 0), hi = min(i + h, E - 1);
+        for (int j = lo; j <= hi; ++j) sum += raw[j];
+        v = sum / static_cast<float>(pool);
+      }
     }
-    keys[i] = float_key(v);
+    const uint32_t key = float_key(v);
+    if (i < E) keys[i] = key;
+    hist_add(hist, i < E, key >> (32 - kHistBits));
   }
 }
 
-struct SelShared {
-  int hist[256];
-  int wcnt[2][32];
-  int bcast[4];
-};
+// The bin of a histogram of `nbins` digits (a multiple of the block size)
+// that holds the kk-th largest key (kk >= 1), and the number of keys in
+// higher bins.  Thread t owns bins nbins-1-q*t .. nbins-q*t-q (descending).
+__device__ void find_bin(SelShared& sh, int nbins, int kk, int& digit, int& above) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int q = nbins / kSelectThreads;
+  const int top = nbins - 1 - q * threadIdx.x;
+  int s = 0;
+  for (int j = 0; j < q; ++j) s += sh.hist[top - j];
+  int incl = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) sh.wsum[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int w = sh.wsum[lane], wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += y;
+    }
+    sh.wsum[lane] = wi - w;  // exclusive prefix over warps
+  }
+  __syncthreads();
+  incl += sh.wsum[warp];
+  const int before = incl - s;
+  if (before < kk && kk <= incl) {
+    int acc = before, j = 0;
+    while (j < q - 1 && acc + sh.hist[top - j] < kk) acc += sh.hist[top - j++];
+    sh.bcast[0] = top - j;
+    sh.bcast[1] = acc;
+  }
+  __syncthreads();
+  digit = sh.bcast[0];
+  above = sh.bcast[1];
+  __syncthreads();
+}
 
-// Threshold key T (the k-th largest) and how many keys equal to T to keep.
+// Threshold key T (the k-th largest) and how many keys equal to T to keep,
+// by 8-bit radix passes over every key (the general path).
 __device__ void radix_select(const uint32_t* keys, int E, int k, SelShared& sh, uint32_t& T,
                              int& need) {
   uint32_t prefix = 0, mask = 0;
   int kk = k;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) sh.hist[i] = 0;
+    for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
     __syncthreads();
-    for (int base = 0; base < E; base += blockDim.x) {
+    for (int base = 0; base < E; base += kSelectThreads) {
       const int i = base + threadIdx.x;
       const bool in = i < E && (keys[i] & mask) == prefix;
-      const uint32_t digit = in ? (keys[i] >> shift) & 255u : 256u;
-      const uint32_t peers = __match_any_sync(0xffffffffu, digit);
-      if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[digit], __popc(peers));
+      hist_add(sh.hist, in, in ? (keys[i] >> shift) & 255u : 0u);
     }
     __syncthreads();
-    if (warp == 0) {
-      // bins in descending digit order; lane l owns digits 255-8l ... 248-8l
-      int c[8], s = 0;
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        c[q] = sh.hist[255 - 8 * lane - q];
-        s += c[q];
-      }
-      int incl = s;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      const int before = incl - s;
-      if (before < kk && kk <= incl) {
-        int acc = before, q = 0;
-        while (acc + c[q] < kk) acc += c[q++];
-        sh.bcast[0] = 255 - 8 * lane - q;  // selected digit
-        sh.bcast[1] = acc;                 // keys with a larger digit (within prefix)
-      }
-    }
-    __syncthreads();
-    const uint32_t dsel = static_cast<uint32_t>(sh.bcast[0]);
-    kk -= sh.bcast[1];
-    prefix |= dsel << shift;
+    int digit, above;  // bins 256 .. 1023 are empty: the 1024-bin search ends in 255 .. 0
+
+    find_bin(sh, 1024, kk, digit, above);
+    kk -= above;
+    prefix |= static_cast<uint32_t>(digit) << shift;
     mask |= 255u << shift;
-    __syncthreads();
   }
   T = prefix;
   need = kk;
 }
 
-// Ordered write of the selected positions of [0, E) to out[0..k).
-__device__ void compact(const uint32_t* keys, int E, int k, uint32_t T, int need, SelShared& sh,
-                        int* out) {
+// Warp segments of [0, E): contiguous, 32-aligned, in warp order, so that a
+// warp's kept positions follow those of the warps before it.
+__device__ __forceinline__ int seg_len(int E) { return (((E + kSelWarps - 1) / kSelWarps) + 31) & ~31; }
+
+// Ordered write of the kept positions of [0, E) to out[0..k): keys above T,
+// and the first `need` keys equal to T in position order.  sh.wcnt holds each
+// warp segment's counts of both.
+__device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int need, SelShared& sh,
+                           int* out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int nwarps = blockDim.x >> 5;
-  const int seg = (((E + nwarps - 1) / nwarps) + 31) & ~31;
+  const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
-  int gt = 0, eq = 0;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int i = b0 + lane;
-    const uint32_t key = i < hi ? keys[i] : 0u;
-    gt += __popc(__ballot_sync(0xffffffffu, i < hi && key > T));
-    eq += __popc(__ballot_sync(0xffffffffu, i < hi && key == T));
-  }
-  if (lane == 0) {
-    sh.wcnt[0][warp] = gt;
-    sh.wcnt[1][warp] = eq;
-  }
-  __syncthreads();
   int eq_base = 0, sel_base = 0;
   for (int w = 0; w < warp; ++w) {
     const int e = sh.wcnt[1][w];
@@ -182,6 +224,87 @@ __device__ void compact(const uint32_t* keys, int E, int k, uint32_t T, int need
     sel_base += __popc(sb);
   }
 }
+
+// Per-warp-segment counts of keys above and equal to T over all of [0, E).
+__device__ void count_segments(const uint32_t* keys, int E, uint32_t T, SelShared& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int seg = seg_len(E);
+  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
+  int gt = 0, eq = 0;
+  for (int b0 = lo; b0 < hi; b0 += 32) {
+    const int i = b0 + lane;
+    const uint32_t key = i < hi ? keys[i] : 0u;
+    gt += __popc(__ballot_sync(0xffffffffu, i < hi && key > T));
+    eq += __popc(__ballot_sync(0xffffffffu, i < hi && key == T));
+  }
+  if (lane == 0) {
+    sh.wcnt[0][warp] = gt;
+    sh.wcnt[1][warp] = eq;
+  }
+  __syncthreads();
+}
+
+// The fast path once the first digit's bin (digit d0, kk-th within it) holds
+// at most `cap` keys: one pass collects that bin's positions into cand[] and
+// counts, per warp segment, the keys of higher bins; the remaining 20 bits are
+// resolved by two 10-bit radix passes over the candidates alone; the
+// candidates then add their own above/equal counts to their segments.
+__device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, int kk, SelShared& sh,
+                                     int* cand, uint32_t& T, int& need) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int seg = seg_len(E);
+  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
+  const uint32_t lt = (1u << lane) - 1u;
+  if (threadIdx.x == 0) sh.ncand = 0;
+  __syncthreads();
+  int gt = 0;
+  for (int b0 = lo; b0 < hi; b0 += 32) {
+    const int i = b0 + lane;
+    const uint32_t d = i < hi ? keys[i] >> (32 - kHistBits) : 0u;
+    gt += __popc(__ballot_sync(0xffffffffu, i < hi && d > d0));
+    const bool in = i < hi && d == d0;
+    const uint32_t b = __ballot_sync(0xffffffffu, in);
+    if (b) {
+      int base = 0;
+      if (lane == __ffs(b) - 1) base = atomicAdd(&sh.ncand, __popc(b));
+      base = __shfl_sync(0xffffffffu, base, __ffs(b) - 1);
+      if (in) cand[base + __popc(b & lt)] = i;
+    }
+  }
+  if (lane == 0) {
+    sh.wcnt[0][warp] = gt;
+    sh.wcnt[1][warp] = 0;
+  }
+  __syncthreads();
+  const int nc = sh.ncand;
+  uint32_t prefix = d0 << (32 - kHistBits), mask = ~0u << (32 - kHistBits);
+  for (int shift = 10; shift >= 0; shift -= 10) {
+    for (int i = threadIdx.x; i < 1024; i += kSelectThreads) sh.hist[i] = 0;
+    __syncthreads();
+    for (int base = 0; base < nc; base += kSelectThreads) {
+      const int c = base + threadIdx.x;
+      const uint32_t key = c < nc ? keys[cand[c]] : 0u;
+      const bool in = c < nc && (key & mask) == prefix;
+      hist_add(sh.hist, in, (key >> shift) & 1023u);
+    }
+    __syncthreads();
+    int digit, above;
+    find_bin(sh, 1024, kk, digit, above);
+    kk -= above;
+    prefix |= static_cast<uint32_t>(digit) << shift;
+    mask |= 1023u << shift;
+  }
+  T = prefix;
+  need = kk;
+  for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
+    const int i = cand[c];
+    const uint32_t key = keys[i];
+    if (key >= T) atomicAdd(&sh.wcnt[key > T ? 0 : 1][i / seg], 1);
+  }
+  __syncthreads();
+}
+
+static_assert(sizeof(SelShared) <= kSelectStaticSmem, "select kernel's static shared memory");
 
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_constant__ SelectParams p) {
   extern __shared__ uint32_t keys[];
@@ -228,18 +351,28 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
   // protected tail [E, n) occupies slots k .. count-1
   for (int j = threadIdx.x; j < n - E; j += blockDim.x) idx[k + j] = E + j;
   if (k == 0) return;
-  const float* raw =
-      p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
-  build_keys(keys, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV);
-  __syncthreads();
   if (k >= E) {
     for (int j = threadIdx.x; j < E; j += blockDim.x) idx[j] = j;
     return;
   }
+  const float* raw =
+      p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
+  for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
+  __syncthreads();
+  build_keys(keys, sh.hist, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV);
+  __syncthreads();
+  int d0, above;
+  find_bin(sh, kHistBins, k, d0, above);
   uint32_t T;
   int need;
-  radix_select(keys, E, k, sh, T, need);
-  compact(keys, E, k, T, need, sh, idx);
+  if (sh.hist[d0] <= p.cand_cap) {
+    select_by_candidates(keys, E, static_cast<uint32_t>(d0), k - above, sh,
+                         reinterpret_cast<int*>(keys + p.S_cap), T, need);
+  } else {  // a crowded first bin (e.g. many equal scores): radix passes over every key
+    radix_select(keys, E, k, sh, T, need);
+    count_segments(keys, E, T, sh);
+  }
+  write_kept(keys, E, k, T, need, sh, idx);
 }
 
 }  // namespace

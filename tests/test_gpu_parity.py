@@ -193,6 +193,18 @@ def test_h2o_recent_override_and_ties(torch, orc):
     parity.check_workload(wl2, device_workload(wl2), wl2.lens)
 
 
+def test_select_crowded_first_bin(torch, orc):
+    # At a 40K capacity the selection's candidate buffer holds fewer positions
+    # than these units have keys.  Layer 0 has zero queries, so all of its
+    # prefix scores tie and its units take the radix passes over every key
+    # (lower positions win the ties); layer 1 keeps live queries and takes the
+    # candidate path at full length.
+    wl = _custom([gen.SNAPKV, gen.H2O], [2048, 1024], [38000, 30000], W=8, H_q=4, H_kv=2, S_cap=40000, d=64)
+    dev = device_workload(wl)
+    dev[0][2].zero_()
+    parity.check_workload(wl, dev, wl.lens)
+
+
 def test_repeat_calls_identical(torch):
     wl = gen.config_tiny(1)
     dev = host_to_dev(torch, gen.host_tensors(wl))
