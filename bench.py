@@ -75,6 +75,32 @@ def score_flops(wl) -> int:
     return tot
 
 
+def h2o_full_flops(wl) -> tuple[int, int]:
+    """(algorithmic, performed) tensor-core flops of the scoring launches when
+    H2O layers score every prompt row.  Algorithmic: each causal q.k product
+    once (2 G d n(n+1)/2 per H2O unit, 2 G W n d per SnapKV unit).  Performed:
+    the row pass (each block of Pb = 256 // G positions against the 256-key
+    super-tiles up to its end) and the key pass (each 256-key super-tile
+    against the blocks from the one holding its first key), 256 rows x 256
+    keys x d per pair."""
+    alg = perf = 0
+    pb = max(1, 256 // wl.G)
+    for l in range(wl.L):
+        m, b = int(wl.route[l]), int(wl.budget[l])
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            if m == gen.H2O and n > 0:
+                alg += wl.G * wl.d * n * (n + 1) * wl.H_kv
+                nb = (n + pb - 1) // pb
+                pairs = sum((min(n, (q + 1) * pb) + 255) // 256 for q in range(nb))
+                pairs += sum(nb - (256 * t) // pb for t in range((n + 255) // 256))
+                perf += pairs * 2 * 256 * 256 * wl.d * wl.H_kv
+            elif m == gen.SNAPKV and n > b:
+                alg += 2 * wl.G * wl.W * n * wl.d * wl.H_kv
+                perf += 2 * (2 * wl.G * wl.W * n * wl.d) * wl.H_kv
+    return alg, perf
+
+
 def workload_bytes(wl):
     tot = sc = ev = 0
     for l in range(wl.L):
@@ -274,11 +300,23 @@ def run_ours(args, rank, world, local_rank):
     need_q = lambda l: wl.route[l] in (gen.SNAPKV, gen.H2O)
     dev = {l: gen.device_layer(wl, l, need_q=need_q(l)) for l in range(wl.L)}
     plan = kvev.Plan.from_workload(wl)
+    if args.h2o_full_prompt:
+        plan.set_h2o_full_prompt(True)  # before sizing the workspace: it holds every row's lse
     bufs = plan.buffers(wl.B, wl.S_cap)
     lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
     K = [dev[l][0] for l in range(wl.L)]
     V = [dev[l][1] for l in range(wl.L)]
     Q = [dev[l][2] for l in range(wl.L)]
+    if args.h2o_full_prompt:
+        # H2O layers score every prompt row: their queries are the whole
+        # prompt's, seeded normal bf16 [B][H_q][S_cap][d]
+        g = torch.Generator(device="cuda")
+        g.manual_seed(4242 + rank)
+        for l in range(wl.L):
+            if wl.route[l] == gen.H2O:
+                Q[l] = torch.randn((wl.B, wl.H_q, wl.S_cap, wl.d), generator=g, device="cuda",
+                                   dtype=torch.float32).to(torch.bfloat16)
+        args.no_e2e = args.no_cpu_baseline = True
     stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
 
@@ -369,7 +407,30 @@ def run_ours(args, rank, world, local_rank):
                "sample": f"{len(units)} (sequence, layer, KV-head) units of the workload, "
                          f"route mix kept, {secs:.1f} s of oracle time"}
 
-    if rank == 0:
+    if rank == 0 and args.h2o_full_prompt:
+        alg, perf = h2o_full_flops(wl)
+        tc_ach = alg / (score_ms / 1e3) / 1e12
+        out = {
+            "metric": "H2O full-prompt prefill eviction: causal attention TFLOP/s of the step",
+            "value": sum_over_ranks(alg) / (ms_step / 1e3) / 1e12, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; full-prompt queries drawn N(0,1) on the device)",
+            "config": workload_config(wl, {"h2o_full_prompt": True, "query_block": max(1, 256 // wl.G)}),
+            "kernel_ms": kernel_ms,
+            "roofline": {"kernel": "h2o_full_kernel row + key passes (and the window kernel)", "bound": "tensor",
+                         "achieved": tc_ach, "peak": tc_peak, "unit": "TFLOP/s", "frac": tc_ach / tc_peak,
+                         "traffic": None, "peak_source": "measured" if "bf16_tflops" in peaks else "fallback",
+                         "tensor_pipe": {"achieved": perf / (score_ms / 1e3) / 1e12, "peak": tc_peak,
+                                         "unit": "TFLOP/s",
+                                         "frac": perf / (score_ms / 1e3) / 1e12 / tc_peak,
+                                         "work": "row pass + key pass, 256 x 256 tiles"}},
+            "clocks": clocks,
+            "gpu_launches": args.steps * 6,  # prologue, window scores, row pass, key pass, select, gather
+            "e2e": None, "cpu_baseline": None,
+        }
+        print(json.dumps(out), flush=True)
+    elif rank == 0:
         out = {
             "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
@@ -603,6 +664,8 @@ def main():
     ap.add_argument("--batch", type=int, default=None,
                     help="use only the first B sequences of the 'long' workload, or B sequences "
                          "in the decode workload (profiling)")
+    ap.add_argument("--h2o-full-prompt", action="store_true",
+                    help="H2O layers score every prompt query row (reports causal-attention TFLOP/s)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

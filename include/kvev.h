@@ -246,14 +246,17 @@ KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const voi
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
                        float *h2o_state, void *workspace, size_t workspace_bytes, void *stream);
 
-/* Sec. 2.1 (H2O's original scoring): with on = 1, the prefill
- * scores of the plan's H2O layers accumulate the attention of every prompt
- * query row, raw[k] = (1/G) sum_g sum_{t=k}^{n-1} p_{g,t}(k), instead of the
+/* Sec. 2.1 (H2O's original scoring): with on = 1, the prefill scores of the
+ * plan's H2O layers accumulate the attention of every prompt query row,
+ *   raw[k] = (1/G) sum_g sum_{t=k}^{n-1} p_{g,t}(k),
+ * p_{g,t} being query row (g, t)'s softmax over keys 0..t, instead of the
  * observation window's.  Q_win[l] of an H2O layer is then the whole prompt's
  * queries, bf16 [B][H_q][S_cap][d]; SnapKV layers keep their window queries.
- * The scores are computed in row blocks of W positions (one score launch per
- * block, S_cap / W launches) and summed in the score array.  Cost grows with
- * n^2.  EINVAL: NULL plan or on not 0/1. */
+ * Two extra launches compute it: a row pass (every row's log-sum-exp, kept in
+ * the workspace) and a key pass (each key's sum over the rows that see it,
+ * written once per key).  Cost grows with n^2.  Set it before
+ * kvev_plan_query(): the workspace then also holds G * S_cap floats per H2O
+ * (sequence, KV head).  EINVAL: NULL plan or on not 0/1. */
 KVEV_API int kvev_plan_set_h2o_full_prompt(kvev_plan *plan, int on);
 
 /* Synchronise the plan's last stream and read-and-clear the device status

@@ -25,7 +25,7 @@ FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", 
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]
 
 LIBS = {
-    "libkvev.so": ["api.cu", "score.cu", "select.cu", "gather.cu", "decode.cu", "planner.cu"],
+    "libkvev.so": ["api.cu", "score.cu", "h2o_full.cu", "select.cu", "gather.cu", "decode.cu", "planner.cu"],
     "libkvev_synth.so": ["synth.cu"],
 }
 

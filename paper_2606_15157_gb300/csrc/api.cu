@@ -25,7 +25,7 @@ struct DevCtx {
   int device = -1;
   int num_sms = 0;
   int smem_optin = 0;
-  size_t score_smem_set = 0, select_smem_set = 0;
+  size_t score_smem_set = 0, select_smem_set = 0, h2o_full_smem_set = 0;
   int* status = nullptr;
 };
 
@@ -58,9 +58,9 @@ constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 
 struct WsLayout {
-  int n_units = 0, R = 0, R_pad = 0, max_items = 0;
+  int n_units = 0, R = 0, R_pad = 0, max_items = 0, n_h2o_units = 0;
   size_t lens = 0, abort_flag = 0, node_cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
-         lam = 0, raw = 0, total = 0;
+         lam = 0, raw = 0, lse = 0, total = 0;
 };
 
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
@@ -85,9 +85,17 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.part = take(sizeof(float2) * static_cast<size_t>(w.max_items) * w.R_pad);  // one per chunk
   w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
   w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
+  if (p.h2o_full) {  // base-2 log-sum-exp of every prompt row of every H2O unit
+    for (int l : p.score_layers) w.n_h2o_units += p.route_pre[l] == KVEV_H2O ? B * p.H_kv : 0;
+    w.lse = take(sizeof(float) * static_cast<size_t>(w.n_h2o_units) * p.G * S_cap);
+  }
   w.total = off;
   return w;
 }
+
+// Prompt positions per query block of the whole-prompt H2O kernels: as many
+// as keep the block's G * Pb rows within two 128-lane row groups.
+int prompt_block(int G) { return std::max(1, 256 / G); }
 
 int64_t rows_per_layer(const kvev_plan& p, int B, int l) {
   return static_cast<int64_t>(B) * p.H_kv * p.slots[l];
@@ -149,7 +157,7 @@ int query_device(DevCtx& c, int dev) {
     return KVEV_ECUDA;
   if (major < 10) return KVEV_ENOTSUP;
   c.device = dev;
-  c.score_smem_set = c.select_smem_set = 0;
+  c.score_smem_set = c.select_smem_set = c.h2o_full_smem_set = 0;
   return KVEV_OK;
 }
 
@@ -578,6 +586,18 @@ int score_regs_ok(int d) {
   return ok[i];
 }
 
+// The same check for the whole-prompt H2O kernel (same warp roles and split).
+int h2o_full_regs_ok(int d) {
+  static std::once_flag once[2];
+  static int ok[2] = {-1, -1};
+  const int i = d == 64 ? 0 : 1;
+  std::call_once(once[i], [&] {
+    const int regs = h2o_full_kernel_regs(d);
+    ok[i] = regs < 0 ? -1 : (regs * kScoreThreads >= kRegsNeeded ? 1 : 0);
+  });
+  return ok[i];
+}
+
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
                const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
                void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
@@ -632,9 +652,9 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   pp.W = P.W;
   bool any_h2o = false;
   for (int i = 0; i < n_slayers; ++i) any_h2o |= P.route_pre[P.score_layers[i]] == KVEV_H2O;
-  // H2O prefill scores over every prompt query row: scored by row blocks of W
-  // positions (blocks of one launch each), accumulated in the score array
-  const bool blocks = P.h2o_full && any_h2o;
+  // H2O prefill scores over every prompt query row: the window kernel scores
+  // the SnapKV layers only, and the whole-prompt kernels the H2O layers
+  const bool full_prompt = P.h2o_full && any_h2o;
 
   // ---- window scores ----------------------------------------------------
   ScoreParams sp;
@@ -647,9 +667,9 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
       const int l = P.score_layers[i];
       if (!encode_map(&sp.kmap[i], K[l], P.d, static_cast<uint64_t>(B) * P.H_kv * S_cap,
                       kSuperKeys) ||
-          !(blocks && P.route_pre[l] == KVEV_H2O
+          !(full_prompt && P.route_pre[l] == KVEV_H2O
                 ? encode_map_prompt(&sp.qmap[i], Q_win[l], P.d, S_cap, static_cast<uint64_t>(B) * P.H_q,
-                                    P.W, P.G)
+                                    prompt_block(P.G), P.G)
                 : encode_map(&sp.qmap[i], Q_win[l], P.d, static_cast<uint64_t>(B) * P.H_q * P.W,
                              ws.R_pad)))
         return KVEV_ECUDA;
@@ -712,51 +732,46 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     score_grid = grid;
     score_smem = smem;
   }
-  // one prologue + score pass; the first prologue also validates the lengths
-  auto pass = [&](int mode, int win0) -> int {
-    pp.mode = mode;
-    pp.win0 = win0;
-    if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
-    if (ws.n_units == 0) return KVEV_OK;
-    sp.row_min = mode == kScoreH2OBlock ? win0 : 0;
-    sp.q_full = mode == kScoreH2OBlock;
-    sp.accumulate = mode == kScoreH2OBlock;
-    return launch_score(sp, P.d, score_grid, score_smem, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
-  };
-  if (!blocks) {
-    mark(KVEV_K_PROLOGUE, 0);
-    pp.mode = kScoreAll;
-    pp.win0 = 0;
-    if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
-    mark(KVEV_K_PROLOGUE, 1);
-    if (ws.n_units > 0) {
-      mark(KVEV_K_SCORE, 0);
-      sp.row_min = 0;
-      sp.q_full = 0;
-      sp.accumulate = 0;
-      if (launch_score(sp, P.d, score_grid, score_smem, s) != cudaSuccess) return KVEV_ECUDA;
-      mark(KVEV_K_SCORE, 1);
-    }
-  } else {
-    // H2O score arrays start from zero; each block adds its rows' attention
-    const size_t per_slot = static_cast<size_t>(B) * P.H_kv * S_cap;
-    float* raw = reinterpret_cast<float*>(wsb + ws.raw);
+  mark(KVEV_K_PROLOGUE, 0);
+  pp.mode = full_prompt ? kScoreNoH2O : kScoreAll;
+  if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+  mark(KVEV_K_PROLOGUE, 1);
+  if (ws.n_units > 0) mark(KVEV_K_SCORE, 0);
+  if (ws.n_units > 0 &&
+      launch_score(sp, P.d, score_grid, score_smem, s) != cudaSuccess)
+    return KVEV_ECUDA;
+  if (full_prompt) {
+    // row pass (lse2 of every prompt row), then key pass (the scores)
+    ScoreParams fp = sp;
+    fp.Pb = prompt_block(P.G);
+    fp.R = P.G * fp.Pb;
+    fp.R_pad = (fp.R + 31) / 32 * 32;
+    fp.n_h2o = 0;
     for (int i = 0; i < n_slayers; ++i)
-      if (P.route_pre[P.score_layers[i]] == KVEV_H2O &&
-          cudaMemsetAsync(raw + static_cast<size_t>(i) * per_slot, 0, per_slot * sizeof(float), s) !=
-              cudaSuccess)
-        return KVEV_ECUDA;
-    mark(KVEV_K_PROLOGUE, 0);
-    mark(KVEV_K_PROLOGUE, 1);
-    mark(KVEV_K_SCORE, 0);
-    for (int win0 = 0; win0 < S_cap; win0 += P.W) {
-      const int rc = pass(kScoreH2OBlock, win0);
-      if (rc != KVEV_OK) return rc;
+      if (P.route_pre[P.score_layers[i]] == KVEV_H2O) fp.h2o_slot[fp.n_h2o++] = i;
+    fp.nb_max = (S_cap + fp.Pb - 1) / fp.Pb;
+    fp.nkt_max = (S_cap + kSuperKeys - 1) / kSuperKeys;
+    fp.lse = reinterpret_cast<float*>(wsb + ws.lse);
+    const int64_t units = static_cast<int64_t>(fp.n_h2o) * B * P.H_kv;
+    if (units * std::max(fp.nb_max, fp.nkt_max) > (1LL << 31) - 1) return KVEV_ENOTSUP;
+    if (h2o_full_regs_ok(P.d) != 1) return KVEV_ENOTSUP;
+    // more than half of the SM's shared memory: one CTA per SM, so its TMEM
+    // allocation never waits on another CTA
+    const size_t fsmem = std::max<size_t>(static_cast<size_t>(h2o_full_smem_bytes(P.d)),
+                                          static_cast<size_t>(D.smem_optin) / 2 + 1024);
+    if (fsmem + 1024 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
+    if (D.h2o_full_smem_set != fsmem) {
+      if (h2o_full_set_smem(P.d, fsmem) != cudaSuccess) return KVEV_ECUDA;
+      D.h2o_full_smem_set = fsmem;
     }
-    const int rc = pass(kScoreNoH2O, 0);  // SnapKV layers, and the lengths the selection reads
-    if (rc != KVEV_OK) return rc;
-    mark(KVEV_K_SCORE, 1);
+    for (int phase = 0; phase < 2; ++phase) {
+      fp.phase = phase;
+      fp.n_items = static_cast<int>(units * (phase == 0 ? fp.nb_max : fp.nkt_max));
+      if (launch_h2o_full(fp, P.d, std::min(D.num_sms, fp.n_items), fsmem, s) != cudaSuccess)
+        return KVEV_ECUDA;
+    }
   }
+  if (ws.n_units > 0) mark(KVEV_K_SCORE, 1);
 
   // ---- selection --------------------------------------------------------
   SelectParams sel;

@@ -25,8 +25,7 @@ constexpr int kMinChunkTiles = 16;
 // normaliser is ready a few load round trips after the unit's last chunk.
 // What a prologue + score launch covers (PrologueParams::mode).
 constexpr int kScoreAll = 0;       // every scoring layer, rows = the observation window
-constexpr int kScoreNoH2O = 1;     // SnapKV layers only (H2O layers are scored by row blocks)
-constexpr int kScoreH2OBlock = 2;  // H2O layers, rows = one block of W prompt positions
+constexpr int kScoreNoH2O = 1;     // SnapKV layers only (H2O layers are scored over the whole prompt)
 constexpr int kTreeFanIn = 4;
 constexpr int kTreeLevels = 5;        // internal levels: up to 4^5 = 1024 chunks per unit
 constexpr int kSoftmaxWGs = 4;        // softmax warpgroups of the score kernel
@@ -71,9 +70,8 @@ struct PrologueParams {
   int* status;
   int* node_cnt;      // [items][kTreeLevels] arrival counters of the merge tree (zeroed here)
   int n_node_cnt;     // counters in node_cnt (workspace capacity)
-  int W;              // observation window (the row block of kScoreH2OBlock)
-  int mode;           // kScoreAll, kScoreNoH2O, or kScoreH2OBlock (H2O rows [win0, win0 + W))
-  int win0;           // first query position of the row block (kScoreH2OBlock)
+  int W;              // observation window
+  int mode;           // kScoreAll, or kScoreNoH2O (H2O layers are scored over the whole prompt)
   int* ready;
   int* abort_flag;
   int* chunk_start;   // [n_units + 1]
@@ -86,10 +84,6 @@ struct ScoreParams {
   int n_units, B, H_kv, H_q, G, W, R, R_pad, S_cap;
   int chunk_keys;     // keys per work item (multiple of 128)
   int q_rows;         // rows of a Q shared-memory buffer (128 or 256)
-  int row_min;        // window rows at positions below this do not exist (a partial row block)
-  int q_full;         // Q maps cover the whole prompt, bf16 [B*H_q][S_cap][d] (3-D, one box of
-                      // G heads x W positions ending at the unit's length)
-  int accumulate;     // add the scores to raw instead of storing them (row blocks of a prompt)
   int q_bufs;         // Q buffers (2: the next entry's Q loads during this entry; 1: it
                       // loads once this entry is done, leaving room for more K stages)
   int stages;         // K tile ring depth
@@ -108,6 +102,15 @@ struct ScoreParams {
   float* raw;         // [n_units][S_cap] window scores
   long long wait_ns;
   int stall_unit;
+  // ---- whole-prompt H2O scoring (h2o_full.cu) ----
+  int phase;          // 0: row pass (lse2 of every prompt row), 1: key pass (scores)
+  int Pb;             // prompt positions per query block (G * Pb <= 256 rows)
+  int n_h2o;          // H2O scoring layers
+  int h2o_slot[kMaxScoreLayers];  // their scoring-layer indices
+  int nb_max;         // query blocks of a full-capacity unit: ceil(S_cap / Pb)
+  int nkt_max;        // 256-key super-tiles of a full-capacity unit
+  int n_items;        // items of the pass: (nb_max or nkt_max) x H2O units
+  float* lse;         // [H2O unit][G][S_cap] base-2 log-sum-exp of every prompt row
 };
 
 struct SelectParams {
@@ -559,6 +562,10 @@ cudaError_t launch_decode_init(const DecodeParams& p, cudaStream_t s);
 cudaError_t launch_decode_step(const DecodeParams& p, size_t smem, cudaStream_t s);
 int score_kernel_regs(int d);
 cudaError_t score_set_smem(int d, size_t smem);
+int h2o_full_smem_bytes(int d);
+int h2o_full_kernel_regs(int d);
+cudaError_t h2o_full_set_smem(int d, size_t smem);
+cudaError_t launch_h2o_full(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s);
 cudaError_t select_set_smem(size_t smem);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s, int num_sms);

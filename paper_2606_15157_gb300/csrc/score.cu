@@ -33,7 +33,7 @@
 // the tensor core keeps filling the other slots meanwhile.  The softmax
 // warpgroups never wait on each other.  setmaxnreg moves registers from
 // warpgroup 0 to the softmax warpgroups.
-#include "kvev_internal.cuh"
+#include "score_common.cuh"
 
 namespace kvev {
 
@@ -165,54 +165,12 @@ struct EntryIter {
   }
 };
 
-// Bounded wait on an mbarrier phase; false if it ran out or another role
-// aborted.  Each try sleeps in hardware for up to kWaitSliceNs, so the abort
-// flag and the time limit are checked at least that often.
-constexpr uint32_t kWaitSliceNs = 20000;
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, const ScoreParams& p) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait_sleep(bar, parity, kWaitSliceNs)) {
-    if (ld_volatile(p.abort_flag)) return false;
-    if (globaltimer_ns() - t0 > static_cast<uint64_t>(p.wait_ns)) {
-      atomicExch(p.abort_flag, 1);
-      atomicOr(p.status, kStatusTimeout);
-      return false;
-    }
-  }
-  return true;
-}
-
-// wait_bar by every lane of a warp; the warp agrees on the outcome (all lanes
-// see the same phase eventually, but a time-out may hit only some of them).
-__device__ __forceinline__ bool wait_bar_warp(uint64_t* bar, uint32_t parity, const ScoreParams& p) {
-  return __all_sync(0xffffffffu, wait_bar(bar, parity, p));
-}
-
-// Bounded wait used while shutting down: ignores the abort flag, gives up after
-// `ns` nanoseconds (asynchronous copies and MMAs finish on their own).
-__device__ __forceinline__ void wait_bar_drain(uint64_t* bar, uint32_t parity, uint64_t ns) {
-  const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait_sleep(bar, parity, kWaitSliceNs))
-    if (globaltimer_ns() - t0 > ns) return;
-}
-
 // ---------------------------------------------------------------------------
 // Producer: TMA loads of Q (once per item) and of K tiles (twice per item).
 // ---------------------------------------------------------------------------
 template <int D>
 __device__ __forceinline__ void load_q(const ScoreParams& p, const Smem& sm, uint32_t e, const ItemInfo& it) {
   const uint32_t qb = e % p.q_bufs;
-  if (p.q_full) {
-    // G heads x the last W positions of the (truncated) prompt, one 3-D box per
-    // 64-column block; it lands as the same G*W rows of 128 bytes
-    mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R) * D * 2);
-#pragma unroll
-    for (int kc = 0; kc < D / 64; ++kc)
-      tma_load_3d(sm.qbuf + qb * sm.qbytes + static_cast<size_t>(kc) * p.q_rows * 128, &p.qmap[it.ls],
-                  kc * 64, it.n - p.W, it.s * p.H_q + it.h * p.G, &sm.qfull[qb]);
-    return;
-  }
   mbar_expect_tx(&sm.qfull[qb], static_cast<uint32_t>(p.R_pad) * D * 2);
   const int qrow = (it.s * p.H_q + it.h * p.G) * p.W;
 #pragma unroll
@@ -372,74 +330,6 @@ __device__ __forceinline__ int row_pos(const ScoreParams& p, int r, int n) {
   return n - p.W + (r % p.W);
 }
 
-// Position of row r if the row exists, else -1: rows before the sequence
-// start, and rows of a partial row block that belong to the previous block.
-__device__ __forceinline__ int row_live(const ScoreParams& p, int r, int n) {
-  const int t = row_pos(p, r, n);
-  return t >= p.row_min ? t : -1;
-}
-
-__device__ __forceinline__ float max32(const float (&v)[32]) {
-  float t[11];
-#pragma unroll
-  for (int j = 0; j < 10; ++j) t[j] = fmax3(v[3 * j], v[3 * j + 1], v[3 * j + 2]);
-  t[10] = fmaxf(v[30], v[31]);
-  const float a = fmax3(t[0], t[1], t[2]), b = fmax3(t[3], t[4], t[5]);
-  const float c = fmax3(t[6], t[7], t[8]), e = fmax3(t[9], t[10], a);
-  return fmax3(b, c, e);
-}
-
-__device__ __forceinline__ float sum4x2(const float2 (&a)[4]) {
-  const float2 s = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
-  return s.x + s.y;
-}
-
-// Keys of a 32-key chunk that row position tr cannot see are set to -inf.
-__device__ __forceinline__ void mask_chunk(float (&v)[32], int k0, int tr) {
-#pragma unroll
-  for (int i = 0; i < 32; ++i)
-    if (k0 + i > tr) v[i] = -INFINITY;
-}
-
-// One sweep-1 unit for one row: online base-2 (max, sum) update over the
-// thread's 64 keys (two 32-key halves), with one rescale of the running sum.
-__device__ __forceinline__ void s1_chunk64(const float (&v0)[32], const float (&v1)[32], float c, float& m,
-                                           float& z) {
-  const float mnew = fmaxf(m, fmaxf(max32(v0), max32(v1)) * c);
-  const float base = mnew == -INFINITY ? 0.f : mnew;
-  const float zs = z * ex2_approx(m - base);  // m = -inf -> 0
-  const float2 cc = make_float2(c, c), nb = make_float2(-base, -base);
-  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                 make_float2(0.f, 0.f)};
-#pragma unroll
-  for (int i = 0; i < 32; i += 2) {
-    const float2 t0 = ffma2(make_float2(v0[i], v0[i + 1]), cc, nb);
-    const float2 t1 = ffma2(make_float2(v1[i], v1[i + 1]), cc, nb);
-    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
-    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
-  }
-  z = zs + sum4x2(a);
-  m = mnew;
-}
-
-// One 32-row chunk of sweep 2 for this thread's key: sum of exp2(s*c - lse2_r)
-// into four packed accumulators; nl = -lse2 of the chunk's rows (shared memory).
-// Every row of the chunk counts for this key: no per-element checks.
-__device__ __forceinline__ void s2_chunk_full(const uint32_t (&rr)[32], float c, const float* nl,
-                                              float2 (&a)[4]) {
-  const float2 cc = make_float2(c, c);
-#pragma unroll
-  for (int i = 0; i < 32; i += 4) {
-    const float4 l4 = lds4(nl + i);
-    const float2 t0 = ffma2(make_float2(__uint_as_float(rr[i]), __uint_as_float(rr[i + 1])), cc,
-                            make_float2(l4.x, l4.y));
-    const float2 t1 = ffma2(make_float2(__uint_as_float(rr[i + 2]), __uint_as_float(rr[i + 3])),
-                            cc, make_float2(l4.z, l4.w));
-    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
-    a[((i >> 1) + 1) & 3] =
-        fadd2(a[((i >> 1) + 1) & 3], make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
-  }
-}
 
 __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&rr)[32], bool full,
                                          const float* nl, int r0, int k, int n, float2 (&a)[4]) {
@@ -450,7 +340,7 @@ __device__ __forceinline__ void s2_chunk(const ScoreParams& p, const uint32_t (&
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       const int r = r0 + i;
-      if (r < p.R && k <= row_live(p, r, n)) {
+      if (r < p.R && k <= row_pos(p, r, n)) {
         const float e = ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
         if (i & 1) a[(i >> 1) & 3].y += e; else a[(i >> 1) & 3].x += e;
       }
@@ -512,10 +402,8 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       const int t = first + jj * stride;
       const ItemInfo it = decode_item(p, t, load_item(p, t));
       float m0 = -INFINITY, z0 = 0.f, m1 = -INFINITY, z1 = 0.f;
-      const int tr0 = lrow < p.R ? row_live(p, lrow, it.n) : -1;
-      const int tr1 = 128 + lrow < p.R ? row_live(p, 128 + lrow, it.n) : -1;
-      // every row of the window exists (no row before the sequence or the block)
-      const bool rows_all = it.n - p.W >= p.row_min;
+      const int tr0 = lrow < p.R ? row_pos(p, lrow, it.n) : -1;
+      const int tr1 = 128 + lrow < p.R ? row_pos(p, 128 + lrow, it.n) : -1;
       // One unit per (256-key super-tile, 128-row group): this warpgroup's 32
       // keys of each 128-key half, for the thread's row of the group.  Rows
       // that do not exist (tr < 0) are computed like the others and dropped
@@ -524,7 +412,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int j = 0; j < nst; ++j) {
         const int kb = it.key0 + j * kSuperKeys;
         const int k0 = kb + 64 * wg;                       // keys k0 .. k0 + 63
-        const bool full = rows_all && kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
+        const bool full = kb + kSuperKeys - 1 <= it.n - p.W;  // every key visible to every row
         for (int h = 0; h < nh; ++h) {
           ok = slot_wait(p, sm, g, ok);
           uint32_t r0[32], r1[32];
@@ -569,7 +457,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
       for (int i = 0; i < it.ntiles; ++i) {
         const int kb = it.key0 + i * kTileKeys;
         const int k = kb + lrow;
-        const bool key_full = it.n - p.W >= p.row_min && kb + kTileKeys - 1 <= it.n - p.W;
+        const bool key_full = kb + kTileKeys - 1 <= it.n - p.W;
         float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
         ok = slot_wait(p, sm, g, ok);
@@ -600,12 +488,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
             float sum = 0.f;
 #pragma unroll
             for (int w = 0; w < kSoftmaxWGs; ++w) sum += sm.red[w * kRedTiles * 128 + q];
-            if (ok && key0 + q < it.n) {
-              if (p.accumulate)
-                out[key0 + q] += sum * p.inv_G;
-              else
-                out[key0 + q] = sum * p.inv_G;
-            }
+            if (ok && key0 + q < it.n) out[key0 + q] = sum * p.inv_G;
           }
           // the batch's rows may be overwritten, and after the entry's last
           // batch every warpgroup is done reading lam
@@ -626,13 +509,6 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
 // into its own and carries the result one level up.  Whoever completes the
 // root turns it into the unit's lse2 and releases it.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ float2 merge_ms(float2 a, float2 e) {  // (max, sum) in base 2
-  if (e.x == -INFINITY) return a;
-  if (a.x == -INFINITY) return e;
-  const float m = fmaxf(a.x, e.x);
-  return make_float2(m, a.y * ex2_approx(a.x - m) + e.y * ex2_approx(e.x - m));
-}
-
 __device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   constexpr int kRowsPerLane = 8;  // R_pad <= 256
   const int lane = threadIdx.x & 31;
@@ -830,7 +706,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
 __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ PrologueParams p) {
   __shared__ int warp_sums[32];
   __shared__ int carry;
-  __shared__ int unit_len[1024];  // length each unit is scored over
   const int tid = threadIdx.x;
   if (tid == 0) {
     carry = 0;
@@ -853,17 +728,11 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     if (u < p.n_units) {
       const int ls = u / per_layer;
       const int s = (u - ls * per_layer) / p.H_kv;
-      int n = p.lens[s];
+      const int n = p.lens[s];
       const bool h2o = p.slayer_method[ls] == KVEV_H2O;
-      bool need = n > 0 && (h2o || n > p.slayer_budget[ls]);
-      if (p.mode == kScoreNoH2O && h2o) need = false;
-      if (p.mode == kScoreH2OBlock) {
-        // the prompt truncated after the block: its last W positions are the rows
-        n = min(n, p.win0 + p.W);
-        need = h2o && n > p.win0;
-      }
+      // H2O layers scored over the whole prompt have their own kernels
+      const bool need = n > 0 && (h2o ? p.mode != kScoreNoH2O : n > p.slayer_budget[ls]);
       c = need ? (n + p.chunk_keys - 1) / p.chunk_keys : 0;
-      unit_len[tid] = n;
       p.ready[u] = 0;
     }
     // block-wide exclusive scan of c
@@ -889,7 +758,7 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     const int excl = carry + (w > 0 ? warp_sums[w - 1] : 0) + x - c;
     if (u < p.n_units) {
       p.chunk_start[u] = excl;
-      const int n = unit_len[tid];
+      const int n = p.lens[(u % per_layer) / p.H_kv];
       for (int q = 0; q < c; ++q) {
         const int key0 = q * p.chunk_keys;
         const int nk = min(p.chunk_keys, n - key0);

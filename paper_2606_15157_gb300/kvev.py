@@ -341,6 +341,12 @@ class Plan:
         if h2o_full_prompt:
             _check(load().kvev_plan_set_h2o_full_prompt(self.handle, 1), "kvev_plan_set_h2o_full_prompt")
 
+    def set_h2o_full_prompt(self, on: bool = True):
+        """H2O layers score every prompt query row (their Q_win is then the
+        whole prompt's queries, [B][H_q][S_cap][d])."""
+        _check(load().kvev_plan_set_h2o_full_prompt(self.handle, 1 if on else 0),
+               "kvev_plan_set_h2o_full_prompt")
+
     @classmethod
     def from_workload(cls, wl):
         return cls(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel,

@@ -1,8 +1,9 @@
 """GPU parity of H2O prefill scoring over every prompt query row (H2O's
-original accumulated attention, Sec. 2.1): the library computes it in row
-blocks of W positions and sums them; the oracle evaluates the definition with
-the whole prompt as the window.  SnapKV layers of the same plan keep their
-observation-window scores, identical to a plan without the option."""
+original accumulated attention, Sec. 2.1): the library computes each row's
+normaliser in a row pass and the key sums in a key pass; the oracle evaluates
+the definition with the whole prompt as the window.  SnapKV layers of the same
+plan keep their observation-window scores, identical to a plan without the
+option."""
 import numpy as np
 import pytest
 
@@ -29,12 +30,22 @@ def _bf16_bits(rng, shape, scale=1.0):
     return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)  # round to nearest even
 
 
-@pytest.mark.parametrize("lens", [(700, 1000), (16, 1)])
-def test_h2o_full_prompt_scores_and_selection(torch, lens):
+# (H_q, H_kv, d, lens): G = 4 fills 256-row blocks of 64 positions; G = 3
+# leaves a 255-row block of 85 positions; G = 8 gives blocks of 32 positions.
+GEOMETRIES = [
+    (8, 2, 128, (700, 1000)),
+    (8, 2, 128, (16, 1)),
+    (12, 4, 64, (300, 0, 517)),
+    (16, 2, 64, (450, 129)),
+]
+
+
+@pytest.mark.parametrize("H_q,H_kv,d,lens", GEOMETRIES)
+def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens):
     from paper_2606_15157_gb300 import kvev
     import oracle
     route = [gen.H2O, gen.SNAPKV, gen.H2O]
-    wl = gen.Workload(name="h2o_full", L=3, H_q=8, H_kv=2, d=128, B=len(lens), lens=np.asarray(lens, np.int32),
+    wl = gen.Workload(name="h2o_full", L=3, H_q=H_q, H_kv=H_kv, d=d, B=len(lens), lens=np.asarray(lens, np.int32),
                       S_cap=1024, W=16, pool_kernel=5, pool_type=gen.POOL_MAX,
                       route=np.asarray(route, np.int32), budget=np.asarray([256, 200, 96], np.int32),
                       sink=4, seed=11, sink_tokens=4, h2o_recent=-1)
@@ -93,6 +104,8 @@ def test_h2o_full_prompt_scores_and_selection(torch, lens):
     torch.cuda.synchronize()
     for s in range(wl.B):
         n = int(lens[s])
+        if n <= wl.budget[1]:  # kept whole: the layer scores nothing for this sequence
+            continue
         a = plan.scores(bufs, wl.B, wl.S_cap, 1)[s, :, :n]
         b = ref.scores(rbufs, wl.B, wl.S_cap, 1)[s, :, :n]
         assert torch.equal(a, b)
