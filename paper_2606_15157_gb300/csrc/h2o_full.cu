@@ -273,18 +273,32 @@ __device__ __forceinline__ void f_lam(const ScoreParams& p, const FSmem& sm) {
     const int qb0 = (f.blk * kSuperKeys) / p.Pb;
     const int ns = n_stream(p, f);
     const float* lse = p.lse + static_cast<size_t>(f.hu) * p.G * p.S_cap;
+    // lane's eight rows of a block: position (or -1) and lse2, all loads in
+    // flight at once; block j + 1's loads go out before the wait for its buffer
+    float v[8];
+    int tt[8];
+    auto fetch = [&](int j) {
+      const int q0 = (qb0 + j) * p.Pb;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int r = lane + 32 * q;
+        tt[q] = block_row_pos(p, r, q0, f.n);
+        v[q] = tt[q] >= 0 ? __ldcg(&lse[static_cast<size_t>(r / p.Pb) * p.S_cap + tt[q]]) : INFINITY;
+      }
+    };
+    fetch(0);
     for (int j = 0; j < ns; ++j) {
       const uint32_t lb = lq & 1;
       if (!wait_bar_warp(&sm.lempty[lb], ((lq >> 1) & 1) ^ 1, p)) return;
-      const int q0 = (qb0 + j) * p.Pb;
-      for (int r = lane; r < 256; r += 32) {
-        const int t = block_row_pos(p, r, q0, f.n);
-        sm.lam[lb * 256 + r] = t >= 0 ? -__ldcg(&lse[static_cast<size_t>(r / p.Pb) * p.S_cap + t]) : -INFINITY;
-        sm.tpos[lb * 256 + r] = t;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        sm.lam[lb * 256 + lane + 32 * q] = -v[q];
+        sm.tpos[lb * 256 + lane + 32 * q] = tt[q];
       }
       __syncwarp();
       mbar_arrive_elect(&sm.lfull[lb]);
       ++lq;
+      if (j + 1 < ns) fetch(j + 1);
     }
   }
 }
@@ -304,13 +318,19 @@ __device__ __forceinline__ void f_take(const FSmem& sm, uint32_t lane_base, uint
   mbar_arrive_elect(&sm.tempty[s0]);
 }
 
+__device__ __forceinline__ int lds1i(const int* p) {
+  int v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)));
+  return v;
+}
+
 // Key sum over 32 rows with per-row checks: rows that do not exist (tp < 0)
 // or that cannot see key k (k > position) add nothing.
 __device__ __forceinline__ void s2_chunk_rows(const uint32_t (&rr)[32], float c, const float* nl, const int* tp,
                                               int k, float2 (&a)[4]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
-    if (k <= tp[i]) {
+    if (k <= lds1i(tp + i)) {
       const float e = ex2_approx(fmaf(__uint_as_float(rr[i]), c, lds1(nl + i)));
       if (i & 1) a[(i >> 1) & 3].y += e; else a[(i >> 1) & 3].x += e;
     }
