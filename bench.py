@@ -281,7 +281,7 @@ def run_reference(args, rank, world):
 
 def kernel_hash() -> str:
     h = hashlib.sha256()
-    for f in ("score.cu", "kvev_internal.cuh"):
+    for f in ("score.cu", "score_common.cuh", "kvev_internal.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2606_15157_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
