@@ -459,8 +459,9 @@ def run_ours(args, rank, world, local_rank):
 def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_ranks,
             sum_over_ranks):
     """Same metric through the public API, starting every step from pinned host
-    memory: the inputs the tensor-core path streams (K and Q_win of the SnapKV /
-    H2O layers) are copied to the device on four copy streams, and the tensors
+    memory: the inputs the tensor-core path streams (the prompt rows of K and
+    Q_win of the SnapKV / H2O layers) are copied to the device on four copy
+    streams, and the tensors
     that are only gathered row by row (V of every layer, K of the StreamingLLM
     layers) stay in pinned host memory, read in place over the host link by
     the gather kernel; the kept indices and counts are read back.  The bytes
@@ -477,7 +478,13 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
         if scoring[l]:
             K_arg.append(Kd)
             Q_arg.append(Qd)
-            copies += [(Kh, Kd), (Qh, Qd)]
+            # the prompt rows of each (sequence, KV head): a contiguous slice of
+            # [B][H_kv][S_cap][d]; rows past a sequence's length are never read
+            for s in range(wl.B):
+                n = int(wl.lens[s])
+                if n > 0:
+                    copies += [(Kh[s, h, :n], Kd[s, h, :n]) for h in range(wl.H_kv)]
+            copies.append((Qh, Qd))
         else:
             K_arg.append(Kh)
             Q_arg.append(None)
