@@ -19,8 +19,8 @@
 // the protected recent window (r = h2o_recent for H2O, 0 for TOVA) is
 // evicted, ties to the higher position, and the new token takes its place
 // (unless the new token itself is the one evicted).  The retained K rows are
-// streamed once (16-byte loads, d/8 lanes per row); logits stay in shared
-// memory.
+// streamed once, as 16-byte loads feeding m16n8k16 tensor-core products of
+// the G query rows; logits stay in shared memory.
 #include "kvev_internal.cuh"
 
 namespace kvev {
@@ -29,8 +29,6 @@ namespace {
 
 constexpr int kDecodeThreads = 256;
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // Unit index -> layer: the last layer whose first unit is <= u (layers
 // without slots own no units and share their unit_off with the next layer).
@@ -140,88 +138,84 @@ __device__ __forceinline__ void place_new(const DecodeParams& p, const UnitRef& 
   }
 }
 
+// One m16n8k16 bf16 tensor-core product with fp32 accumulation (per warp):
+// d[16 x 8] += a[16 x 16] * b[16 x 8].
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 // H2O / TOVA unit.  lg: [G][cap + 1] floats of shared memory.
+//
+// Logits: a warp takes 16 slots at a time and forms S[16 slots][8 heads] =
+// K Q^T on the tensor core (m16n8k16, heads past G are zero columns).  The
+// dot product runs over d in a permuted order that lets every lane fill its
+// A fragment from 16-byte loads of whole K rows: in the k-step pair kp, lane
+// quadrant t (= lane % 4) holds dims kp*32 + t*8 + [0, 8) of its two slot
+// rows; k-step 2kp + w takes elements 4w .. 4w + 3 of that slice (the low two
+// as fragment columns 2t, 2t+1, the high two as 2t+8, 2t+9), and Q's B
+// fragment is loaded in the same order.
 template <int D, int G>
 __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int n, int c,
                             float* lg, DecShared& sh) {
-  constexpr int LPS = D / 8;     // lanes per slot row (16 bytes each)
-  constexpr int SPW = 32 / LPS;  // slot rows per warp per pass
-  constexpr int SPB = SPW * (kDecodeThreads / 32);
+  constexpr int KP = D / 32;  // k-step pairs
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int sub = lane % LPS, grp = lane / LPS;
+  const int gid = lane >> 2, tig = lane & 3;
   const int ld = ly.cap + 1;  // row stride of lg
   const uint16_t* Kb = static_cast<const uint16_t*>(p.K) + r.rows0 * D;
   const uint16_t* qn =
       static_cast<const uint16_t*>(p.q_new[r.l]) + (static_cast<size_t>(r.s) * p.H_q + r.h * G) * D;
   const uint16_t* kn = static_cast<const uint16_t*>(p.k_new[r.l]) + (static_cast<size_t>(r.s) * p.H_kv + r.h) * D;
 
-  // this lane's 8 elements of each query row, scaled into the exp2 domain
-  float q[G][8];
+  // B fragments: head gid (column), dims kp*32 + tig*8 + 4w + [0, 4) of k-step 2kp + w
+  uint32_t bq[2 * KP][2];
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    const uint4 v = *reinterpret_cast<const uint4*>(qn + g * D + sub * 8);
-    const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+  for (int kp = 0; kp < KP; ++kp) {
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      q[g][2 * e] = bf16_lo(w4[e]) * p.scale_log2;
-      q[g][2 * e + 1] = bf16_hi(w4[e]) * p.scale_log2;
+    for (int w = 0; w < 2; ++w) {
+      uint2 v = make_uint2(0, 0);
+      if (gid < G) v = *reinterpret_cast<const uint2*>(qn + gid * D + kp * 32 + tig * 8 + 4 * w);
+      bq[2 * kp + w][0] = v.x;
+      bq[2 * kp + w][1] = v.y;
     }
   }
-  // logits (base 2) of slots 0..c-1 and of the new token at index c; kU row
-  // passes per iteration, their loads issued before any arithmetic
-  constexpr int kU = 4;
+  // Slots 0..c-1 from the arena and the new token (index c) from its own k
+  // row, 16 per tile; tiles are dealt to the warps in turn.
   const int cnt = c + 1;
-  for (int j0 = 0; j0 < cnt; j0 += kU * SPB) {
-    uint4 kv[kU];
+  const int ntiles = (cnt + 15) / 16;
+  for (int t = warp; t < ntiles; t += kDecodeThreads / 32) {
+    const int j0 = t * 16 + gid, j1 = j0 + 8;  // this lane's two slot rows
+    uint4 X[KP], Y[KP];
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int j = j0 + u * SPB + warp * SPW + grp;
-      kv[u] = make_uint4(0, 0, 0, 0);
-      if (j < c) kv[u] = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j) * D + sub * 8));
-      else if (j == c) kv[u] = *reinterpret_cast<const uint4*>(kn + sub * 8);
+    for (int kp = 0; kp < KP; ++kp) {
+      const int off = kp * 32 + tig * 8;
+      X[kp] = make_uint4(0, 0, 0, 0);
+      Y[kp] = make_uint4(0, 0, 0, 0);
+      if (j0 < c) X[kp] = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j0) * D + off));
+      else if (j0 == c) X[kp] = *reinterpret_cast<const uint4*>(kn + off);
+      if (j1 < c) Y[kp] = __ldcs(reinterpret_cast<const uint4*>(Kb + static_cast<size_t>(j1) * D + off));
+      else if (j1 == c) Y[kp] = *reinterpret_cast<const uint4*>(kn + off);
     }
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int j = j0 + u * SPB + warp * SPW + grp;
-      const uint32_t w4[4] = {kv[u].x, kv[u].y, kv[u].z, kv[u].w};
-      float kf[8];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        kf[2 * e] = bf16_lo(w4[e]);
-        kf[2 * e + 1] = bf16_hi(w4[e]);
-      }
-      float a[G];
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        a[g] = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) a[g] = fmaf(q[g][e], kf[e], a[g]);
-      }
-      // Sum each head's partials over the row's LPS lanes, splitting the G
-      // values between lane halves at every step (log2(LPS) + G - 1 shuffles
-      // instead of G * log2(LPS)); afterwards lane `sub` holds the total of
-      // head sub / (LPS / G).
-      int nv = G;
-#pragma unroll
-      for (int o = LPS / 2; o > 0; o >>= 1) {
-        if (nv > 1) {
-          const bool upper = (sub & o) != 0;
-          const int half = nv / 2;
-#pragma unroll
-          for (int i = 0; i < G / 2; ++i) {
-            if (i < half) {
-              const float send = upper ? a[i] : a[i + half];
-              const float keep = upper ? a[i + half] : a[i];
-              a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-            }
-          }
-          nv = half;
-        } else {
-          a[0] += __shfl_xor_sync(0xffffffffu, a[0], o);
-        }
-      }
-      constexpr int kLanesPerHead = LPS / G;
-      if (sub % kLanesPerHead == 0 && j < cnt) lg[(sub / kLanesPerHead) * ld + j] = a[0];
+    for (int kp = 0; kp < KP; ++kp) {
+      const uint32_t a0[4] = {X[kp].x, Y[kp].x, X[kp].y, Y[kp].y};
+      const uint32_t a1[4] = {X[kp].z, Y[kp].z, X[kp].w, Y[kp].w};
+      mma_16816(acc, a0, bq[2 * kp][0], bq[2 * kp][1]);
+      mma_16816(acc, a1, bq[2 * kp + 1][0], bq[2 * kp + 1][1]);
+    }
+    // acc: (slot j0, heads 2tig, 2tig+1) and (slot j1, same heads)
+    const int h0 = 2 * tig;
+    if (h0 < G) {
+      if (j0 < cnt) lg[h0 * ld + j0] = acc[0] * p.scale_log2;
+      if (j1 < cnt) lg[h0 * ld + j1] = acc[2] * p.scale_log2;
+    }
+    if (h0 + 1 < G) {
+      if (j0 < cnt) lg[(h0 + 1) * ld + j0] = acc[1] * p.scale_log2;
+      if (j1 < cnt) lg[(h0 + 1) * ld + j1] = acc[3] * p.scale_log2;
     }
   }
   __syncthreads();
