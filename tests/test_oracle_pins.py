@@ -42,8 +42,8 @@ def test_alloc_hand_case_clamp_and_largest_remainder(orc):
 
 
 def test_alloc_hand_case_iterated_clamping(orc):
-    # b~ = [1, 5, 10, 84]: round 1 fixes layers 0,1; the re-split gives layer 2
-    # 80*10/94 = 8.5 < 10 so round 2 fixes it too; layer 3 takes the rest.
+    # b~ = [1, 5, 10, 84]: the first clamping pass fixes layers 0,1; the re-split gives layer 2
+    # 80*10/94 = 8.5 < 10 so the second pass fixes it too; layer 3 takes the rest.
     b = orc.alloc_from_scores([1, 5, 10, 84], 100, 10)
     assert b.tolist() == [10, 10, 10, 70]
 
