@@ -357,6 +357,14 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
   }
   const float* raw =
       p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
+  // pull the unit's scores into L2 in 16 KiB pieces (16-byte aligned, whole
+  // 16-byte blocks: the score array is one 256-byte aligned workspace region)
+  {
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(raw) & ~uintptr_t(15);
+    const uintptr_t a1 = (reinterpret_cast<uintptr_t>(raw + E) + 15) & ~uintptr_t(15);
+    const uintptr_t a = a0 + static_cast<uintptr_t>(threadIdx.x) * 16384;
+    if (a < a1) prefetch_l2_bulk(reinterpret_cast<const void*>(a), static_cast<uint32_t>(a1 - a < 16384 ? a1 - a : 16384));
+  }
   for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
   __syncthreads();
   build_keys(keys, sh.hist, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV);
