@@ -27,6 +27,12 @@ namespace kvev {
 
 namespace {
 
+// Bulk prefetch of [src, src + bytes) into L2 (src 16-byte aligned, bytes a
+// multiple of 16).
+__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 constexpr int kHistBits = 12;              // first radix digit: the top 12 bits of a key
 constexpr int kHistBins = 1 << kHistBits;
 constexpr int kSelWarps = kSelectThreads / 32;
