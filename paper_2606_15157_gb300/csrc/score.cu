@@ -15,24 +15,25 @@
 //            max / sum of exp2 in registers -> per-chunk partials;
 //   sweep 2: S^T = K Q^T on the tensor core (keys on TMEM lanes), each thread
 //            owns one key and sums exp2(s*log2e/sqrt(d) - lse2_r) over the rows.
-// Work items are chunks of chunk_keys keys.  A CTA runs sweep 1 of item j+1
-// before sweep 2 of item j, so the re-read of item j's K tiles (one round of
-// the whole grid later, ~grid*chunk bytes of new traffic) is served by L2 and
-// the per-unit normaliser is ready without any CTA idling.  The last chunk of a
-// unit to finish sweep 1 combines the partials and publishes lse (release
-// flag); sweep-2 readers spin on it with a time bound.  All CTAs are
-// co-resident (cooperative launch) and a unit spans at most two rounds of
+// Work items are chunks of chunk_keys keys (an even number of 128-key tiles,
+// swept in 256-key super-tiles).  A CTA runs sweep 1 of item j + kLag before
+// sweep 2 of item j, so the unit's normaliser, which needs every chunk of the
+// unit (some on other CTAs), is almost always published by the time sweep 2
+// needs it.  The chunk whose partials complete the unit's merge tree publishes
+// lse2 (release flag); sweep-2 readers wait on it with a time bound.  All CTAs
+// are co-resident (cooperative launch) and a unit spans at most two rounds of
 // items, so the wait always ends.
 //
 // Roles per CTA (640 threads, five warpgroups): warp 0 issues TMA loads (one
-// thread), warp 1 owns TMEM and issues tcgen05.mma (one thread), warps 2-3
-// idle; warpgroups 1-4 are softmax warpgroups.  TMEM is four 128-column
-// slots, one per 128-row group of a tile's accumulator (a tile uses one or
-// two), and softmax warpgroup w owns slot w: it copies the slot to registers
-// in 64-column pieces and releases it before the last piece's arithmetic, so
-// the tensor core keeps filling the other slots meanwhile.  The softmax
-// warpgroups never wait on each other.  setmaxnreg moves registers from
-// warpgroup 0 to the softmax warpgroups.
+// thread); warp 1 owns TMEM and issues tcgen05.mma (an elected lane); warp 2
+// publishes each chunk's row partials and climbs the unit's merge tree; warp 3
+// stages -lse2 for sweep 2; warpgroups 1-4 are softmax warpgroups.  The tensor
+// core fills 256-column TMEM units (two adjacent 128-column slots) in a ring
+// of two: sweep 1 one unit per (super-tile, 128-row group), sweep 2 one unit
+// per 128-key tile.  All four softmax warpgroups consume every unit, 64
+// columns each, copying them with one tcgen05.ld and releasing the unit
+// before any arithmetic.  setmaxnreg moves registers from warpgroup 0 to the
+// softmax warpgroups.
 #include "score_common.cuh"
 
 namespace kvev {
