@@ -311,6 +311,23 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
+def rank_reducers(dist: bool, device: str):
+    """(max over ranks, sum over ranks) of a host float: an all-reduce of one
+    fp64 value on `device` (NCCL between GPU ranks, gloo on CPU); the identity
+    for a single process."""
+    if not dist:
+        return (lambda x: x), (lambda x: x)
+    import torch
+    import torch.distributed as td
+
+    def red(x: float, op) -> float:
+        t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+        td.all_reduce(t, op=op)
+        return float(t.item())
+
+    return (lambda x: red(x, td.ReduceOp.MAX)), (lambda x: red(x, td.ReduceOp.SUM))
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     from paper_2606_15157_gb300 import kvev
@@ -350,15 +367,7 @@ def run_ours(args, rank, world, local_rank):
             td.barrier()
         torch.cuda.synchronize()
 
-    def reduce(x: float, op) -> float:
-        if not dist:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        td.all_reduce(t, op=op)
-        return float(t.item())
-
-    max_over_ranks = lambda x: reduce(x, td.ReduceOp.MAX) if dist else x
-    sum_over_ranks = lambda x: reduce(x, td.ReduceOp.SUM) if dist else x
+    max_over_ranks, sum_over_ranks = rank_reducers(dist, "cuda")
 
     # ---- device-resident timed region ----
     kvev.kvev_plan_enable_timing(plan.handle, True)
@@ -662,10 +671,9 @@ def run_decode(args, rank, world, local_rank):
             td.barrier()
     per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
     ms = evs[0].elapsed_time(evs[-1]) / args.steps
-    if dist:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        td.all_reduce(t, op=td.ReduceOp.MAX)
-        ms = float(t.item())
+    max_over_ranks, sum_over_ranks = rank_reducers(dist, "cuda")
+    ms = max_over_ranks(ms)
+    all_bytes = sum_over_ranks(float(step_bytes))
     assert plan.status() == kvev.OK
     peaks = {}
     try:
@@ -673,7 +681,7 @@ def run_decode(args, rank, world, local_rank):
     except (OSError, ValueError):
         pass
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
-    value = world * step_bytes / (ms / 1e3) / 1e9
+    value = all_bytes / (ms / 1e3) / 1e9
     achieved = step_bytes / (statistics.median(per) / 1e3) / 1e9
     if rank == 0:
         out = {
