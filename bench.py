@@ -596,17 +596,21 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
             "pipelining": "two device copies of the streamed inputs; uploads overlap the previous step"}
 
 
-def decode_step_bytes(wl, counts):
+def decode_step_bytes(wl, counts, supplied_attention=False):
     """Algorithmic bytes of one decode step: for H2O/TOVA units the retained K rows,
-    the new token's k/q, the slots' positions and acc (read and written); for every
-    unit the new K/V row written (and StreamingLLM's position scan)."""
+    the new token's k/q, the slots' positions and acc (read and written), or with
+    the attention supplied by the caller that attention row (4 B per slot) instead
+    of K and q; for every unit the new K/V row written (and StreamingLLM's
+    position scan)."""
     row = wl.d * 2
     tot = 0
     for l in range(wl.L):
         md = int(wl.route_decode[l])
         c = counts[l]
         units = wl.B * wl.H_kv
-        if md in (gen.H2O, gen.TOVA):
+        if md in (gen.H2O, gen.TOVA) and supplied_attention:
+            tot += units * (4 * (c + 1) + c * 12 + row + 2 * row)
+        elif md in (gen.H2O, gen.TOVA):
             tot += units * (c * row + c * 12 + row * (1 + wl.G) + 2 * row)
         elif md == gen.STREAMING:
             tot += units * (c * 4 + 2 * row)
@@ -643,12 +647,28 @@ def run_decode(args, rank, world, local_rank):
     toks = [[gen.device_decode_tokens(wl, t, l) for l in range(wl.L)] for t in range(total)]
     torch.cuda.synchronize()
     counts = [int(wl.budget[l]) for l in range(wl.L)]
-    step_bytes = decode_step_bytes(wl, counts)
+    step_bytes = decode_step_bytes(wl, counts, args.decode_attn)
     stream = torch.cuda.current_stream()
+    attn = None
+    if args.decode_attn:
+        # the caller's decode attention would supply these every step; any valid
+        # rows cost the same, so one seeded set of distributions is reused
+        g = torch.Generator(device="cuda")
+        g.manual_seed(77 + rank)
+        attn = []
+        for l, (_, cap, _) in enumerate(arena.layers):
+            if cap > 0 and int(wl.route_decode[l]) in (gen.H2O, gen.TOVA):
+                a = torch.rand((wl.B, wl.H_kv, cap + 1), generator=g, device="cuda")
+                attn.append(a / a.sum(dim=2, keepdim=True))
+            else:
+                attn.append(None)
 
     def run(t):
         k = [x[0] for x in toks[t]]
         v = [x[1] for x in toks[t]]
+        if attn is not None:
+            arena.step_attn(k, v, attn, stream)
+            return
         q = [x[2] for x in toks[t]]
         arena.step(k, v, q, stream)
 
@@ -691,6 +711,8 @@ def run_decode(args, rank, world, local_rank):
             "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded; shapes of LLaMA-3.1-8B decode with compacted caches)",
             "config": {"workload": wl.name, "layers": wl.L, "batch": wl.B, "cache_slots": 2048,
+                       "attention": "supplied by the caller (kvev_decode_step_attn)" if args.decode_attn
+                       else "computed from q_new and the retained K",
                        "route_decode": {"h2o": int((wl.route_decode == gen.H2O).sum()),
                                         "streaming": int((wl.route_decode == gen.STREAMING).sum()),
                                         "append": int(((wl.route_decode == gen.FULL) &
@@ -721,6 +743,8 @@ def main():
                          "in the decode workload (profiling)")
     ap.add_argument("--h2o-full-prompt", action="store_true",
                     help="H2O layers score every prompt query row (reports causal-attention TFLOP/s)")
+    ap.add_argument("--decode-attn", action="store_true",
+                    help="decode workload: the caller supplies the attention (kvev_decode_step_attn)")
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

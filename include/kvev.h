@@ -369,6 +369,24 @@ KVEV_API int kvev_decode_step(kvev_plan *plan, int B, int growth, void *dec_K, v
                               void *dec_state, const void *const *k_new, const void *const *v_new,
                               const void *const *q_new, void *stream);
 
+/* The decode step with the attention supplied by the caller's own decode
+ * attention kernel (the fused form of Sec. 2.1's H2O / TOVA decode rules: the
+ * caller's attention already reads the retained K, so the step reads none).
+ *   attn[L]  host array of device pointers; for every H2O / TOVA layer fp32
+ *            [B][H_kv][cap_l + 1] (cap_l from kvev_decode_layer): for each
+ *            unit (s, h) with count c, entries 0..c-1 are the group-mean
+ *            softmax weights of the new token's queries on arena slots
+ *            0..c-1 (slot order of the arena, as in dec_K) and entry c the
+ *            weight on the new token itself, the softmax running over the
+ *            retained slots and the new token; entries past c are not read.
+ *            NULL for other layers.  4-byte aligned.
+ * Everything else (append, acc update, eviction, StreamingLLM, FULL) is as in
+ * kvev_decode_step; no queries are needed.  EINVAL if attn or an H2O / TOVA
+ * layer's entry is NULL or misaligned. */
+KVEV_API int kvev_decode_step_attn(kvev_plan *plan, int B, int growth, void *dec_K, void *dec_V,
+                                   void *dec_state, const void *const *k_new,
+                                   const void *const *v_new, const float *const *attn, void *stream);
+
 /* ---- measurement ---------------------------------------------------------- */
 
 /* Kernels of one kvev_evict_prefill() call, in launch order. */

@@ -1021,10 +1021,13 @@ extern "C" int kvev_decode_init(kvev_plan* plan, int B, int growth, const void* 
   return launch_decode_init(dp, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
 }
 
-extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_V,
-                                void* dec_state, const void* const* k_new,
-                                const void* const* v_new, const void* const* q_new,
-                                void* stream) {
+namespace {
+
+// One decode step; the H2O / TOVA layers take their attention from q_new
+// (attn == nullptr) or from the caller (attn[l]).
+int decode_step_impl(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_V, void* dec_state,
+                     const void* const* k_new, const void* const* v_new, const void* const* q_new,
+                     const float* const* attn, void* stream) {
   if (!plan || B < 0) return KVEV_EINVAL;
   kvev_plan& P = *plan;
   DecLayout d;
@@ -1033,7 +1036,8 @@ extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K,
   if (B == 0) return KVEV_OK;
   if (!dec_state || (reinterpret_cast<uintptr_t>(dec_state) & 255u)) return KVEV_EINVAL;
   if (d.units > 0) {
-    if (!dec_K || !dec_V || !k_new || !v_new || !q_new || !aligned16(dec_K) || !aligned16(dec_V))
+    if (!dec_K || !dec_V || !k_new || !v_new || (!q_new && !attn) || !aligned16(dec_K) ||
+        !aligned16(dec_V))
       return KVEV_EINVAL;
     if (!decode_supported(P.d, P.G)) return KVEV_ENOTSUP;
   }
@@ -1044,10 +1048,15 @@ extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K,
     if (d.cap[l] == 0) continue;
     if (!k_new[l] || !v_new[l] || !aligned16(k_new[l]) || !aligned16(v_new[l])) return KVEV_EINVAL;
     const bool attends = P.route_dec[l] == KVEV_H2O || P.route_dec[l] == KVEV_TOVA;
-    if (attends && (!q_new[l] || !aligned16(q_new[l]))) return KVEV_EINVAL;
+    if (attends && attn) {
+      if (!attn[l] || (reinterpret_cast<uintptr_t>(attn[l]) & 3u)) return KVEV_EINVAL;
+      dp.attn[l] = attn[l];
+    } else if (attends && (!q_new[l] || !aligned16(q_new[l]))) {
+      return KVEV_EINVAL;
+    }
     dp.k_new[l] = k_new[l];
     dp.v_new[l] = v_new[l];
-    dp.q_new[l] = q_new[l];
+    dp.q_new[l] = q_new ? q_new[l] : nullptr;
   }
   rc = ensure_device(plan);
   if (rc != KVEV_OK) return rc;
@@ -1058,6 +1067,25 @@ extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   P.last_stream = s;
   return launch_decode_step(dp, smem, s) == cudaSuccess ? KVEV_OK : KVEV_ECUDA;
+}
+
+}  // namespace
+
+extern "C" int kvev_decode_step(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_V,
+                                void* dec_state, const void* const* k_new,
+                                const void* const* v_new, const void* const* q_new,
+                                void* stream) {
+  return decode_step_impl(plan, B, growth, dec_K, dec_V, dec_state, k_new, v_new, q_new, nullptr,
+                          stream);
+}
+
+extern "C" int kvev_decode_step_attn(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_V,
+                                     void* dec_state, const void* const* k_new,
+                                     const void* const* v_new, const float* const* attn,
+                                     void* stream) {
+  if (!attn) return KVEV_EINVAL;
+  return decode_step_impl(plan, B, growth, dec_K, dec_V, dec_state, k_new, v_new, nullptr, attn,
+                          stream);
 }
 
 // ---------------------------------------------------------------------------

@@ -148,28 +148,14 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4],
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// H2O / TOVA unit.  lg: [G][cap + 1] floats of shared memory.
-//
-// Logits: a warp takes 16 slots at a time and forms S[16 slots][8 heads] =
-// K Q^T on the tensor core (m16n8k16, heads past G are zero columns).  The
-// dot product runs over d in a permuted order that lets every lane fill its
-// A fragment from 16-byte loads of whole K rows: in the k-step pair kp, lane
-// quadrant t (= lane % 4) holds dims kp*32 + t*8 + [0, 8) of its two slot
-// rows; k-step 2kp + w takes elements 4w .. 4w + 3 of that slice (the low two
-// as fragment columns 2t, 2t+1, the high two as 2t+8, 2t+9), and Q's B
-// fragment is loaded in the same order.
+// Logits (base 2) of the G query rows against slots 0..c-1 and the new token
+// (index c) into lg[head][j].
 template <int D, int G>
-__device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int n, int c,
-                            float* lg, DecShared& sh) {
+__device__ __forceinline__ void unit_logits(const DecodeParams& p, const uint16_t* Kb, const uint16_t* qn,
+                                            const uint16_t* kn, int c, int ld, float* lg) {
   constexpr int KP = D / 32;  // k-step pairs
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, tig = lane & 3;
-  const int ld = ly.cap + 1;  // row stride of lg
-  const uint16_t* Kb = static_cast<const uint16_t*>(p.K) + r.rows0 * D;
-  const uint16_t* qn =
-      static_cast<const uint16_t*>(p.q_new[r.l]) + (static_cast<size_t>(r.s) * p.H_q + r.h * G) * D;
-  const uint16_t* kn = static_cast<const uint16_t*>(p.k_new[r.l]) + (static_cast<size_t>(r.s) * p.H_kv + r.h) * D;
-
   // B fragments: head gid (column), dims kp*32 + tig*8 + 4w + [0, 4) of k-step 2kp + w
   uint32_t bq[2 * KP][2];
 #pragma unroll
@@ -218,11 +204,43 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
       if (j1 < cnt) lg[(h0 + 1) * ld + j1] = acc[3] * p.scale_log2;
     }
   }
+}
+
+// H2O / TOVA unit.  lg: [G][cap + 1] floats of shared memory.
+//
+// Logits: a warp takes 16 slots at a time and forms S[16 slots][8 heads] =
+// K Q^T on the tensor core (m16n8k16, heads past G are zero columns).  The
+// dot product runs over d in a permuted order that lets every lane fill its
+// A fragment from 16-byte loads of whole K rows: in the k-step pair kp, lane
+// quadrant t (= lane % 4) holds dims kp*32 + t*8 + [0, 8) of its two slot
+// rows; k-step 2kp + w takes elements 4w .. 4w + 3 of that slice (the low two
+// as fragment columns 2t, 2t+1, the high two as 2t+8, 2t+9), and Q's B
+// fragment is loaded in the same order.
+template <int D, int G>
+__device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int n, int c,
+                            float* lg, DecShared& sh) {
+  const int ld = ly.cap + 1;  // row stride of lg
+  const uint16_t* Kb = static_cast<const uint16_t*>(p.K) + r.rows0 * D;
+  const uint16_t* kn = static_cast<const uint16_t*>(p.k_new[r.l]) + (static_cast<size_t>(r.s) * p.H_kv + r.h) * D;
+  const uint16_t* qn = p.q_new[r.l] == nullptr
+                           ? nullptr
+                           : static_cast<const uint16_t*>(p.q_new[r.l]) +
+                                 (static_cast<size_t>(r.s) * p.H_q + r.h * G) * D;
+
+  // attention supplied by the caller's own decode attention: slots 0..c-1, then the new token
+  const float* at = p.attn[r.l] == nullptr
+                        ? nullptr
+                        : p.attn[r.l] + (static_cast<size_t>(r.s) * p.H_kv + r.h) * static_cast<size_t>(ld);
+  if (at == nullptr) unit_logits<D, G>(p, Kb, qn, kn, c, ld, lg);
+  const int cnt = c + 1;
   __syncthreads();
-  // per-head softmax statistics
+  // per-head softmax statistics (not needed when the attention is supplied)
   float mg[G], zg[G];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
+    mg[g] = 0.f;
+    zg[g] = 1.f;
+    if (at != nullptr) continue;
     float m = -INFINITY;
     for (int j = threadIdx.x; j < cnt; j += blockDim.x) m = fmaxf(m, lg[g * ld + j]);
     mg[g] = block_max(m, sh);
@@ -238,9 +256,13 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
   int bp = -1, bs = -1;
   for (int j = threadIdx.x; j < cnt; j += blockDim.x) {
     float pj = 0.f;
+    if (at != nullptr) {
+      pj = at[j];
+    } else {
 #pragma unroll
-    for (int g = 0; g < G; ++g) pj += exp2f(lg[g * ld + j] - mg[g]) / zg[g];
-    pj *= 1.0f / static_cast<float>(G);
+      for (int g = 0; g < G; ++g) pj += exp2f(lg[g * ld + j] - mg[g]) / zg[g];
+      pj *= 1.0f / static_cast<float>(G);
+    }
     const float a = (ly.method == KVEV_H2O && j < c) ? accr[j] + pj : pj;
     lg[j] = a;
     const int pos = j < c ? posr[j] : n;

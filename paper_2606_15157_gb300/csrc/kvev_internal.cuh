@@ -142,6 +142,7 @@ struct DecodeParams {
   const void* k_new[kMaxLayers];  // [B][H_kv][d] bf16 per layer
   const void* v_new[kMaxLayers];  // [B][H_kv][d]
   const void* q_new[kMaxLayers];  // [B][H_q][d]
+  const float* attn[kMaxLayers];  // [B][H_kv][cap + 1] caller-supplied attention, or null
   int L, B, H_kv, H_q, G, d, units;
   float scale_log2;   // log2(e) / sqrt(d)
   void* K;            // arena rows [rows][d] bf16

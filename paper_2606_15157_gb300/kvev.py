@@ -31,7 +31,7 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
            "kvev_plan_last_timings", "kvev_evict_prefill_noalloc", "kvev_decode_query",
            "kvev_decode_layer", "kvev_decode_state_offsets", "kvev_decode_init",
-           "kvev_decode_step", "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
+           "kvev_decode_step", "kvev_decode_step_attn", "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
            "kvev_route_toprank", "kvev_route_install", "kvev_plan_save", "kvev_plan_load",
            "kvev_plan_set_h2o_full_prompt"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
@@ -82,6 +82,7 @@ def load(path: str = LIB_PATH):
         L.kvev_decode_state_offsets.argtypes = [vp, C.c_int, C.c_int, P(sz)]
         L.kvev_decode_init.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
         L.kvev_decode_step.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
+        L.kvev_decode_step_attn.argtypes = [vp, C.c_int, C.c_int, vp, vp, vp, vp, vp, vp, vp]
         L.kvev_profile_cosine.argtypes = [vp, vp, vp, C.c_int, C.c_int, i64]
         L.kvev_score_ppl.argtypes = [vp, vp, C.c_double, C.c_int, C.c_int]
         L.kvev_score_entropy.argtypes = [vp, vp, C.c_int, i64, C.c_int]
@@ -215,6 +216,14 @@ def kvev_decode_step(handle, B, growth, dec_K, dec_V, dec_state, k_ptrs, v_ptrs,
     arr = C.c_void_p * len(k_ptrs)
     return load().kvev_decode_step(handle, B, growth, dec_K, dec_V, dec_state, arr(*k_ptrs),
                                    arr(*v_ptrs), arr(*q_ptrs), stream)
+
+
+def kvev_decode_step_attn(handle, B, growth, dec_K, dec_V, dec_state, k_ptrs, v_ptrs, attn_ptrs,
+                          stream) -> int:
+    """Pointer-level call; returns the status code (does not raise)."""
+    arr = C.c_void_p * len(k_ptrs)
+    return load().kvev_decode_step_attn(handle, B, growth, dec_K, dec_V, dec_state, arr(*k_ptrs),
+                                        arr(*v_ptrs), arr(*attn_ptrs), stream)
 
 
 def kvev_status(handle: int) -> int:
@@ -474,6 +483,18 @@ class DecodeArena:
                                 bufs["out_count"].data_ptr(), bufs["h2o_state"].data_ptr(),
                                 lens.data_ptr(), self.K.data_ptr(), self.V.data_ptr(),
                                 self.state.data_ptr(), stream.cuda_stream), "kvev_decode_init")
+
+    def step_attn(self, k_new, v_new, attn, stream=None):
+        """Decode step with caller-supplied attention: attn[l] fp32 [B][H_kv][cap_l + 1]
+        CUDA tensors for H2O / TOVA layers (None elsewhere)."""
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        ptr = lambda t: None if t is None else t.data_ptr()
+        _check(kvev_decode_step_attn(self.plan.handle, self.B, self.growth, self.K.data_ptr(),
+                                     self.V.data_ptr(), self.state.data_ptr(), [ptr(t) for t in k_new],
+                                     [ptr(t) for t in v_new], [ptr(t) for t in attn],
+                                     stream.cuda_stream), "kvev_decode_step_attn")
 
     def step(self, k_new, v_new, q_new, stream=None):
         """k_new, v_new, q_new: per-layer CUDA tensors (or None for layers without an arena)."""

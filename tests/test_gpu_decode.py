@@ -194,6 +194,74 @@ def test_decode_lockstep_mixed_rules(env, d):
                 assert set(range(first, n_now)) <= set(x["pos"].tolist())
 
 
+def _bf16_to_f64(u16):
+    return (np.asarray(u16, np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def supplied_attention(torch, wl, g, toks, layers_attend):
+    """Per H2O / TOVA layer, fp32 [B][H_kv][cap + 1]: the group-mean softmax of the
+    new token's queries over the unit's slots (arena slot order) and the new
+    token (last), in fp64 from the definition."""
+    attn = {}
+    host = {l: tuple(t.view(torch.int16).cpu().numpy().view(np.uint16) for t in toks[l]) for l in layers_attend}
+    for i, (l, s, h, u, r0, cap) in enumerate(g.units):
+        if l not in layers_attend:
+            continue
+        a = attn.setdefault(l, np.zeros((wl.B, wl.H_kv, cap + 1), np.float32))
+        c = int(g.count[u])
+        k, _, q = host[l]
+        keys = np.concatenate([_bf16_to_f64(g.K[r0:r0 + c]), _bf16_to_f64(k[s, h])[None, :]], axis=0)
+        qg = _bf16_to_f64(q[s, h * wl.G:(h + 1) * wl.G])
+        x = qg @ keys.T / np.sqrt(wl.d)                 # [G][c + 1]
+        pr = np.exp(x - x.max(axis=1, keepdims=True))
+        pr /= pr.sum(axis=1, keepdims=True)
+        a[s, h, :c + 1] = pr.mean(axis=0)
+    return {l: torch.from_numpy(v).cuda() for l, v in attn.items()}
+
+
+def test_decode_lockstep_supplied_attention(env):
+    # kvev_decode_step_attn (the caller's decode attention supplies p) against
+    # the oracle, which computes p from the queries itself: same rules, same
+    # lock-step comparison as above.
+    torch, kvev, orc = env
+    wl = gen.config_decode_mixed(seed=5, d=128)
+    growth = wl.decode_steps + 8
+    plan, bufs, arena = prefill_and_arena(torch, kvev, wl, growth)
+    g = Arena(torch, arena, wl)
+    all_units = list(range(len(g.units)))
+    states = [oracle_state(orc, wl, wl.route_decode, g, i) for i in all_units]
+    layers = sorted({g.units[i][0] for i in all_units})
+    attending = {l for l in layers if int(wl.route_decode[l]) in (kvev.H2O, kvev.TOVA)}
+    assert attending
+    ties = 0
+    for step in range(wl.decode_steps):
+        toks, k, v, q = step_tokens(wl, step, layers)
+        attn = supplied_attention(torch, wl, g, toks, attending)
+        arena.step_attn(k, v, [attn.get(l) for l in range(wl.L)])
+        kn, vn, qn = host_tokens(torch, toks, wl, all_units, g)
+        orc.decode_step(states, kn, vn, qn, wl.d, wl.G)
+        g.refresh(torch)
+        assert np.array_equal(g.lens, wl.lens + step + 1)
+        for i in all_units:
+            l, s, h = g.units[i][:3]
+            x = g.unit(i)
+            if compare_unit(states[i], x, f"step {step} layer {l} seq {s} head {h}") == "tie":
+                ties += 1
+                resync(states[i], x)
+    assert plan.status() == kvev.OK
+    assert ties <= len(all_units)
+
+
+def test_decode_step_attn_rejects_missing_rows(env):
+    torch, kvev, orc = env
+    wl = gen.config_decode_mixed(seed=5, d=128)
+    plan, bufs, arena = prefill_and_arena(torch, kvev, wl, 8)
+    layers = [l for l in range(wl.L) if arena.layers[l][1] > 0]
+    toks, k, v, q = step_tokens(wl, 0, layers)
+    with pytest.raises(kvev.KvevError):
+        arena.step_attn(k, v, [None] * wl.L)
+
+
 def test_decode_full_size_sampled(env):
     """The decode workload at full size (batch 16, 16K caches compacted to 2048,
     32 layers): invariants on every unit over a few steps, and lock-step oracle
