@@ -249,6 +249,25 @@ KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const voi
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
                        float *h2o_state, void *workspace, size_t workspace_bytes, void *stream);
 
+/* kvev_evict_prefill with the scores of chosen scoring layers supplied by the
+ * caller: the fused form, where the caller's own prefill attention kernel
+ * already forms the softmax rows and their column sums are the rules' scores.
+ *   scores[L]  host array of device pointers; for a SnapKV or H2O layer NULL
+ *              (the library scores it from Q_win) or fp32 [B][H_kv][S_cap]:
+ *              raw[k] for k < lens[s] exactly as the layer's rule defines it
+ *              (the group mean of the window rows' softmax weights; every
+ *              prompt row's for H2O with kvev_plan_set_h2o_full_prompt).
+ *              SnapKV's pooling, both rules' selection and H2O's decode seed
+ *              (h2o_state) read it; Q_win[l] is not read for such a layer.
+ *              Entries of other layers are ignored.  4-byte aligned.
+ * Everything else as kvev_evict_prefill.  EINVAL if scores is NULL. */
+KVEV_API int kvev_evict_prefill_scored(kvev_plan *plan, const void *const *K, const void *const *V,
+                                       const void *const *Q_win, const float *const *scores,
+                                       const int32_t *lens_dev, int B, int S_cap, void *out_K,
+                                       void *out_V, int32_t *out_idx, int32_t *out_count,
+                                       float *h2o_state, void *workspace, size_t workspace_bytes,
+                                       void *stream);
+
 /* Sec. 2.1 (H2O's original scoring): with on = 1, the prefill scores of the
  * plan's H2O layers accumulate the attention of every prompt query row,
  *   raw[k] = (1/G) sum_g sum_{t=k}^{n-1} p_{g,t}(k),

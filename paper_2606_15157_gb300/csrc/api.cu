@@ -524,8 +524,9 @@ namespace {
 
 // Argument checks shared by the prefill entry points (no device work).
 int check_prefill_args(const kvev_plan& P, const void* const* K, const void* const* V,
-                       const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap,
-                       void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count) {
+                       const void* const* Q_win, const float* const* scores, const int32_t* lens_dev,
+                       int B, int S_cap, void* out_K, void* out_V, int32_t* out_idx,
+                       int32_t* out_count) {
   if (!K || !V || !lens_dev || !out_count) return KVEV_EINVAL;
   if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
   int64_t total_rows = 0;
@@ -535,8 +536,12 @@ int check_prefill_args(const kvev_plan& P, const void* const* K, const void* con
   for (int l = 0; l < P.L; ++l) {
     if (P.route_pre[l] == KVEV_FULL) continue;
     if (!K[l] || !V[l] || !aligned16(K[l]) || !aligned16(V[l])) return KVEV_EINVAL;
-    if (is_scoring(P.route_pre[l]) && (!Q_win || !Q_win[l] || !aligned16(Q_win[l])))
+    if (!is_scoring(P.route_pre[l])) continue;
+    if (scores && scores[l]) {  // supplied by the caller: Q_win[l] is not read
+      if (reinterpret_cast<uintptr_t>(scores[l]) & 3u) return KVEV_EINVAL;
+    } else if (!Q_win || !Q_win[l] || !aligned16(Q_win[l])) {
       return KVEV_EINVAL;
+    }
   }
   return KVEV_OK;
 }
@@ -545,9 +550,30 @@ int check_prefill_args(const kvev_plan& P, const void* const* K, const void* con
 // a device context (properties + status word) and a scratch workspace of at
 // least ws_layout(P, B, S_cap).total bytes (256-byte aligned).
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
-               const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
-               void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
-               void* workspace, cudaStream_t s);
+               const void* const* Q_win, const float* const* scores, const int32_t* lens_dev, int B,
+               int S_cap, void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count,
+               float* h2o_state, void* workspace, cudaStream_t s);
+
+int evict_prefill_impl(kvev_plan* plan, const void* const* K, const void* const* V,
+                       const void* const* Q_win, const float* const* scores, const int32_t* lens_dev,
+                       int B, int S_cap, void* out_K, void* out_V, int32_t* out_idx,
+                       int32_t* out_count, float* h2o_state, void* workspace, size_t workspace_bytes,
+                       void* stream) {
+  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
+  kvev_plan& P = *plan;
+  if (B == 0) return KVEV_OK;
+  int rc = check_prefill_args(P, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                              out_count);
+  if (rc != KVEV_OK) return rc;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return KVEV_EINVAL;
+  if (workspace_bytes < ws_layout(P, B, S_cap).total) return KVEV_ENOMEM;
+  rc = ensure_device(plan);
+  if (rc != KVEV_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P.last_stream = s;
+  return evict_impl(P, P.ctx, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                    out_count, h2o_state, workspace, s);
+}
 
 }  // namespace
 
@@ -556,19 +582,19 @@ extern "C" int kvev_evict_prefill(kvev_plan* plan, const void* const* K, const v
                                   int S_cap, void* out_K, void* out_V, int32_t* out_idx,
                                   int32_t* out_count, float* h2o_state, void* workspace,
                                   size_t workspace_bytes, void* stream) {
-  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
-  kvev_plan& P = *plan;
-  if (B == 0) return KVEV_OK;
-  int rc = check_prefill_args(P, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count);
-  if (rc != KVEV_OK) return rc;
-  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return KVEV_EINVAL;
-  if (workspace_bytes < ws_layout(P, B, S_cap).total) return KVEV_ENOMEM;
-  rc = ensure_device(plan);
-  if (rc != KVEV_OK) return rc;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  P.last_stream = s;
-  return evict_impl(P, P.ctx, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count,
-                    h2o_state, workspace, s);
+  return evict_prefill_impl(plan, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                            out_count, h2o_state, workspace, workspace_bytes, stream);
+}
+
+extern "C" int kvev_evict_prefill_scored(kvev_plan* plan, const void* const* K, const void* const* V,
+                                         const void* const* Q_win, const float* const* scores,
+                                         const int32_t* lens_dev, int B, int S_cap, void* out_K,
+                                         void* out_V, int32_t* out_idx, int32_t* out_count,
+                                         float* h2o_state, void* workspace, size_t workspace_bytes,
+                                         void* stream) {
+  if (!scores) return KVEV_EINVAL;
+  return evict_prefill_impl(plan, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                            out_count, h2o_state, workspace, workspace_bytes, stream);
 }
 
 namespace {
@@ -599,9 +625,10 @@ int h2o_full_regs_ok(int d) {
 }
 
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
-               const void* const* Q_win, const int32_t* lens_dev, int B, int S_cap, void* out_K,
-               void* out_V, int32_t* out_idx, int32_t* out_count, float* h2o_state,
-               void* workspace, cudaStream_t s) {
+               const void* const* Q_win, const float* const* scores, const int32_t* lens_dev, int B,
+               int S_cap, void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count,
+               float* h2o_state, void* workspace, cudaStream_t s) {
+  auto supplied = [&](int l) { return scores != nullptr && scores[l] != nullptr; };
   if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
   int64_t total_rows = 0;
   for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
@@ -630,6 +657,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   for (int i = 0; i < n_slayers; ++i) {
     pp.slayer_method[i] = P.route_pre[P.score_layers[i]];
     pp.slayer_budget[i] = P.budget[P.score_layers[i]];
+    pp.slayer_ext[i] = supplied(P.score_layers[i]) ? 1 : 0;
   }
   pp.lens_in = lens_dev;
   pp.lens = lens_ok;
@@ -651,7 +679,8 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   };
   pp.W = P.W;
   bool any_h2o = false;
-  for (int i = 0; i < n_slayers; ++i) any_h2o |= P.route_pre[P.score_layers[i]] == KVEV_H2O;
+  for (int i = 0; i < n_slayers; ++i)
+    any_h2o |= P.route_pre[P.score_layers[i]] == KVEV_H2O && !supplied(P.score_layers[i]);
   // H2O prefill scores over every prompt query row: the window kernel scores
   // the SnapKV layers only, and the whole-prompt kernels the H2O layers
   const bool full_prompt = P.h2o_full && any_h2o;
@@ -665,6 +694,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     const int q_rows = ws.R_pad > 128 ? 256 : 128;
     for (int i = 0; i < n_slayers; ++i) {
       const int l = P.score_layers[i];
+      if (supplied(l)) continue;  // not scored here: its maps are never used
       if (!encode_map(&sp.kmap[i], K[l], P.d, static_cast<uint64_t>(B) * P.H_kv * S_cap,
                       kSuperKeys) ||
           !(full_prompt && P.route_pre[l] == KVEV_H2O
@@ -748,7 +778,8 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     fp.R_pad = (fp.R + 31) / 32 * 32;
     fp.n_h2o = 0;
     for (int i = 0; i < n_slayers; ++i)
-      if (P.route_pre[P.score_layers[i]] == KVEV_H2O) fp.h2o_slot[fp.n_h2o++] = i;
+      if (P.route_pre[P.score_layers[i]] == KVEV_H2O && !supplied(P.score_layers[i]))
+        fp.h2o_slot[fp.n_h2o++] = i;
     fp.nb_max = (S_cap + fp.Pb - 1) / fp.Pb;
     fp.nkt_max = (S_cap + kSuperKeys - 1) / kSuperKeys;
     fp.lse = reinterpret_cast<float*>(wsb + ws.lse);
@@ -787,6 +818,11 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     ld.h2o_recent = P.h2o_r[l];
     ld.score_slot = P.score_slot[l];
     ld.row_off = off;
+    ld.scores = nullptr;
+    if (ld.score_slot >= 0)
+      ld.scores = supplied(l) ? scores[l]
+                              : reinterpret_cast<const float*>(wsb + ws.raw) +
+                                    static_cast<size_t>(ld.score_slot) * B * P.H_kv * S_cap;
     off += rows_per_layer(P, B, l);
     sel.layer[l] = ld;
     ga.layer[l] = ld;
@@ -802,7 +838,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.pool_type = P.pool_type;
   sel.sink = P.sink;
   sel.lens = lens_ok;
-  sel.raw = reinterpret_cast<float*>(wsb + ws.raw);
   sel.out_idx = out_idx;
   sel.out_count = out_count;
   // dynamic shared memory of the selection: the unit's keys, then as many
@@ -831,7 +866,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   ga.d = P.d;
   ga.total_rows = total_rows;
   ga.out_idx = out_idx;
-  ga.raw = sel.raw;
   ga.out_K = out_K;
   ga.out_V = out_V;
   ga.h2o_state = h2o_state;
@@ -1121,7 +1155,8 @@ extern "C" int kvev_evict_prefill_noalloc(kvev_plan* plan, const void* const* K,
   if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
   kvev_plan& P = *plan;
   if (B == 0) return KVEV_OK;
-  int rc = check_prefill_args(P, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count);
+  int rc = check_prefill_args(P, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                              out_count);
   if (rc != KVEV_OK) return rc;
   if (ws_layout(P, B, S_cap).total > KVEV_NOALLOC_SCRATCH_BYTES) return KVEV_ENOMEM;
   int dev = 0;
@@ -1144,6 +1179,6 @@ extern "C" int kvev_evict_prefill_noalloc(kvev_plan* plan, const void* const* K,
     if (cudaMemsetAsync(device_status, 0, sizeof(int32_t), s) != cudaSuccess) return KVEV_ECUDA;
     nd.ctx.status = reinterpret_cast<int*>(device_status);
   }
-  return evict_impl(P, nd.ctx, K, V, Q_win, lens_dev, B, S_cap, out_K, out_V, out_idx, out_count,
-                    h2o_state, nd.scratch, s);
+  return evict_impl(P, nd.ctx, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                    out_count, h2o_state, nd.scratch, s);
 }

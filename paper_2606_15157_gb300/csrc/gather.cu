@@ -35,7 +35,6 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const __grid_con
   const int rows_per_block = kGatherThreads / tpr;
   const int sub = threadIdx.x % tpr;
   const long long step = static_cast<long long>(gridDim.x) * rows_per_block;
-  const int per_layer = p.B * p.H_kv;
   for (long long row = static_cast<long long>(blockIdx.x) * rows_per_block + threadIdx.x / tpr;
        row < p.total_rows; row += step) {
     const int l = find_layer(p, row);
@@ -59,7 +58,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const __grid_con
     if (sub == 0 && ld.method == KVEV_H2O && p.h2o_state != nullptr) {
       float a = 0.f;
       if (pos >= 0)
-        a = p.raw[(static_cast<size_t>(ld.score_slot) * per_layer + rem) * p.S_cap + pos];
+        a = ld.scores[static_cast<size_t>(rem) * p.S_cap + pos];
       p.h2o_state[row] = a;
     }
   }

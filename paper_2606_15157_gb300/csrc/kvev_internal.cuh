@@ -57,6 +57,8 @@ struct LayerDesc {
   int h2o_recent;     // H2O protected recent window
   int score_slot;     // index among scoring layers, -1 if none
   long long row_off;  // first packed output row of the layer
+  const float* scores;  // [B*H_kv][S_cap] scores of a scoring layer: its workspace slot, or the
+                        // caller's array when the caller supplies them; null otherwise
 };
 
 struct PrologueParams {
@@ -65,6 +67,7 @@ struct PrologueParams {
   int chunk_keys;
   int slayer_method[kMaxScoreLayers];
   int slayer_budget[kMaxScoreLayers];
+  int slayer_ext[kMaxScoreLayers];  // 1: the caller supplies the layer's scores (not scored here)
   const int* lens_in; // caller's lengths
   int* lens;          // validated copy (out-of-range lengths become 0, flagged)
   int* status;
@@ -117,7 +120,6 @@ struct SelectParams {
   LayerDesc layer[kMaxLayers];
   int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink;
   const int* lens;
-  const float* raw;   // [n_units][S_cap]
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
   int cand_cap;       // candidate positions that fit after the keys in dynamic shared memory
@@ -169,7 +171,6 @@ struct GatherParams {
   int L, B, H_kv, S_cap, d;
   long long total_rows;
   const int* out_idx;
-  const float* raw;
   void* out_K;
   void* out_V;
   float* h2o_state;

@@ -732,7 +732,8 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
       const int n = p.lens[s];
       const bool h2o = p.slayer_method[ls] == KVEV_H2O;
       // H2O layers scored over the whole prompt have their own kernels
-      const bool need = n > 0 && (h2o ? p.mode != kScoreNoH2O : n > p.slayer_budget[ls]);
+      const bool need =
+          n > 0 && !p.slayer_ext[ls] && (h2o ? p.mode != kScoreNoH2O : n > p.slayer_budget[ls]);
       c = need ? (n + p.chunk_keys - 1) / p.chunk_keys : 0;
       p.ready[u] = 0;
     }

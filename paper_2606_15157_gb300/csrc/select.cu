@@ -361,8 +361,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
     for (int j = threadIdx.x; j < E; j += blockDim.x) idx[j] = j;
     return;
   }
-  const float* raw =
-      p.raw + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * static_cast<size_t>(p.S_cap);
+  const float* raw = ld.scores + static_cast<size_t>(rem) * p.S_cap;
   // pull the unit's scores into L2 in 16 KiB pieces (16-byte aligned, whole
   // 16-byte blocks: the score array is one 256-byte aligned workspace region)
   {

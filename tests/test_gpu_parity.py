@@ -226,6 +226,52 @@ def test_maximum_capacity(torch, orc):
     assert rc == kvev.ENOTSUP
 
 
+def test_supplied_scores(torch, orc):
+    # kvev_evict_prefill_scored: the scores of layer 0 (SnapKV) and layer 1 (H2O)
+    # come from the caller -- here the oracle's own window scores rounded to
+    # fp32 -- and their Q_win is not passed; layer 3 (SnapKV) is still scored by
+    # the library.  Pooling, selection, gather and the H2O decode seed must
+    # match the oracle on every unit, as in the scored path.
+    import oracle
+    from paper_2606_15157_gb300 import kvev
+    routes = [gen.SNAPKV, gen.H2O, gen.STREAMING, gen.SNAPKV]
+    wl = _custom(routes, [64, 80, 64, 100], [900, 1500, 17], W=16)
+    dev = device_workload(wl)
+    supplied = (0, 1)
+    specs, meta = [], []
+    for l in range(wl.L):
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            Kh, Vh = parity.to_host_u16(dev[l][0][s]), parity.to_host_u16(dev[l][1][s])
+            Qh = None if dev[l][2] is None else parity.to_host_u16(dev[l][2][s])
+            for h in range(wl.H_kv):
+                spec = parity.oracle_spec(wl, l, s, h, Kh[h][:max(n, 1)],
+                                          None if Qh is None else Qh[h * wl.G:(h + 1) * wl.G])
+                spec["n"] = n
+                specs.append(spec)
+                meta.append((l, s, h, n, Kh[h], Vh[h]))
+    results = oracle.evict_units(specs, d=wl.d, G=wl.G)
+    S = {l: np.zeros((wl.B, wl.H_kv, wl.S_cap), np.float32) for l in supplied}
+    for (l, s, h, n, _, _), res in zip(meta, results):
+        if l in supplied and n > 0:
+            S[l][s, h, :n] = res.raw[:n]
+    plan = kvev.Plan.from_workload(wl)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [None if l in supplied else dev[l][2] for l in range(wl.L)]
+    scores = [torch.from_numpy(S[l]).cuda() if l in supplied else None for l in range(wl.L)]
+    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, scores=scores)
+    torch.cuda.synchronize()
+    assert plan.status() == kvev.OK
+    gpu = parity.GpuRun(plan, wl, bufs, np.asarray(wl.lens))
+    for l in supplied:  # the scores the selection read are the supplied ones
+        gpu.scores[l] = S[l]
+    for (l, s, h, n, Kr, Vr), res in zip(meta, results):
+        parity.check_unit(wl, l, s, h, n, res, gpu, Kr, Vr)
+
+
 def test_repeat_calls_identical(torch):
     wl = gen.config_tiny(1)
     dev = host_to_dev(torch, gen.host_tensors(wl))
