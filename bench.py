@@ -724,7 +724,7 @@ def run_decode(args, rank, world, local_rank):
                          "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                          "traffic": None},
             "clocks": clk.summary(),
-            "gpu_launches": 2 * args.steps,
+            "gpu_launches": args.steps,  # one decode_step_kernel per token (it also advances lens)
             "e2e": None, "cpu_baseline": None,
         }
         print(json.dumps(out), flush=True)

@@ -345,7 +345,8 @@ KVEV_API int kvev_evict_prefill_noalloc(kvev_plan *plan, const void *const *K,
  * evicted[units] (position evicted by the last step, -1 if none), int32
  * pos[rows] (position held by a slot, -1 = empty) and fp32 acc[rows] (H2O:
  * accumulated attention; TOVA: the last step's attention), where unit
- * unit_offset(l) + s*H_kv + h.  Slot order carries no meaning.
+ * unit_offset(l) + s*H_kv + h, and after them an internal step counter.  Slot
+ * order carries no meaning.
  * EINVAL when a layer with a FULL prefill rule has a decode-phase rule (its
  * cache is the caller's own). */
 KVEV_API int kvev_decode_query(const kvev_plan *plan, int B, int growth, int64_t *rows,

@@ -887,7 +887,7 @@ namespace {
 struct DecLayout {
   int units = 0;
   int64_t rows = 0;
-  size_t lens = 0, count = 0, evicted = 0, pos = 0, acc = 0, total = 0;
+  size_t lens = 0, count = 0, evicted = 0, pos = 0, acc = 0, done = 0, total = 0;
   std::vector<int> cap, unit_off;
   std::vector<int64_t> row_off;
 };
@@ -923,6 +923,7 @@ int dec_layout(const kvev_plan& P, int B, int growth, DecLayout& d) {
   d.evicted = take(sizeof(int32_t) * std::max(d.units, 1));
   d.pos = take(sizeof(int32_t) * std::max<int64_t>(d.rows, 1));
   d.acc = take(sizeof(float) * std::max<int64_t>(d.rows, 1));
+  d.done = take(sizeof(int32_t));  // units finished in the current step (internal)
   d.total = off;
   return KVEV_OK;
 }
@@ -981,6 +982,7 @@ void set_state_ptrs(DecodeParams& dp, const DecLayout& d, void* dec_K, void* dec
   dp.evicted = reinterpret_cast<int32_t*>(sb + d.evicted);
   dp.pos = reinterpret_cast<int32_t*>(sb + d.pos);
   dp.acc = reinterpret_cast<float*>(sb + d.acc);
+  dp.done = reinterpret_cast<int32_t*>(sb + d.done);
 }
 
 }  // namespace

@@ -329,10 +329,10 @@ __device__ void stream_unit(const DecodeParams& p, const DecLayer& ly, const Uni
   place_new(p, r, D, ev < c ? ev : -1, n, 0.f, c, evicted_pos);
 }
 
+// The step of unit blockIdx.x (called by the whole block; returns early on
+// an inconsistent state, which it records in the status word).
 template <int D, int G>
-__global__ void __launch_bounds__(kDecodeThreads) decode_step_kernel(const __grid_constant__ DecodeParams p) {
-  extern __shared__ float lg[];
-  __shared__ DecShared sh;
+__device__ __forceinline__ void step_unit(const DecodeParams& p, float* lg, DecShared& sh) {
   const int u = blockIdx.x;
   const int l = find_dec_layer(p, u);
   const DecLayer& ly = p.layer[l];
@@ -355,7 +355,25 @@ __global__ void __launch_bounds__(kDecodeThreads) decode_step_kernel(const __gri
   else if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
 }
 
-// After every unit of the step: the sequences are one token longer.
+template <int D, int G>
+__global__ void __launch_bounds__(kDecodeThreads) decode_step_kernel(const __grid_constant__ DecodeParams p) {
+  extern __shared__ float lg[];
+  __shared__ DecShared sh;
+  step_unit<D, G>(p, lg, sh);
+  // The last unit of the step to finish advances every sequence by one token:
+  // every other CTA has read lens before it counted itself done.
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(p.done, 1) == static_cast<int>(gridDim.x) - 1) {
+      for (int s = 0; s < p.B; ++s) p.lens[s] += 1;
+      *p.done = 0;
+      __threadfence();
+    }
+  }
+}
+
+// A step of a route without decode units: the sequences are one token longer.
 __global__ void decode_advance_kernel(int32_t* lens, int B) {
   for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < B; s += gridDim.x * blockDim.x) lens[s] += 1;
 }
@@ -389,6 +407,7 @@ __global__ void __launch_bounds__(kDecodeThreads) decode_init_kernel(const __gri
   if (threadIdx.x == 0) {
     p.count[u] = c;
     p.evicted[u] = -1;
+    if (u == 0) *p.done = 0;
   }
   if (u == 0)  // the first unit also copies the sequence lengths
     for (int i = threadIdx.x; i < p.B; i += blockDim.x) p.lens[i] = p.lens_in[i];
@@ -430,10 +449,8 @@ cudaError_t launch_decode_init(const DecodeParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_decode_step(const DecodeParams& p, size_t smem, cudaStream_t st) {
-  if (p.units > 0) {
-    const cudaError_t e = p.d == 64 ? launch_step_d<64>(p, smem, st) : launch_step_d<128>(p, smem, st);
-    if (e != cudaSuccess) return e;
-  }
+  if (p.units > 0)  // the step kernel advances lens itself
+    return p.d == 64 ? launch_step_d<64>(p, smem, st) : launch_step_d<128>(p, smem, st);
   decode_advance_kernel<<<1, 256, 0, st>>>(p.lens, p.B);
   return cudaGetLastError();
 }

@@ -154,6 +154,7 @@ struct DecodeParams {
   int32_t* count;     // [units]
   int32_t* evicted;   // [units]: position evicted by the last step, -1 = none
   int32_t* lens;      // [B]
+  int32_t* done;      // units finished in the current step; the last one advances lens
   int* status;
   // initialisation from the packed prefill output
   const void* pre_K;
