@@ -965,12 +965,15 @@ int dec_params(const kvev_plan& P, int B, const DecLayout& d, DecodeParams& dp) 
 }
 
 // Shared memory of the step kernel: the logits of the largest H2O/TOVA unit.
-size_t dec_smem(const kvev_plan& P, const DecLayout& d) {
+// Dynamic shared memory of a decode step: G rows of logits per slot, or one
+// row (the new keys) when the attention is supplied.
+size_t dec_smem(const kvev_plan& P, const DecLayout& d, bool supplied_attention = false) {
   int cap = 0;
   for (int l = 0; l < P.L; ++l)
     if (d.cap[l] > 0 && (P.route_dec[l] == KVEV_H2O || P.route_dec[l] == KVEV_TOVA))
       cap = std::max(cap, d.cap[l]);
-  return cap == 0 ? 0 : sizeof(float) * static_cast<size_t>(P.G) * (cap + 1);
+  const size_t rows = supplied_attention ? 1 : static_cast<size_t>(P.G);
+  return cap == 0 ? 0 : sizeof(float) * rows * (cap + 1);
 }
 
 void set_state_ptrs(DecodeParams& dp, const DecLayout& d, void* dec_K, void* dec_V, void* state) {
@@ -1096,7 +1099,7 @@ int decode_step_impl(kvev_plan* plan, int B, int growth, void* dec_K, void* dec_
   }
   rc = ensure_device(plan);
   if (rc != KVEV_OK) return rc;
-  const size_t smem = dec_smem(P, d);
+  const size_t smem = dec_smem(P, d, attn != nullptr);
   if (smem + 1024 > static_cast<size_t>(P.ctx.smem_optin)) return KVEV_ENOTSUP;
   set_state_ptrs(dp, d, dec_K, dec_V, dec_state);
   dp.status = P.ctx.status;
