@@ -109,3 +109,98 @@ def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens):
         a = plan.scores(bufs, wl.B, wl.S_cap, 1)[s, :, :n]
         b = ref.scores(rbufs, wl.B, wl.S_cap, 1)[s, :, :n]
         assert torch.equal(a, b)
+
+
+def _full_prompt_workload(n, seed):
+    route = [gen.H2O, gen.SNAPKV, gen.H2O]
+    return gen.Workload(name=f"h2o_full_{n}", L=3, H_q=32, H_kv=8, d=128, B=1, lens=np.asarray([n], np.int32),
+                        S_cap=n, W=32, pool_kernel=7, pool_type=gen.POOL_AVG,
+                        route=np.asarray(route, np.int32), budget=np.asarray([512, 512, 768], np.int32),
+                        sink=4, seed=seed, sink_tokens=4, h2o_recent=-1)
+
+
+def _run_full_prompt(torch, wl, rng):
+    from paper_2606_15157_gb300 import kvev
+    dev, q_full = {}, {}
+    for l in range(wl.L):
+        K, V, Qw = gen.device_layer(wl, l, need_q=wl.route[l] == gen.SNAPKV)
+        if wl.route[l] == gen.H2O:
+            qb = _bf16_bits(rng, (wl.B, wl.H_q, wl.S_cap, wl.d))
+            q_full[l] = qb
+            Qw = torch.from_numpy(qb.view(np.int16)).cuda().view(torch.bfloat16)
+        dev[l] = (K, V, Qw)
+    lens_dev = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    plan = kvev.Plan(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel, wl.pool_type,
+                     wl.sink, wl.recent, wl.h2o_recent, h2o_full_prompt=True)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    plan.evict_prefill([dev[l][0] for l in range(wl.L)], [dev[l][1] for l in range(wl.L)],
+                       [dev[l][2] for l in range(wl.L)], lens_dev, wl.B, wl.S_cap, bufs)
+    torch.cuda.synchronize()
+    assert plan.status() == kvev.OK
+    return plan, bufs, dev, q_full, parity.GpuRun(plan, wl, bufs, np.asarray(wl.lens))
+
+
+def test_h2o_full_prompt_8k_properties(torch):
+    # The geometry the full-prompt bench measures (8,192 positions, 32/8 heads,
+    # d = 128: 128 query blocks and 32 key super-tiles per unit).  Two sampled
+    # H2O units against the oracle, and every H2O unit: each query row's softmax sums to 1, so the scores of a KV head
+    # (averaged over its G query heads) sum to n and are positive; the kept
+    # set is the recent window plus the top (b - r) of the unit's own scores
+    # before it (ties to the lower position); the H2O state holds the kept
+    # positions' scores.
+    wl = _full_prompt_workload(8192, 21)
+    n = int(wl.lens[0])
+    plan, bufs, dev, q_full, gpu = _run_full_prompt(torch, wl, np.random.default_rng(8))
+    for l in (0, 2):
+        sc = gpu.scores[l][0].astype(np.float64)
+        np.testing.assert_allclose(sc.sum(axis=1), n, rtol=2e-3)
+        assert (sc[:, :n] > 0).all()
+        b = int(wl.budget[l])
+        r = b // 2
+        for h in range(wl.H_kv):
+            base, _ = gpu.unit_rows(l, 0, h)
+            cnt = int(gpu.count[l, 0, h])
+            kept = gpu.idx[base: base + cnt]
+            assert cnt == b
+            key = gpu.scores[l][0, h, :n - r]
+            order = np.lexsort((np.arange(n - r), -key))  # larger score first, then lower position
+            expect = set(order[:b - r].tolist()) | set(range(n - r, n))
+            assert set(kept.tolist()) == expect
+            np.testing.assert_array_equal(gpu.state[base: base + cnt], gpu.scores[l][0, h, kept])
+    # and two sampled units against the oracle
+    import oracle
+    specs, meta = [], []
+    for (l, h) in ((0, 5), (2, 1)):
+        Kh = parity.to_host_u16(dev[l][0][0])
+        Vh = parity.to_host_u16(dev[l][1][0])
+        spec = parity.oracle_spec(wl, l, 0, h, Kh[h][:n],
+                                  np.ascontiguousarray(q_full[l][0, h * wl.G:(h + 1) * wl.G, :n]))
+        spec["W"] = n
+        spec["n"] = n
+        specs.append(spec)
+        meta.append((l, 0, h, n, Kh[h], Vh[h]))
+    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=2)
+    for (l, s, h, n_, Kr, Vr), res in zip(meta, results):
+        parity.check_unit(wl, l, s, h, n_, res, gpu, Kr, Vr)
+
+
+def test_h2o_full_prompt_2k_oracle(torch):
+    # The same geometry at 2,048 positions (32 query blocks, 8 key super-tiles):
+    # two sampled H2O units against the oracle with the whole prompt as the window.
+    import oracle
+    wl = _full_prompt_workload(2048, 22)
+    n = int(wl.lens[0])
+    plan, bufs, dev, q_full, gpu = _run_full_prompt(torch, wl, np.random.default_rng(9))
+    specs, meta = [], []
+    for (l, h) in ((0, 3), (2, 6)):
+        Kh = parity.to_host_u16(dev[l][0][0])
+        Vh = parity.to_host_u16(dev[l][1][0])
+        spec = parity.oracle_spec(wl, l, 0, h, Kh[h][:n],
+                                  np.ascontiguousarray(q_full[l][0, h * wl.G:(h + 1) * wl.G, :n]))
+        spec["W"] = n
+        spec["n"] = n
+        specs.append(spec)
+        meta.append((l, 0, h, n, Kh[h], Vh[h]))
+    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=2)
+    for (l, s, h, n_, Kr, Vr), res in zip(meta, results):
+        parity.check_unit(wl, l, s, h, n_, res, gpu, Kr, Vr)
