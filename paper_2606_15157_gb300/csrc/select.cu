@@ -15,12 +15,13 @@
 // The k-th largest key is found over an order-preserving uint32 image of the
 // fp32 scores held in shared memory.  The pass that builds the keys also
 // histograms their top 12 bits; the bin holding the k-th key is then the only
-// one that matters: one pass gathers its positions (and counts, per warp
-// segment, the keys above it), two 10-bit radix passes over those candidates
-// alone fix the threshold key, and one ordered pass (ballot/popc prefix
-// counts) writes the kept positions.  Three passes over the unit's keys in
-// all; a first bin too crowded for the candidate buffer takes four 8-bit
-// radix passes over every key instead.
+// one that matters: each warp counts, then gathers in position order, that
+// bin's positions in its segment (counting the keys above it), two 10-bit
+// radix passes over those candidates alone fix the threshold key, and one
+// ordered pass (ballot/popc prefix counts) writes the kept positions.  Four
+// light passes over the unit's keys in all, none through a shared counter; a
+// first bin too crowded for the candidate buffer takes four 8-bit radix
+// passes over every key instead.
 #include "kvev_internal.cuh"
 
 namespace kvev {
@@ -251,35 +252,47 @@ __device__ void count_segments(const uint32_t* keys, int E, uint32_t T, SelShare
 }
 
 // The fast path once the first digit's bin (digit d0, kk-th within it) holds
-// at most `cap` keys: one pass collects that bin's positions into cand[] and
-// counts, per warp segment, the keys of higher bins; the remaining 20 bits are
-// resolved by two 10-bit radix passes over the candidates alone; the
-// candidates then add their own above/equal counts to their segments.
+// at most `cap` keys.  Each warp counts its segment's keys of that bin and of
+// higher bins; a block prefix over the warps gives each warp its own range of
+// cand[], which it fills in position order (no shared counter).  The remaining
+// 20 bits are resolved by two 10-bit radix passes over the candidates alone
+// (their digits are spread out, so plain shared-memory atomics), and each warp
+// then counts its own candidates above and equal to T.
 __device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, int kk, SelShared& sh,
                                      int* cand, uint32_t& T, int& need) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   const uint32_t lt = (1u << lane) - 1u;
-  if (threadIdx.x == 0) sh.ncand = 0;
-  __syncthreads();
-  int gt = 0;
+  int gt = 0, mine = 0;
   for (int b0 = lo; b0 < hi; b0 += 32) {
     const int i = b0 + lane;
     const uint32_t d = i < hi ? keys[i] >> (32 - kHistBits) : 0u;
     gt += __popc(__ballot_sync(0xffffffffu, i < hi && d > d0));
-    const bool in = i < hi && d == d0;
-    const uint32_t b = __ballot_sync(0xffffffffu, in);
-    if (b) {
-      int base = 0;
-      if (lane == __ffs(b) - 1) base = atomicAdd(&sh.ncand, __popc(b));
-      base = __shfl_sync(0xffffffffu, base, __ffs(b) - 1);
-      if (in) cand[base + __popc(b & lt)] = i;
-    }
+    mine += __popc(__ballot_sync(0xffffffffu, i < hi && d == d0));
   }
-  if (lane == 0) {
-    sh.wcnt[0][warp] = gt;
-    sh.wcnt[1][warp] = 0;
+  if (lane == 0) sh.wsum[warp] = mine;
+  __syncthreads();
+  if (warp == 0) {  // exclusive prefix of the per-warp candidate counts
+    const int v = sh.wsum[lane];
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    sh.wsum[lane] = incl - v;
+    if (lane == 31) sh.ncand = incl;
+  }
+  __syncthreads();
+  const int first = sh.wsum[warp];  // this warp's range of cand[]: [first, first + mine)
+  int at = first;
+  for (int b0 = lo; b0 < hi; b0 += 32) {
+    const int i = b0 + lane;
+    const bool in = i < hi && (keys[i] >> (32 - kHistBits)) == d0;
+    const uint32_t b = __ballot_sync(0xffffffffu, in);
+    if (in) cand[at + __popc(b & lt)] = i;
+    at += __popc(b);
   }
   __syncthreads();
   const int nc = sh.ncand;
@@ -287,11 +300,9 @@ __device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, i
   for (int shift = 10; shift >= 0; shift -= 10) {
     for (int i = threadIdx.x; i < 1024; i += kSelectThreads) sh.hist[i] = 0;
     __syncthreads();
-    for (int base = 0; base < nc; base += kSelectThreads) {
-      const int c = base + threadIdx.x;
-      const uint32_t key = c < nc ? keys[cand[c]] : 0u;
-      const bool in = c < nc && (key & mask) == prefix;
-      hist_add(sh.hist, in, (key >> shift) & 1023u);
+    for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
+      const uint32_t key = keys[cand[c]];
+      if ((key & mask) == prefix) atomicAdd(&sh.hist[(key >> shift) & 1023u], 1);
     }
     __syncthreads();
     int digit, above;
@@ -302,10 +313,16 @@ __device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, i
   }
   T = prefix;
   need = kk;
-  for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
-    const int i = cand[c];
-    const uint32_t key = keys[i];
-    if (key >= T) atomicAdd(&sh.wcnt[key > T ? 0 : 1][i / seg], 1);
+  int eq = 0;
+  for (int c0 = 0; c0 < mine; c0 += 32) {
+    const bool v = c0 + lane < mine;
+    const uint32_t key = v ? keys[cand[first + c0 + lane]] : 0u;
+    gt += __popc(__ballot_sync(0xffffffffu, v && key > T));
+    eq += __popc(__ballot_sync(0xffffffffu, v && key == T));
+  }
+  if (lane == 0) {
+    sh.wcnt[0][warp] = gt;
+    sh.wcnt[1][warp] = eq;
   }
   __syncthreads();
 }
