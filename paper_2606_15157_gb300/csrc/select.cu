@@ -93,9 +93,55 @@ __device__ __forceinline__ void build_keys_pooled(uint32_t* keys, int* hist, con
   }
 }
 
+// The same with 16-byte loads, for a 16-byte aligned score row: thread t of a
+// round takes keys 4t .. 4t+3, whose windows (P <= 9) lie in the three
+// aligned 4-float chunks starting at 4t - 4, 4t and 4t + 4.  Only chunks that
+// start before E are read (E <= S_cap, a multiple of 4, so none leaves the
+// row); entries outside [0, E) count as -inf (max) or 0 (avg).
+template <int P>
+__device__ __forceinline__ void build_keys_pooled4(uint32_t* keys, int* hist, const float* raw, int E,
+                                                   bool is_max) {
+  constexpr int h = P / 2;
+  static_assert(h <= 4, "the three chunks cover windows of up to 9");
+  const float fill = is_max ? -INFINITY : 0.f;
+  for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
+    const int i0 = b0 + 4 * threadIdx.x;  // first of this thread's four keys
+    float w[12];
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+      const int st = i0 - 4 + 4 * c;
+      float4 v = make_float4(fill, fill, fill, fill);
+      if (st >= 0 && st < E) v = *reinterpret_cast<const float4*>(raw + st);
+      w[4 * c + 0] = st + 0 < E ? v.x : fill;
+      w[4 * c + 1] = st + 1 < E ? v.y : fill;
+      w[4 * c + 2] = st + 2 < E ? v.z : fill;
+      w[4 * c + 3] = st + 3 < E ? v.w : fill;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u;
+      float v = w[4 + u - h];
+#pragma unroll
+      for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[4 + u - h + j]) : v + w[4 + u - h + j];
+      const uint32_t key = float_key(is_max ? v : v / static_cast<float>(P));
+      if (i < E) keys[i] = key;
+      hist_add(hist, i < E, key >> (32 - kHistBits));
+    }
+  }
+}
+
 __device__ void build_keys(uint32_t* keys, int* hist, const float* raw, int E, int pool, int pool_type,
-                           bool do_pool) {
+                           bool do_pool, bool aligned4) {
   const bool is_max = pool_type == KVEV_POOL_MAX;
+  if (do_pool && aligned4) {
+    switch (pool) {
+      case 3: build_keys_pooled4<3>(keys, hist, raw, E, is_max); return;
+      case 5: build_keys_pooled4<5>(keys, hist, raw, E, is_max); return;
+      case 7: build_keys_pooled4<7>(keys, hist, raw, E, is_max); return;
+      case 9: build_keys_pooled4<9>(keys, hist, raw, E, is_max); return;
+      default: break;
+    }
+  }
   if (do_pool) {
     switch (pool) {  // common widths with fully unrolled windows
       case 3: build_keys_pooled<3>(keys, hist, raw, E, is_max); return;
@@ -389,7 +435,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
   }
   for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
   __syncthreads();
-  build_keys(keys, sh.hist, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV);
+  const bool aligned4 = (reinterpret_cast<uintptr_t>(raw) & 15u) == 0 && (p.S_cap & 3) == 0;
+  build_keys(keys, sh.hist, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV, aligned4);
   __syncthreads();
   int d0, above;
   find_bin(sh, kHistBins, k, d0, above);
