@@ -176,7 +176,8 @@ def kvev_evict_prefill_scored(handle, K_ptrs, V_ptrs, Q_ptrs, score_ptrs, lens_p
     """Pointer-level call with caller-supplied scores; returns the status code."""
     Ln = len(K_ptrs)
     arr = C.c_void_p * Ln
-    Ka, Va, Sa = arr(*K_ptrs), arr(*V_ptrs), arr(*score_ptrs)
+    Ka, Va = arr(*K_ptrs), arr(*V_ptrs)
+    Sa = arr(*score_ptrs) if score_ptrs is not None else None
     Qa = arr(*Q_ptrs) if Q_ptrs is not None else None
     return load().kvev_evict_prefill_scored(handle, Ka, Va, Qa, Sa, lens_ptr, B, S_cap, out_K, out_V,
                                             out_idx, out_count, h2o_state, workspace, workspace_bytes,

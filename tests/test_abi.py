@@ -169,7 +169,32 @@ def test_evict_argument_errors_before_device_work(kv):
     assert kv.kvev_evict_prefill(**dict(args, workspace=fake + 16)) == kv.EINVAL      # 256-B alignment
     assert kv.kvev_evict_prefill(**dict(args, workspace_bytes=64)) == kv.ENOMEM
     assert kv.kvev_evict_prefill(**dict(args, B=0)) == kv.OK                          # nothing to do
+    # caller-supplied scores: the array itself is required; with a layer's scores given, its Q_win
+    # is not, but they must be 4-byte aligned
+    sargs = dict(args, score_ptrs=[None, None])
+    assert kv.kvev_evict_prefill_scored(**dict(sargs, score_ptrs=None)) == kv.EINVAL
+    assert kv.kvev_evict_prefill_scored(**dict(sargs, Q_ptrs=[None, fake])) == kv.EINVAL
+    assert kv.kvev_evict_prefill_scored(**dict(sargs, Q_ptrs=[None, fake], score_ptrs=[fake + 2, None])) == kv.EINVAL
+    assert kv.kvev_evict_prefill_scored(**dict(sargs, Q_ptrs=[None, fake], score_ptrs=[fake, None],
+                                                workspace_bytes=64)) == kv.ENOMEM  # past the checks
     kv.kvev_plan_destroy(h)
+
+
+def test_decode_step_argument_errors(kv):
+    # both decode entry points validate before any device work: the supplied-attention
+    # form needs an attention row array for its H2O / TOVA layers instead of q_new
+    wl = gen.config_decode_mixed()
+    plan = kv.Plan.from_workload(wl)
+    fake = 1 << 20
+    L = wl.L
+    step = dict(handle=plan.handle, B=wl.B, growth=8, dec_K=fake, dec_V=fake, dec_state=fake,
+                k_ptrs=[fake] * L, v_ptrs=[fake] * L, stream=None)
+    assert kv.kvev_decode_step(**step, q_ptrs=[None] * L) == kv.EINVAL
+    assert kv.kvev_decode_step(**dict(step, dec_state=fake + 16), q_ptrs=[fake] * L) == kv.EINVAL
+    assert kv.kvev_decode_step_attn(**step, attn_ptrs=[None] * L) == kv.EINVAL
+    assert kv.kvev_decode_step_attn(**step, attn_ptrs=[fake + 2] * L) == kv.EINVAL
+    assert kv.kvev_decode_step_attn(**dict(step, B=0), attn_ptrs=[fake] * L) == kv.OK
+    plan.close()
 
 
 def test_decode_arena_layout(kv):
