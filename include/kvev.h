@@ -240,10 +240,10 @@ KVEV_API int kvev_plan_scores_offset(const kvev_plan *plan, int B, int S_cap, in
  *   Any rule with b_l >= lens[s] keeps every position.
  * Top-k ties keep the lower position.
  * EINVAL on null/misaligned pointers or B < 0, S_cap < 1; ENOMEM if the
- * workspace is smaller than kvev_plan_query() reports.  ENOTSUP when a
- * plan with SnapKV or H2O layers gets a capacity whose selection does not fit
- * one CTA's shared memory: 4 * S_cap + 18 KiB must not exceed the device's
- * opt-in shared memory per block (S_cap <= 53,504 on a GB300). */
+ * workspace is smaller than kvev_plan_query() reports.  The selection keeps
+ * a unit's keys in shared memory up to S_cap = 53,504 (GB300's opt-in limit
+ * per block); larger capacities keep them in the workspace, which then grows
+ * by 8 bytes per position per (scoring layer, sequence, KV head). */
 KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const *V,
                        const void *const *Q_win, const int32_t *lens_dev, int B, int S_cap,
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,

@@ -60,7 +60,7 @@ bool is_scoring(int m) { return m == KVEV_SNAPKV || m == KVEV_H2O; }
 struct WsLayout {
   int n_units = 0, R = 0, R_pad = 0, max_items = 0, n_h2o_units = 0;
   size_t lens = 0, abort_flag = 0, node_cnt = 0, ready = 0, chunk_start = 0, item = 0, part = 0,
-         lam = 0, raw = 0, lse = 0, total = 0;
+         lam = 0, raw = 0, lse = 0, sel_keys = 0, total = 0;
 };
 
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
@@ -85,6 +85,8 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.part = take(sizeof(float2) * static_cast<size_t>(w.max_items) * w.R_pad);  // one per chunk
   w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
   w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
+  if (S_cap > kSelectSmemCapMax)  // the selection's keys and candidates, per scoring unit
+    w.sel_keys = take(sizeof(uint32_t) * 2 * static_cast<size_t>(w.n_units) * S_cap);
   if (p.h2o_full) {  // base-2 log-sum-exp of every prompt row of every H2O unit
     for (int l : p.score_layers) w.n_h2o_units += p.route_pre[l] == KVEV_H2O ? B * p.H_kv : 0;
     w.lse = take(sizeof(float) * static_cast<size_t>(w.n_h2o_units) * p.G * S_cap);
@@ -843,7 +845,10 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   // dynamic shared memory of the selection: the unit's keys, then as many
   // candidate positions (at most S_cap) as fit next to the static part
   size_t sel_smem = 0;
-  if (ws.n_units > 0) {
+  if (ws.n_units > 0 && S_cap > kSelectSmemCapMax) {
+    sel.keys_g = reinterpret_cast<uint32_t*>(wsb + ws.sel_keys);
+    sel.cand_cap = S_cap;
+  } else if (ws.n_units > 0) {
     const size_t keys_b = sizeof(uint32_t) * static_cast<size_t>(S_cap);
     if (keys_b + kSelectStaticSmem + 1024 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
     const size_t room = static_cast<size_t>(D.smem_optin) - kSelectStaticSmem - 1024 - keys_b;

@@ -43,6 +43,10 @@ constexpr int kRegsSoftmax = 104;
 constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
 constexpr int kSelectThreads = 1024;
 constexpr int kSelectStaticSmem = 17 * 1024;  // bound on the select kernel's static shared memory
+// Largest capacity whose selection keys fit a CTA's shared memory next to the
+// static part (227 KiB opt-in per block on GB300); above it the keys and the
+// candidate positions live in a workspace region instead.
+constexpr int kSelectSmemCapMax = (227 * 1024 - kSelectStaticSmem - 1024) / 4;
 constexpr int kWsAlign = 256;
 
 // Bits of the device status word.
@@ -123,6 +127,8 @@ struct SelectParams {
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
   int cand_cap;       // candidate positions that fit after the keys in dynamic shared memory
+  uint32_t* keys_g;   // capacities above kSelectSmemCapMax: [scoring unit][2][S_cap] keys, then
+                      // candidate positions, in the workspace (null: shared memory)
 };
 
 // Per-layer description of the decode arena.

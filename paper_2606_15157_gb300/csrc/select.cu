@@ -375,8 +375,9 @@ __device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, i
 
 static_assert(sizeof(SelShared) <= kSelectStaticSmem, "select kernel's static shared memory");
 
+template <bool kKeysInWorkspace>
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_constant__ SelectParams p) {
-  extern __shared__ uint32_t keys[];
+  extern __shared__ uint32_t keys_smem[];
   __shared__ SelShared sh;
   const int per_layer = p.B * p.H_kv;
   const int l = blockIdx.x / per_layer;
@@ -425,6 +426,11 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
     return;
   }
   const float* raw = ld.scores + static_cast<size_t>(rem) * p.S_cap;
+  // the unit's keys, then its candidate positions: shared memory, or the
+  // workspace for capacities whose keys do not fit
+  uint32_t* keys = kKeysInWorkspace
+                       ? p.keys_g + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * 2 * p.S_cap
+                       : keys_smem;
   // pull the unit's scores into L2 in 16 KiB pieces (16-byte aligned, whole
   // 16-byte blocks: the score array is one 256-byte aligned workspace region)
   {
@@ -455,13 +461,16 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
 }  // namespace
 
 cudaError_t select_set_smem(size_t smem) {
-  return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(select_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(smem));
 }
 
 cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s) {
   if (grid == 0) return cudaSuccess;
-  select_kernel<<<grid, kSelectThreads, smem, s>>>(p);
+  if (p.keys_g != nullptr)
+    select_kernel<true><<<grid, kSelectThreads, 0, s>>>(p);
+  else
+    select_kernel<false><<<grid, kSelectThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -205,25 +205,14 @@ def test_select_crowded_first_bin(torch, orc):
     parity.check_workload(wl, dev, wl.lens)
 
 
-def test_maximum_capacity(torch, orc):
-    # The largest capacity the selection's shared memory takes (4 * S_cap +
-    # 18 KiB within the opt-in limit per block), with sequences that fill it;
-    # one position more is refused with ENOTSUP.
-    from paper_2606_15157_gb300 import kvev
-    optin = getattr(torch.cuda.get_device_properties(0), "shared_memory_per_block_optin", None)
-    if not optin:
-        pytest.skip("opt-in shared memory size not reported")
-    s_max = (optin - 18 * 1024) // 4
-    wl = _custom([gen.SNAPKV, gen.H2O], [512, 300], [s_max, s_max - 777], W=8, H_q=4, H_kv=2, S_cap=s_max,
-                 d=64)
-    parity.check_workload(wl, device_workload(wl), wl.lens)
-    wl2 = _custom([gen.SNAPKV], [512], [s_max + 1], W=8, H_q=4, H_kv=2, S_cap=s_max + 1, d=64)
-    dev = device_workload(wl2)
-    plan = kvev.Plan.from_workload(wl2)
-    bufs = plan.buffers(wl2.B, wl2.S_cap)
-    lens = torch.from_numpy(np.asarray(wl2.lens, np.int32)).cuda()
-    rc = plan.evict_prefill([dev[0][0]], [dev[0][1]], [dev[0][2]], lens, wl2.B, wl2.S_cap, bufs, check=False)
-    assert rc == kvev.ENOTSUP
+def test_capacity_beyond_shared_memory(torch, orc):
+    # Up to 53,504 positions the selection holds a unit's keys in shared memory;
+    # past it, in the workspace.  Both sides of the bound, with sequences that
+    # fill the capacity, against the oracle.
+    for s_cap in (53504, 65536):
+        wl = _custom([gen.SNAPKV, gen.H2O], [512, 300], [s_cap, s_cap - 777], W=8, H_q=4, H_kv=2,
+                     S_cap=s_cap, d=64)
+        parity.check_workload(wl, device_workload(wl), wl.lens)
 
 
 def test_supplied_scores(torch, orc):
