@@ -45,26 +45,30 @@ __device__ __forceinline__ int find_dec_layer(const DecodeParams& p, int u) {
 struct DecShared {
   float f[kDecodeThreads / 32];
   int i[2 * (kDecodeThreads / 32)];
+  float g[8][kDecodeThreads / 32];  // per-head partials of the G <= 8 query heads
 };
 
-__device__ __forceinline__ float block_max(float v, DecShared& sh) {
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+// Block-wide max (kMax) or sum of G values per thread, all heads in one
+// exchange: warp shuffles, then one shared-memory round.
+template <int G, bool kMax>
+__device__ __forceinline__ void block_reduce_heads(float (&v)[G], DecShared& sh) {
+#pragma unroll
+  for (int g = 0; g < G; ++g)
+    for (int o = 16; o > 0; o >>= 1) {
+      const float y = __shfl_xor_sync(0xffffffffu, v[g], o);
+      v[g] = kMax ? fmaxf(v[g], y) : v[g] + y;
+    }
   __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
+  if ((threadIdx.x & 31) == 0)
+#pragma unroll
+    for (int g = 0; g < G; ++g) sh.g[g][threadIdx.x >> 5] = v[g];
   __syncthreads();
-  float r = sh.f[0];
-  for (int i = 1; i < kDecodeThreads / 32; ++i) r = fmaxf(r, sh.f[i]);
-  return r;
-}
-
-__device__ __forceinline__ float block_sum(float v, DecShared& sh) {
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) sh.f[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float r = 0.f;
-  for (int i = 0; i < kDecodeThreads / 32; ++i) r += sh.f[i];
-  return r;
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float r = sh.g[g][0];
+    for (int w = 1; w < kDecodeThreads / 32; ++w) r = kMax ? fmaxf(r, sh.g[g][w]) : r + sh.g[g][w];
+    v[g] = r;
+  }
 }
 
 // Eviction order: smaller key first, then higher position first.
@@ -240,13 +244,20 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
   for (int g = 0; g < G; ++g) {
     mg[g] = 0.f;
     zg[g] = 1.f;
-    if (at != nullptr) continue;
-    float m = -INFINITY;
-    for (int j = threadIdx.x; j < cnt; j += blockDim.x) m = fmaxf(m, lg[g * ld + j]);
-    mg[g] = block_max(m, sh);
-    float z = 0.f;
-    for (int j = threadIdx.x; j < cnt; j += blockDim.x) z += exp2f(lg[g * ld + j] - mg[g]);
-    zg[g] = block_sum(z, sh);
+  }
+  if (at == nullptr) {
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      mg[g] = -INFINITY;
+      for (int j = threadIdx.x; j < cnt; j += blockDim.x) mg[g] = fmaxf(mg[g], lg[g * ld + j]);
+    }
+    block_reduce_heads<G, true>(mg, sh);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      zg[g] = 0.f;
+      for (int j = threadIdx.x; j < cnt; j += blockDim.x) zg[g] += exp2f(lg[g * ld + j] - mg[g]);
+    }
+    block_reduce_heads<G, false>(zg, sh);
   }
   // group-mean attention -> new keys (each thread overwrites row 0 at its own j only)
   const float* accr = p.acc + r.rows0;
