@@ -391,6 +391,41 @@ def test_h2o_decode_tie_evicts_higher_position(orc):
     assert st.evicted == 3
 
 
+def test_tova_decode_hand_case(orc):
+    # TOVA keeps only the current step's attention (no accumulation) and may
+    # evict the new token itself (no recent window).  q = 8 e0 and k_j = x_j e0
+    # with d = 64 make the logits exactly x_j (8 x_j / sqrt(64)).  Step 1: the
+    # slots hold positions 0,1,2 with x = [1, 0, 2] and the new token (position
+    # 3) has x = 0.5, so p = softmax([1, 0, 2, .5]); the stale acc [9, 9, 9]
+    # must be replaced, and position 1 (x = 0) goes.  Step 2: the new token
+    # (position 4, x = -3) is the least attended and is the one evicted.
+    d, G = 64, 1
+
+    def krow(x):
+        r = np.zeros(d, np.uint16)
+        r[0] = bf16(x)
+        return r
+
+    K = np.stack([krow(1.0), krow(0.0), krow(2.0)])
+    st = orc.DecodeState(orc.TOVA, b=3, cap=6, d=d, n=3, pos=[0, 1, 2], K=K, V=K, acc=[9.0, 9.0, 9.0])
+    q = np.zeros((G, d), np.uint16)
+    q[0, 0] = bf16(8.0)
+    orc.decode_step([st], [krow(0.5)], [krow(0.5)], [q], d, G)
+    x = np.array([1.0, 0.0, 2.0, 0.5])
+    p = np.exp(x - x.max()) / np.exp(x - x.max()).sum()
+    assert st.evicted == 1 and st.count == 3
+    got = dict(zip(st.pos[: st.count].tolist(), st.acc[: st.count].tolist()))
+    assert sorted(got) == [0, 2, 3]
+    assert np.allclose([got[0], got[2], got[3]], p[[0, 2, 3]], rtol=0, atol=1e-12)
+    orc.decode_step([st], [krow(-3.0)], [krow(-3.0)], [q], d, G)
+    x2 = np.array([1.0, 2.0, 0.5, -3.0])
+    p2 = np.exp(x2 - x2.max()) / np.exp(x2 - x2.max()).sum()
+    assert st.evicted == 4 and st.count == 3
+    got = dict(zip(st.pos[: st.count].tolist(), st.acc[: st.count].tolist()))
+    assert sorted(got) == [0, 2, 3]
+    assert np.allclose([got[0], got[2], got[3]], p2[:3], rtol=0, atol=1e-12)
+
+
 def test_streaming_decode_rolls_oldest_non_sink(orc):
     d, G = 64, 1
     pos = [0, 1, 6, 7, 8, 9]
