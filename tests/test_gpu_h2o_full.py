@@ -204,3 +204,43 @@ def test_h2o_full_prompt_2k_oracle(torch):
     results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=2)
     for (l, s, h, n_, Kr, Vr), res in zip(meta, results):
         parity.check_unit(wl, l, s, h, n_, res, gpu, Kr, Vr)
+
+
+def test_full_prompt_with_one_layer_supplied(torch):
+    # A full-prompt plan in which layer 0 (H2O) takes the caller's scores
+    # (kvev_evict_prefill_scored; its Q is not passed) while layer 2 (H2O) is
+    # scored over the whole prompt by the library: layer 0 selects exactly on
+    # the supplied scores, layer 2 matches the plan without supplied scores.
+    from paper_2606_15157_gb300 import kvev
+    wl = _full_prompt_workload(1024, 31)
+    n = int(wl.lens[0])
+    plan, bufs, dev, q_full, gpu = _run_full_prompt(torch, wl, np.random.default_rng(10))
+    rng = np.random.default_rng(11)
+    sup = rng.random((wl.B, wl.H_kv, wl.S_cap)).astype(np.float32)
+    plan2 = kvev.Plan(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel, wl.pool_type,
+                      wl.sink, wl.recent, wl.h2o_recent, h2o_full_prompt=True)
+    bufs2 = plan2.buffers(wl.B, wl.S_cap)
+    lens_dev = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    Q = [None] + [dev[l][2] for l in range(1, wl.L)]
+    scores = [torch.from_numpy(sup).cuda(), None, None]
+    plan2.evict_prefill([dev[l][0] for l in range(wl.L)], [dev[l][1] for l in range(wl.L)], Q, lens_dev,
+                        wl.B, wl.S_cap, bufs2, scores=scores)
+    torch.cuda.synchronize()
+    assert plan2.status() == kvev.OK
+    g2 = parity.GpuRun(plan2, wl, bufs2, np.asarray(wl.lens))
+    b = int(wl.budget[0])
+    r = b // 2
+    for h in range(wl.H_kv):
+        base, _ = g2.unit_rows(0, 0, h)
+        kept = g2.idx[base: base + b]
+        key = sup[0, h, :n - r]
+        order = np.lexsort((np.arange(n - r), -key))
+        assert set(kept.tolist()) == set(order[:b - r].tolist()) | set(range(n - r, n))
+        np.testing.assert_array_equal(g2.state[base: base + b], sup[0, h, kept])
+    # layer 2: the same as in the plan where the library scores both H2O layers
+    assert np.array_equal(g2.scores[2][0, :, :n], gpu.scores[2][0, :, :n])
+    for h in range(wl.H_kv):
+        b2 = int(wl.budget[2])
+        base, _ = g2.unit_rows(2, 0, h)
+        base1, _ = gpu.unit_rows(2, 0, h)
+        assert np.array_equal(g2.idx[base: base + b2], gpu.idx[base1: base1 + b2])
