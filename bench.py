@@ -102,6 +102,8 @@ def h2o_full_flops(wl) -> tuple[int, int]:
 
 
 def workload_bytes(wl):
+    """(algorithmic bytes, score-kernel bytes, evicted rows) of one step over
+    the whole batch; evicted rows count every (sequence, layer, KV head)."""
     tot = sc = ev = 0
     for l in range(wl.L):
         for s in range(wl.B):
@@ -473,7 +475,11 @@ def run_ours(args, rank, world, local_rank):
             "data": "synthetic (seeded; shapes of LLaMA-3.1-8B long-context workloads)",
             "config": workload_config(wl, {"parallelism": f"independent batch per GPU x{world}"}),
             "hbm_frac": {"of_measured": value / hbm_peak, "of_nominal_8TBs": value / NOMINAL_HBM_GBS},
-            "evicted_tokens_per_s": all_evicted / (ms_step / 1e3),
+            # tokens dropped from a layer's cache, counted once per (sequence,
+            # layer) and once per (sequence, layer, KV head): every head keeps
+            # b_l of the n positions, each its own choice
+            "evicted_tokens_per_s": all_evicted / wl.H_kv / (ms_step / 1e3),
+            "evicted_rows_per_s": all_evicted / (ms_step / 1e3),
             "kernel_ms": kernel_ms,
             "roofline": {"kernel": "score_kernel", "bound": "hbm", "achieved": achieved,
                          "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
