@@ -1,6 +1,7 @@
 """Host-side checks of the C ABI (no GPU needed, no kernel launched).
 
-* the shared libraries load and export every symbol include/*.h declares;
+* the shared libraries load and export every symbol include/*.h declares,
+  and the ctypes binding passes each the parameters its prototype lists;
 * the library's allocator equals the oracle's bit for bit;
 * plan validation, byte accounting (App. E worked example) and layer offsets;
 * argument errors are reported before any device work.
@@ -243,3 +244,43 @@ def test_decode_layout_rejects_rules_without_a_retained_cache(kv):
     assert kv.kvev_decode_step(h, 0, 10, fake, fake, fake, [None, fake], [None, fake],
                                [None, fake], None) == kv.OK       # nothing to do
     kv.kvev_plan_destroy(h)
+
+
+def _prototypes(header, macro):
+    """{name: [parameter declarations]} of every function the header declares."""
+    txt = open(os.path.join(ROOT, "include", header)).read()
+    txt = re.sub(r"/\*.*?\*/", " ", txt, flags=re.S)
+    txt = re.sub(r"//[^\n]*", " ", txt)
+    out = {}
+    for m in re.finditer(macro + r"\s+[\w\s\*]*?\b(kvev_\w+)\s*\(([^)]*)\)\s*;", txt):
+        params = [p.strip() for p in m.group(2).split(",") if p.strip()]
+        out[m.group(1)] = [] if params == ["void"] else params
+    return out
+
+
+def _kind(decl):
+    """The ctypes class a C parameter declaration marshals to."""
+    if "*" in decl:
+        return "ptr"
+    t = decl.rsplit(None, 1)[0] if len(decl.split()) > 1 else decl
+    return {"int": "i32", "int32_t": "i32", "int64_t": "i64", "size_t": "size",
+            "double": "f64", "float": "f32"}[t.replace("const ", "").strip()]
+
+
+def test_binding_argtypes_match_header(kv):
+    # every prototype in kvev.h against the ctypes signature the binding
+    # installs: same number of parameters, and each of the same kind (pointer,
+    # 32- or 64-bit integer, size_t, double, float) on both sides
+    protos = _prototypes("kvev.h", "KVEV_API")
+    assert set(protos) == set(kv.EXPORTS)
+    lib = kv.load()
+    ct = {C.c_void_p: "ptr", C.c_int: "i32", C.c_int32: "i32", C.c_int64: "i64", C.c_size_t: "size",
+          C.c_double: "f64", C.c_float: "f32"}
+    for name, params in protos.items():
+        argtypes = getattr(lib, name).argtypes
+        assert argtypes is not None and len(argtypes) == len(params), name
+        for decl, a in zip(params, argtypes):
+            got = "ptr" if (isinstance(a, type) and issubclass(a, C._Pointer)) else ct.get(a)
+            want = _kind(decl)
+            # size_t and int64_t are both 64-bit on the supported (LP64) hosts
+            assert got == want or {got, want} == {"i64", "size"}, (name, decl, a)
