@@ -11,6 +11,8 @@ per-(sequence, layer) definitions and check the workloads' shapes.
     written.
   - Flops: Q_win K^T over the whole group, 2 W H_q n d per sweep, two sweeps,
     on every layer that scores.
+The reference arm (the oracle on the host cores) is run briefly in a
+subprocess: its JSON line, and silence on ranks other than 0.
 """
 import numpy as np
 
@@ -69,3 +71,38 @@ def test_identity_layers_count_every_row():
             assert a * wl.H_kv == 8 * wl.d * wl.H_kv * n and c == 0
             a, c = bench.unit_bytes(wl, l, n + 1)
             assert a * wl.H_kv == _layer_bytes(wl, l, n + 1) and c > 0
+
+
+def _run_bench(args, env_extra):
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, **env_extra)
+    p = subprocess.run([sys.executable, os.path.join(root, "bench.py")] + args, cwd=root, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert p.returncode == 0, p.stderr[-2000:]
+    lines = [ln for ln in p.stdout.splitlines() if ln.startswith("{")]
+    return [json.loads(ln) for ln in lines]
+
+
+def test_reference_arm_prints_the_contract_line():
+    # the reference arm is the oracle on the host cores: one JSON line with the
+    # ours-arm metric, unit and direction, a cpu_baseline record and a zero-copy e2e
+    out = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3", "--ref-units", "2"], {})
+    assert len(out) == 1
+    r = out[0]
+    assert r["impl"] == "reference" and r["metric"] == bench.METRIC and r["unit"] == "GB/s"
+    assert r["higher_is_better"] is True and r["value"] > 0 and r["steps"] == 1 and r["warmup"] == 3
+    assert r["cpu_baseline"]["kind"] == "oracle" and r["cpu_baseline"]["cores"] >= 1
+    assert r["cpu_baseline"]["value"] == r["value"]
+    assert r["e2e"] == {"value": r["value"], "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert r["config"]["workload"] == "long_b8_16k-32k"
+
+
+def test_reference_arm_other_ranks_do_no_work():
+    # under torchrun only rank 0 runs the oracle and prints; the others exit 0
+    out = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3", "--ref-units", "2"],
+                     {"WORLD_SIZE": "2", "RANK": "1", "LOCAL_RANK": "1"})
+    assert out == []
