@@ -75,6 +75,17 @@ def score_flops(wl) -> int:
     return tot
 
 
+def score_exp2(wl) -> int:
+    """exp2 evaluations of the window-score kernel: one per (window row, key)
+    in each sweep (sweep 1 for the row's running sum, sweep 2 for the key's
+    normalised weight), i.e. two per multiply-add column of score_flops."""
+    return score_flops(wl) // (2 * wl.d)
+
+
+# MUFU exp2 rate of one SM: one warp instruction (32 lanes) per clock
+MUFU_EX2_PER_CLK_SM = 32
+
+
 def h2o_full_flops(wl) -> tuple[int, int]:
     """(algorithmic, performed) tensor-core flops of the scoring launches when
     H2O layers score every prompt row.  Algorithmic: each causal q.k product
@@ -410,6 +421,11 @@ def run_ours(args, rank, world, local_rank):
     achieved = score_bytes / (score_ms / 1e3) / 1e9
     tc_peak = float(peaks.get("bf16_tflops", 1900.0))
     tc_achieved = score_flops(wl) / (score_ms / 1e3) / 1e12
+    # MUFU: peak from the unit count and the SM clock sampled under load
+    n_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
+    mhz = clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0
+    mufu_peak = MUFU_EX2_PER_CLK_SM * n_sms * mhz * 1e6 / 1e9
+    mufu_achieved = score_exp2(wl) / (score_ms / 1e3) / 1e9
     kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
     traffic = None
     tf = os.path.join(ROOT, "profiles", "score_traffic.json")
@@ -488,7 +504,12 @@ def run_ours(args, rank, world, local_rank):
                                          "frac": tc_achieved / tc_peak,
                                          "work": "two sweeps of Q_win K^T (bf16 in, fp32 accumulate)",
                                          "peak_source": "measured" if "bf16_tflops" in peaks
-                                         else "fallback"}},
+                                         else "fallback"},
+                         "mufu": {"achieved": mufu_achieved, "peak": mufu_peak, "unit": "Gexp2/s",
+                                  "frac": mufu_achieved / mufu_peak,
+                                  "work": "one exp2 per (window row, key) in each of the two sweeps",
+                                  "peak_source": f"{MUFU_EX2_PER_CLK_SM} exp2/clock/SM x {n_sms} SMs x "
+                                                 f"{mhz:.0f} MHz (median SM clock under load)"}},
             "clocks": clocks,
             "gpu_launches": kernels_launched,
             "e2e": e2e,

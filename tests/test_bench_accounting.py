@@ -10,7 +10,7 @@ per-(sequence, layer) definitions and check the workloads' shapes.
   - A layer whose budget covers the sequence: every row of K and V read and
     written.
   - Flops: Q_win K^T over the whole group, 2 W H_q n d per sweep, two sweeps,
-    on every layer that scores.
+    on every layer that scores; one exp2 per (window row, key) per sweep.
 The reference arm (the oracle on the host cores) is run briefly in a
 subprocess: its JSON line, and silence on ranks other than 0.
 """
@@ -58,6 +58,9 @@ def test_bytes_flops_and_evicted_follow_the_definitions():
     flops = sum(2 * 2 * wl.W * wl.H_q * int(n) * wl.d for l in range(wl.L) for n in wl.lens
                 if wl.route[l] == gen.H2O or (wl.route[l] == gen.SNAPKV and n > wl.budget[l]))
     assert bench.score_flops(wl) == flops
+    exp2 = sum(2 * wl.G * wl.W * int(n) * wl.H_kv for l in range(wl.L) for n in wl.lens
+               if wl.route[l] == gen.H2O or (wl.route[l] == gen.SNAPKV and n > wl.budget[l]))
+    assert bench.score_exp2(wl) == exp2
 
 
 def test_identity_layers_count_every_row():
