@@ -283,7 +283,9 @@ KVEV_API int kvev_plan_set_h2o_full_prompt(kvev_plan *plan, int on);
 
 /* Synchronise the plan's last stream and read-and-clear the device status
  * word: *device_status receives KVEV_OK, KVEV_ETIMEOUT or KVEV_EDEVICE.
- * Returns ECUDA if the readback itself failed. */
+ * Returns ECUDA if the readback itself failed.  Status bits of
+ * kvev_evict_prefill_noalloc() calls go to that call's own device_status
+ * word and are never reported here. */
 KVEV_API int kvev_status(kvev_plan *plan, int *device_status);
 
 /* Bound (in nanoseconds) of every in-kernel wait; a wait that runs out
@@ -314,10 +316,13 @@ KVEV_API int kvev_plan_debug_stall_unit(kvev_plan *plan, int unit);
  *   - The call allocates nothing: no cudaMalloc/cudaFree and no allocating
  *     library routine.  Inputs and outputs are the caller's, as for
  *     kvev_evict_prefill().
- *   - device_status: optional device int32 (NULL allowed) that the call zeroes
- *     on `stream` and in which the kernels record their status bits
- *     (1 = a bounded wait ran out, 2 = an in-kernel check failed).
- *     kvev_status() does not see this entry point's calls.
+ *   - device_status: required device int32 (4-byte aligned; NULL is
+ *     EINVAL) that the call zeroes on `stream` and in which the kernels
+ *     record their status bits (1 = a bounded wait ran out, 2 = an in-kernel
+ *     check failed).  It is the only place these calls report device-side
+ *     errors: read it after the stream's work is done; any non-zero value
+ *     means the outputs of that call are not valid.  kvev_status() never
+ *     reports this entry point's calls.
  *   - The first call on each device looks up the scratch array's device
  *     address for that device (with that device current); make that first
  *     call before any stream capture on the device.

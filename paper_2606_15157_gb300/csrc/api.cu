@@ -1141,7 +1141,6 @@ extern "C" int kvev_decode_step_attn(kvev_plan* plan, int B, int growth, void* d
 namespace {
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[KVEV_NOALLOC_SCRATCH_BYTES];
-static __device__ int g_noalloc_status;  // status word used when the caller passes none
 
 constexpr int kMaxDevices = 64;
 
@@ -1149,7 +1148,6 @@ struct NoallocDevice {
   bool ready = false;
   DevCtx ctx;
   void* scratch = nullptr;  // device address of g_noalloc_scratch on this device
-  int* status = nullptr;    // device address of g_noalloc_status on this device
 };
 
 std::mutex g_noalloc_mu;
@@ -1162,7 +1160,10 @@ extern "C" int kvev_evict_prefill_noalloc(kvev_plan* plan, const void* const* K,
                                           const int32_t* lens_dev, int B, int S_cap, void* out_K,
                                           void* out_V, int32_t* out_idx, int32_t* out_count,
                                           float* h2o_state, int32_t* device_status, void* stream) {
-  if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
+  // The status word is required: the scratch is shared by every call, so the
+  // kernels' status bits can only reach the caller through its own word.
+  if (!plan || B < 0 || S_cap < 1 || !device_status) return KVEV_EINVAL;
+  if (reinterpret_cast<uintptr_t>(device_status) & 3u) return KVEV_EINVAL;
   kvev_plan& P = *plan;
   if (B == 0) return KVEV_OK;
   int rc = check_prefill_args(P, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
@@ -1177,18 +1178,13 @@ extern "C" int kvev_evict_prefill_noalloc(kvev_plan* plan, const void* const* K,
   if (!nd.ready) {  // once per device, with that device current
     rc = query_device(nd.ctx, dev);
     if (rc != KVEV_OK) return rc;
-    if (cudaGetSymbolAddress(&nd.scratch, g_noalloc_scratch) != cudaSuccess ||
-        cudaGetSymbolAddress(reinterpret_cast<void**>(&nd.status), g_noalloc_status) !=
-            cudaSuccess)
-      return KVEV_ECUDA;
+    if (cudaGetSymbolAddress(&nd.scratch, g_noalloc_scratch) != cudaSuccess) return KVEV_ECUDA;
     nd.ready = true;
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  nd.ctx.status = nd.status;
-  if (device_status) {
-    if (cudaMemsetAsync(device_status, 0, sizeof(int32_t), s) != cudaSuccess) return KVEV_ECUDA;
-    nd.ctx.status = reinterpret_cast<int*>(device_status);
-  }
+  if (cudaMemsetAsync(device_status, 0, sizeof(int32_t), s) != cudaSuccess) return KVEV_ECUDA;
+  nd.ctx.status = reinterpret_cast<int*>(device_status);
+  P.last_stream = s;
   return evict_impl(P, nd.ctx, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
                     out_count, h2o_state, nd.scratch, s);
 }

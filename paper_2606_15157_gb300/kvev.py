@@ -341,12 +341,6 @@ def kvev_plan_load(data: bytes) -> int:
     return h.value
 
 
-def alloc_pyramid(L: int, B_total: int, b_min: int) -> np.ndarray:
-    """Pyramidal schedule: weights decreasing linearly with depth (1.5 -> 0.5) fed to Eq. 3."""
-    w = np.ones(1) if L == 1 else 1.5 - np.arange(L) / (L - 1)
-    return kvev_alloc_from_scores(w, B_total, b_min, T_IDENTITY)
-
-
 # ---------------------------------------------------------------------------
 # Convenience: a plan plus its buffers, with torch tensors as device memory
 # ---------------------------------------------------------------------------

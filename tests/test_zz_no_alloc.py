@@ -102,5 +102,81 @@ def test_noalloc_rejects_requests_beyond_its_scratch(env):
     fake = 1 << 20  # never dereferenced: the size check comes before any device work
     ptrs = [fake] * wl.L
     rc = kvev.kvev_evict_prefill_noalloc(plan.handle, ptrs, ptrs, ptrs, fake, wl.B, wl.S_cap, fake,
-                                         fake, fake, fake, fake, None, None)
+                                         fake, fake, fake, fake, fake, None)
     assert rc == kvev.ENOMEM
+
+
+def _tiny_call(torch, kvev, plan, wl, dev, status):
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    b = plan.buffers(wl.B, wl.S_cap)
+    ptr = lambda t: t.data_ptr()
+    rc = kvev.kvev_evict_prefill_noalloc(
+        plan.handle, [ptr(dev[l][0]) for l in range(wl.L)], [ptr(dev[l][1]) for l in range(wl.L)],
+        [ptr(dev[l][2]) for l in range(wl.L)], lens.data_ptr(), wl.B, wl.S_cap,
+        b["out_K"].data_ptr(), b["out_V"].data_ptr(), b["out_idx"].data_ptr(),
+        b["out_count"].data_ptr(), b["h2o_state"].data_ptr(),
+        None if status is None else status.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    return rc, b
+
+
+def _tiny_env(torch):
+    wl = gen.config_tiny(seed=1)
+    host = gen.host_tensors(wl)
+    f = lambda a: torch.from_numpy(a.view(np.int16)).cuda().view(torch.bfloat16)
+    return wl, {l: (f(K), f(V), f(Q)) for l, (K, V, Q) in host.items()}
+
+
+def test_noalloc_requires_a_status_word(env):
+    # The status word is where this call's device-side errors go; without one
+    # they could not be seen, so the call refuses to run.
+    torch, kvev = env
+    wl, dev = _tiny_env(torch)
+    plan = kvev.Plan.from_workload(wl)
+    rc, _ = _tiny_call(torch, kvev, plan, wl, dev, None)
+    assert rc == kvev.EINVAL
+
+
+def test_noalloc_reports_a_wait_that_ran_out(env):
+    # A unit whose normaliser is never published (test hook): the kernels give
+    # up after the plan's short wait limit and record the timeout bit in the
+    # caller's status word, not in the plan's; a clean call then reports 0.
+    torch, kvev = env
+    wl, dev = _tiny_env(torch)
+    plan = kvev.Plan.from_workload(wl)
+    kvev.kvev_plan_set_wait_limit(plan.handle, 20_000_000)  # 20 ms
+    kvev.kvev_plan_debug_stall_unit(plan.handle, 0)
+    status = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    rc, _ = _tiny_call(torch, kvev, plan, wl, dev, status)
+    assert rc == kvev.OK
+    torch.cuda.synchronize()
+    assert int(status.item()) & 1  # the timeout bit
+    assert plan.status() == kvev.OK  # never reported through the plan
+    kvev.kvev_plan_debug_stall_unit(plan.handle, -1)
+    rc, _ = _tiny_call(torch, kvev, plan, wl, dev, status)
+    assert rc == kvev.OK
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+
+
+def test_noalloc_call_allocates_no_device_memory(env):
+    # After a first call (which looks up the scratch address on this device),
+    # a call leaves the device's free memory exactly as it was.
+    torch, kvev = env
+    wl, dev = _tiny_env(torch)
+    plan = kvev.Plan.from_workload(wl)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    b = plan.buffers(wl.B, wl.S_cap)
+    args = ([dev[l][0].data_ptr() for l in range(wl.L)], [dev[l][1].data_ptr() for l in range(wl.L)],
+            [dev[l][2].data_ptr() for l in range(wl.L)], lens.data_ptr(), wl.B, wl.S_cap,
+            b["out_K"].data_ptr(), b["out_V"].data_ptr(), b["out_idx"].data_ptr(),
+            b["out_count"].data_ptr(), b["h2o_state"].data_ptr(), status.data_ptr(),
+            torch.cuda.current_stream().cuda_stream)
+    assert kvev.kvev_evict_prefill_noalloc(plan.handle, *args) == kvev.OK
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(3):
+        assert kvev.kvev_evict_prefill_noalloc(plan.handle, *args) == kvev.OK
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert int(status.item()) == 0
