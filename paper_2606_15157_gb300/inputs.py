@@ -207,8 +207,9 @@ def plant_recipe(seed: int, L: int, n: int, W: int) -> dict:
             st = lo + int(uniform01(seed, T_HOST, 2000 + l) * max(hi - lo, 1))
         else:                # prefix-focused, just after the sink tokens
             st = 4
-        # attention logit gap that puts ~90% of the mass on the planted set
-        gap = math.log(9.0 * (n - s) / s)
+        # attention logit gap that puts ~95% of the mass on the planted set, so
+        # that the smallest set covering 90% of it is most of the planted set
+        gap = math.log(19.0 * (n - s) / s)
         gammas.append(np.float32(gap * math.sqrt(128.0) / 4.0))
         starts.append(st)
         sizes.append(s)
@@ -291,9 +292,13 @@ def config_decode_mixed(seed: int = 0, steps: int = 24, d: int = 128) -> Workloa
 # --------------------------------------------------------------------------
 
 def _unit_u(wl: Workload, layer: int, h: int) -> np.ndarray:
-    """Planted direction of (layer, kv head), ~unit norm: N(0, I/d) in fp32."""
+    """Planted direction of (layer, kv head): a N(0, I) draw scaled to unit norm in fp32.
+    The norm is exact (fsum in double), so every head's planted logit gap is the
+    recipe's gap, not gap * |u|^2 with |u|^2 spread by about +-12% at d = 128."""
     idx = np.arange(h * wl.d, (h + 1) * wl.d, dtype=np.uint64)
-    return gauss_f32(stream_key(wl.seed, T_U, layer), idx) * np.float32(1.0 / math.sqrt(wl.d))
+    x = gauss_f32(stream_key(wl.seed, T_U, layer), idx)
+    norm = math.sqrt(math.fsum(float(v) * float(v) for v in x))
+    return x * np.float32(1.0 / norm)
 
 
 def k_rows(wl: Workload, layer: int, s: int, h: int, pos: np.ndarray) -> np.ndarray:

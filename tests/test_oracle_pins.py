@@ -247,6 +247,33 @@ def test_scores_last_key_seen_only_by_last_row(orc):
     assert abs(raw[n - 1] - p_last / G) < 1e-13
 
 
+def test_scores_matrix_form_tiny_config(orc):
+    # A second restatement of the window scores in matrix form (numpy, float64):
+    # logits = Q K^T / sqrt(d) for all G*W window rows at once, the causal mask
+    # as a boolean matrix, a row softmax over the visible keys, and the column
+    # sums divided by G.  The oracle's per-row loops must agree with it to
+    # 1e-12 on every (layer, KV head) of the tiny config, window keys included.
+    wl = gen.config_tiny(seed=0)
+    n, W, G, d = int(wl.lens[0]), wl.W, wl.G, wl.d
+    pos = np.arange(n, dtype=np.int64)
+    t = n - W + np.arange(W)                       # absolute position of window row i
+    visible = pos[None, :] <= t[:, None]           # [W][n]
+    for l in range(wl.L):
+        for h in range(wl.H_kv):
+            K = gen.k_rows(wl, l, 0, h, pos)
+            Q = gen.q_group(wl, l, 0, h)
+            Kf = gen.bf16_bits_to_f32(K).astype(np.float64)
+            Qf = gen.bf16_bits_to_f32(Q.reshape(G * W, d)).astype(np.float64)
+            S = (Qf @ Kf.T) / math.sqrt(d)                       # [G*W][n]
+            S = np.where(np.tile(visible, (G, 1)), S, -np.inf)
+            P = np.exp(S - S.max(axis=1, keepdims=True))
+            P /= P.sum(axis=1, keepdims=True)
+            ref = P.sum(axis=0) / G
+            raw = orc.window_scores(K, Q, n, W)
+            assert np.allclose(raw, ref, rtol=1e-12, atol=1e-16), (l, h)
+            assert abs(raw.sum() - W) < 1e-9
+
+
 # --------------------------------------------------------------------------
 # Pooling and selection
 # --------------------------------------------------------------------------
