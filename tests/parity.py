@@ -171,23 +171,31 @@ def check_workload(wl, layers_dev, lens_np, units=None, nthreads=0, stats=None):
     gpu = GpuRun(plan, wl, bufs, lens_np)
     if units is None:
         units = [(l, s, h) for l in range(wl.L) for s in range(wl.B) for h in range(wl.H_kv)]
-    specs, meta = [], []
-    cache = {}
-    for (l, s, h) in units:
-        n = int(lens_np[s])
-        if (l, s) not in cache:
-            K, V, Q = layers_dev[l]
-            cache[(l, s)] = (to_host_u16(K[s]), to_host_u16(V[s]),
-                             None if Q is None else to_host_u16(Q[s]))
-        Kh, Vh, Qh = cache[(l, s)]
-        Qg = None if Qh is None else Qh[h * wl.G:(h + 1) * wl.G]
-        spec = oracle_spec(wl, l, s, h, Kh[h][:max(n, 1)], Qg)
-        spec["n"] = n
-        if wl.route[l] == gen.FULL:
-            spec["b"] = max(n, 1)
-        specs.append(spec)
-        meta.append((l, s, h, n, Kh[h], Vh[h]))
-    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=nthreads)
-    for (l, s, h, n, Kr, Vr), res in zip(meta, results):
-        check_unit(wl, l, s, h, n, res, gpu, Kr, Vr, stats)
+    # One oracle call per layer: the host copies of a layer's inputs are freed
+    # before the next layer's (a full-size workload is tens of GB).
+    by_layer = {}
+    for u in units:
+        by_layer.setdefault(u[0], []).append(u)
+    for l in sorted(by_layer):
+        specs, meta = [], []
+        cache = {}
+        for (_, s, h) in by_layer[l]:
+            n = int(lens_np[s])
+            if s not in cache:
+                K, V, Q = layers_dev[l]
+                cache[s] = (to_host_u16(K[s]), to_host_u16(V[s]),
+                            None if Q is None else to_host_u16(Q[s]))
+            Kh, Vh, Qh = cache[s]
+            Qg = None if Qh is None else Qh[h * wl.G:(h + 1) * wl.G]
+            spec = oracle_spec(wl, l, s, h, Kh[h][:max(n, 1)], Qg)
+            spec["n"] = n
+            if wl.route[l] == gen.FULL:
+                spec["b"] = max(n, 1)
+            specs.append(spec)
+            meta.append((l, s, h, n, Kh[h], Vh[h]))
+        results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=nthreads)
+        for (_, s, h, n, Kr, Vr), res in zip(meta, results):
+            check_unit(wl, l, s, h, n, res, gpu, Kr, Vr, stats)
+        if stats is not None:
+            stats["units_checked"] = stats.get("units_checked", 0) + len(meta)
     return plan, bufs, gpu

@@ -300,3 +300,108 @@ def test_decode_full_size_sampled(env):
             assert len(np.unique(p)) == c and p.min() >= 0
             assert int(wl.lens[s]) + step in set(p.tolist()) or md in (kvev.TOVA,)
     assert plan.status() == kvev.OK
+
+
+class SampledArena:
+    """Host copies of a few units of a DecodeArena (the whole arena is several GB)."""
+
+    def __init__(self, torch, arena, wl, units):
+        self.a, self.wl, self.units = arena, wl, units  # units: [(l, s, h, u, r0, cap)]
+        rows = np.concatenate([np.arange(r0, r0 + cap) for (_, _, _, _, r0, cap) in units])
+        self.rows = torch.from_numpy(rows.astype(np.int64)).cuda()
+        self.starts = np.cumsum([0] + [cap for (*_, cap) in units])
+        self.uidx = torch.tensor([u for (_, _, _, u, _, _) in units], dtype=torch.int64).cuda()
+
+    def refresh(self, torch):
+        a = self.a
+        self.K = a.K.view(torch.int16).index_select(0, self.rows).cpu().numpy().view(np.uint16)
+        self.V = a.V.view(torch.int16).index_select(0, self.rows).cpu().numpy().view(np.uint16)
+        self.pos = a.pos().index_select(0, self.rows).cpu().numpy()
+        self.acc = a.acc().index_select(0, self.rows).cpu().numpy()
+        self.count = a.count().index_select(0, self.uidx).cpu().numpy()
+        self.lens = a.lens().cpu().numpy()
+
+    def unit(self, i):
+        c = int(self.count[i])
+        sl = slice(self.starts[i], self.starts[i] + c)
+        return {"count": c, "pos": self.pos[sl], "acc": self.acc[sl].astype(np.float64),
+                "K": self.K[sl], "V": self.V[sl]}
+
+
+def test_decode_all_steps_full_size(env):
+    """The decode workload at its full length: batch 16, 16K caches compacted to
+    2048 slots, 32 layers (H2O, StreamingLLM and append-only decode rules), all
+    256 steps.  Every unit is checked on the device after every step (slot
+    count, unique valid positions, the newest token, the sinks and the recent
+    window of each rule); 32 sampled units (12 H2O, 10 StreamingLLM, 10
+    append-only) are replayed in lock step by the oracle over all 256 steps."""
+    torch, kvev, orc = env
+    wl = gen.config_decode(seed=2)
+    steps = wl.decode_steps
+    assert steps == 256 and wl.B == 16
+    growth = steps
+    plan, bufs, arena = prefill_and_arena(torch, kvev, wl, growth)
+    n0 = int(wl.lens[0])
+    assert np.all(wl.lens == n0)
+    units, layer_info = [], []
+    for l, (off, cap, u0) in enumerate(arena.layers):
+        if cap == 0:
+            continue
+        md, b = int(wl.route_decode[l]), int(wl.budget[l])
+        layer_info.append((l, off, cap, u0, md, b))
+        for s in range(wl.B):
+            for h in range(wl.H_kv):
+                i = s * wl.H_kv + h
+                units.append((l, s, h, u0 + i, off + i * cap, cap))
+    rng = np.random.default_rng(11)
+    want = {kvev.H2O: 12, kvev.STREAMING: 10, kvev.FULL: 10}
+    sample = []
+    for md, k in want.items():
+        idx = [i for i, un in enumerate(units) if int(wl.route_decode[un[0]]) == md]
+        assert len(idx) >= k
+        sample += [units[int(j)] for j in rng.choice(idx, size=k, replace=False)]
+    g = SampledArena(torch, arena, wl, sample)
+    g.refresh(torch)
+    full_like = Arena.__new__(Arena)  # oracle_state reads units / unit() / lens from its argument
+    full_like.units, full_like.unit, full_like.lens = sample, g.unit, g.lens
+    states = [oracle_state(orc, wl, wl.route_decode, full_like, i) for i in range(len(sample))]
+    layers = [li[0] for li in layer_info]
+    exp_count = torch.zeros(arena.units, dtype=torch.int32, device="cuda")
+    ties = 0
+    for step in range(steps):
+        toks, k, v, q = step_tokens(wl, step, layers)
+        arena.step(k, v, q)
+        # lock-step replay of the sampled units
+        kn, vn, qn = host_tokens(torch, toks, wl, range(len(sample)), full_like)
+        orc.decode_step(states, kn, vn, qn, wl.d, wl.G)
+        g.refresh(torch)
+        assert np.all(g.lens == n0 + step + 1)
+        for i, (l, s, h, *_r) in enumerate(sample):
+            if compare_unit(states[i], g.unit(i), f"step {step} layer {l} seq {s} head {h}") == "tie":
+                ties += 1
+                resync(states[i], g.unit(i))
+        # every unit, on the device
+        n = n0 + step + 1
+        pos = arena.pos()
+        for (l, off, cap, u0, md, b) in layer_info:
+            c = b + step + 1 if md == kvev.FULL else b
+            exp_count[u0: u0 + wl.B * wl.H_kv] = c
+            P = torch.sort(pos[off: off + wl.B * wl.H_kv * cap].view(wl.B * wl.H_kv, cap), dim=1)[0]
+            where = f"step {step} layer {l} rule {md}"
+            assert bool((P[:, :cap - c] == -1).all()), where
+            val = P[:, cap - c:]
+            assert bool((val[:, 0] >= 0).all()) and bool((val[:, 1:] > val[:, :-1]).all()), where
+            assert bool((val[:, -1] == n - 1).all()), where  # the newest token is kept
+            ar = lambda lo, hi: torch.arange(lo, hi, dtype=torch.int32, device="cuda")[None, :]
+            if md == kvev.STREAMING:
+                assert bool((val[:, :wl.sink] == ar(0, wl.sink)).all()), where
+                assert bool((val[:, wl.sink:] == ar(n - (c - wl.sink), n)).all()), where
+            elif md == kvev.H2O:
+                r = b // 2
+                assert bool((val[:, c - r:] == ar(n - r, n)).all()), where
+            else:
+                assert bool((val[:, c - (step + 1):] == ar(n0, n)).all()), where
+        assert torch.equal(arena.count(), exp_count), f"step {step}: counts"
+    assert plan.status() == kvev.OK
+    assert ties <= len(sample) * 4
+    print("decode 256 steps: near-tie resyncs", ties)

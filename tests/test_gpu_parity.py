@@ -111,18 +111,20 @@ def _sample_units(wl, k, seed):
     return sorted(set(units))
 
 
-def test_long_context_batch_sampled(torch, orc):
+def test_long_context_batch_every_unit(torch, orc):
     # Full-size headline workload (batch 8, ragged 16K-32K, W=64) in the launch
-    # configuration the benchmark times; the oracle checks sampled units and
-    # every unit is checked against properties that hold at any size.
+    # configuration the benchmark times: every (layer, sequence, KV head) unit
+    # against the oracle (all host cores), plus properties that hold at any size.
+    import oracle
     wl = gen.config_long(kvev_alloc, seed=0)
     wl_o = gen.config_long(oracle_alloc, seed=0)
     assert np.array_equal(wl.budget, wl_o.budget)
     dev = device_workload(wl)
     stats = {}
-    plan, bufs, gpu = parity.check_workload(wl_o, dev, wl.lens, units=_sample_units(wl, 4, 0),
-                                            stats=stats)
-    print("long sampled", stats)
+    plan, bufs, gpu = parity.check_workload(wl_o, dev, wl.lens, stats=stats,
+                                            nthreads=oracle.max_threads())
+    assert stats["units_checked"] == wl.L * wl.B * wl.H_kv
+    print("long, every unit", stats)
     # properties over every unit
     for l in range(wl.L):
         b = int(wl.budget[l])
@@ -147,6 +149,29 @@ def test_long_context_batch_sampled(torch, orc):
         ref = torch.gather(src, 2, idx.unsqueeze(-1).expand(-1, -1, -1, wl.d))
         got = outK[base0: base0 + wl.B * wl.H_kv * b].view(torch.int16).view(wl.B, wl.H_kv, b, wl.d)
         assert torch.equal(ref, got)
+
+
+def test_long_context_fixed_32k_sampled(torch, orc):
+    # The fixed-length variant of the headline (batch 8, every sequence 32,768
+    # tokens): sampled units of every rule against the oracle, and every unit's
+    # kept count and protected window.
+    import oracle
+    wl = gen.config_long(kvev_alloc, seed=0, fixed_len=32768)
+    wl_o = gen.config_long(oracle_alloc, seed=0, fixed_len=32768)
+    assert np.array_equal(wl.budget, wl_o.budget) and np.all(wl.lens == 32768)
+    dev = device_workload(wl)
+    stats = {}
+    plan, bufs, gpu = parity.check_workload(wl_o, dev, wl.lens, units=_sample_units(wl, 6, 1),
+                                            stats=stats, nthreads=oracle.max_threads())
+    print("long fixed 32K, sampled", stats)
+    for l in range(wl.L):
+        b = int(wl.budget[l])
+        assert np.all(gpu.count[l] == min(b, 32768))
+        base0 = plan.layer_offset(wl.B, l)
+        blk = gpu.idx[base0: base0 + wl.B * wl.H_kv * b].reshape(wl.B * wl.H_kv, b)
+        prot = {gen.SNAPKV: wl.W, gen.H2O: b // 2, gen.STREAMING: b - wl.sink}[int(wl.route[l])]
+        assert np.all(blk[:, b - prot:] == np.arange(32768 - prot, 32768)[None, :])
+        assert np.all(np.diff(blk, axis=1) > 0)
 
 
 def _custom(L_routes, budgets, lens, W=16, d=128, H_q=8, H_kv=2, S_cap=None, pool=(5, gen.POOL_MAX),
