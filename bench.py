@@ -16,6 +16,7 @@ no collective on the data path; rank 0 prints one JSON line.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import hashlib
 import json
 import os
@@ -341,6 +342,62 @@ def rank_reducers(dist: bool, device: str):
     return (lambda x: red(x, td.ReduceOp.MAX)), (lambda x: red(x, td.ReduceOp.SUM))
 
 
+def time_prefill(plan, wl, K, V, Q, lens, bufs, stream, steps, barrier, kvev):
+    """Device time of `steps` back-to-back prefill evictions (inputs resident in
+    HBM): (ms per step, per-kernel mean ms, clock summary, kernels launched)."""
+    import torch
+    kvev.kvev_plan_enable_timing(plan.handle, True)
+    per_kernel = {k: [] for k in kvev.KERNEL_NAMES}
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        barrier()
+        ev0.record(stream)
+        for _ in range(steps):
+            plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
+            for k, v in kvev.kvev_plan_last_timings(plan.handle).items():
+                if v >= 0:
+                    per_kernel[k].append(v)
+        ev1.record(stream)
+        barrier()
+    launched = sum(len(v) for v in per_kernel.values())
+    means = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
+    return ev0.elapsed_time(ev1) / steps, means, clk.summary(), launched
+
+
+def cudart():
+    """The CUDA runtime that torch loaded (the same library instance, so torch's
+    stream handles are valid in calls made through it)."""
+    paths = []
+    try:
+        paths = [ln.split()[-1] for ln in open("/proc/self/maps") if "libcudart.so" in ln]
+    except OSError:
+        pass
+    lib = ctypes.CDLL(paths[0] if paths else "libcudart.so")
+    vp, sz = ctypes.c_void_p, ctypes.c_size_t
+    lib.cudaMemcpy2DAsync.argtypes = [vp, sz, vp, sz, sz, sz, ctypes.c_int, vp]
+    lib.cudaMemcpy2DAsync.restype = ctypes.c_int
+    return lib
+
+
+def host_link_peak(nbytes: int = 2 << 30, reps: int = 5) -> dict:
+    """Host -> device copy rate of one large pinned buffer (cudaMemcpyAsync)."""
+    import torch
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    d = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    d.copy_(h, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        d.copy_(h, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    gbs = reps * nbytes / (e0.elapsed_time(e1) / 1e3) / 1e9
+    del h, d
+    return {"h2d_gbs": gbs, "how": f"one pinned {nbytes >> 30} GiB host buffer copied to the device, "
+                                   f"{reps} times, CUDA events"}
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     from paper_2606_15157_gb300 import kvev
@@ -387,24 +444,11 @@ def run_ours(args, rank, world, local_rank):
     for _ in range(args.warmup):
         plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
     barrier()
-    per_kernel = {k: [] for k in kvev.KERNEL_NAMES}
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local_rank) as clk:
-        barrier()
-        ev0.record(stream)
-        for _ in range(args.steps):
-            plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
-            for k, v in kvev.kvev_plan_last_timings(plan.handle).items():
-                if v >= 0:
-                    per_kernel[k].append(v)
-        ev1.record(stream)
-        barrier()
-    ms_total = ev0.elapsed_time(ev1)
-    ms_step = max_over_ranks(ms_total / args.steps)
+    ms_local, kernel_ms, clocks, kernels_launched = time_prefill(plan, wl, K, V, Q, lens, bufs, stream,
+                                                                  args.steps, barrier, kvev)
+    ms_step = max_over_ranks(ms_local)
     status = plan.status()
     assert status == kvev.OK, f"device status {status}"
-    clocks = clk.summary()
-    kernels_launched = sum(len(v) for v in per_kernel.values())
     all_bytes = sum_over_ranks(float(tot_bytes))
     all_evicted = sum_over_ranks(float(evicted))
     value = all_bytes / (ms_step / 1e3) / 1e9
@@ -417,7 +461,7 @@ def run_ours(args, rank, world, local_rank):
         pass
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
-    score_ms = statistics.mean(per_kernel["score"]) if per_kernel["score"] else float("nan")
+    score_ms = kernel_ms["score"] if kernel_ms["score"] is not None else float("nan")
     achieved = score_bytes / (score_ms / 1e3) / 1e9
     tc_peak = float(peaks.get("bf16_tflops", 1900.0))
     tc_achieved = score_flops(wl) / (score_ms / 1e3) / 1e12
@@ -426,7 +470,6 @@ def run_ours(args, rank, world, local_rank):
     mhz = clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0
     mufu_peak = MUFU_EX2_PER_CLK_SM * n_sms * mhz * 1e6 / 1e9
     mufu_achieved = score_exp2(wl) / (score_ms / 1e3) / 1e9
-    kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
     traffic = None
     tf = os.path.join(ROOT, "profiles", "score_traffic.json")
     if os.path.exists(tf):
@@ -459,6 +502,34 @@ def run_ours(args, rank, world, local_rank):
         cpu = {"value": nb / secs / 1e9, "unit": "GB/s", "cores": cores, "kind": "oracle",
                "sample": f"{len(units)} (sequence, layer, KV-head) units of the workload, "
                          f"route mix kept, {secs:.1f} s of oracle time"}
+
+    # ---- sustained: the same step over at least 0.5 s of device time ----
+    sustained = None
+    if not args.no_extras and not args.h2o_full_prompt:
+        n_s = max(args.steps, int(np.ceil(500.0 / max(ms_step, 1e-3))))
+        ms_s, _, clk_s, _ = time_prefill(plan, wl, K, V, Q, lens, bufs, stream, n_s, barrier, kvev)
+        ms_s = max_over_ranks(ms_s)
+        assert plan.status() == kvev.OK
+        sustained = {"value": all_bytes / (ms_s / 1e3) / 1e9, "unit": "GB/s", "ms_per_step": ms_s,
+                     "steps": n_s, "device_seconds": n_s * ms_s / 1e3, "clocks": clk_s}
+
+    extras = {}
+    if not args.no_extras and not args.h2o_full_prompt and args.workload == "long" and not args.batch:
+        del dev, K, V, Q, bufs
+        plan.close()
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        extras["long32k"] = fixed_length_variant(args, rank, kvev, barrier, max_over_ranks, sum_over_ranks)
+        torch.cuda.empty_cache()
+        extras["decode"] = decode_measure(args, rank, world, local_rank, B=16, steps=max(args.steps, 50),
+                                          warmup=args.warmup, attn_supplied=False)
+        torch.cuda.empty_cache()
+    if not args.no_extras and not args.h2o_full_prompt:
+        extras["host_link"] = host_link_peak()
+        if e2e is not None:
+            link = e2e["h2d_bytes_per_step"] / (e2e["ms_per_step"] / 1e3) / 1e9
+            e2e["host_link_gbs"] = link
+            e2e["host_link_frac"] = link / extras["host_link"]["h2d_gbs"]
 
     if rank == 0 and args.h2o_full_prompt:
         alg, perf = h2o_full_flops(wl)
@@ -514,8 +585,54 @@ def run_ours(args, rank, world, local_rank):
             "gpu_launches": kernels_launched,
             "e2e": e2e,
             "cpu_baseline": cpu,
+            "sustained": sustained,
         }
+        out.update(extras)
         print(json.dumps(out), flush=True)
+
+
+def fixed_length_variant(args, rank, kvev, barrier, max_over_ranks, sum_over_ranks):
+    """The headline's fixed-length variant: batch 8, every sequence 32,768
+    tokens, same route and allocation; device-resident inputs, same timing."""
+    import torch
+    wl = make_workload("long32k", rank, kvev.alloc_from_scores)
+    tot_bytes, score_bytes, evicted = workload_bytes(wl)
+    need_q = lambda l: wl.route[l] in (gen.SNAPKV, gen.H2O)
+    dev = {l: gen.device_layer(wl, l, need_q=need_q(l)) for l in range(wl.L)}
+    plan = kvev.Plan.from_workload(wl)
+    bufs = plan.buffers(wl.B, wl.S_cap)
+    lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
+    K = [dev[l][0] for l in range(wl.L)]
+    V = [dev[l][1] for l in range(wl.L)]
+    Q = [dev[l][2] for l in range(wl.L)]
+    stream = torch.cuda.current_stream()
+    kvev.kvev_plan_enable_timing(plan.handle, True)
+    for _ in range(args.warmup):
+        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
+    barrier()
+    steps = max(10, min(args.steps, 40))
+    ms, kms, clk, _ = time_prefill(plan, wl, K, V, Q, lens, bufs, stream, steps, barrier, kvev)
+    ms = max_over_ranks(ms)
+    assert plan.status() == kvev.OK
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    value = sum_over_ranks(float(tot_bytes)) / (ms / 1e3) / 1e9
+    ach = score_bytes / (kms["score"] / 1e3) / 1e9
+    out = {"workload": wl.name, "value": value, "unit": "GB/s", "ms_per_step": ms, "steps": steps,
+           "hbm_frac": {"of_measured": value / hbm_peak, "of_nominal_8TBs": value / NOMINAL_HBM_GBS},
+           "evicted_tokens_per_s": sum_over_ranks(float(evicted)) / wl.H_kv / (ms / 1e3),
+           "kernel_ms": kms,
+           "roofline": {"kernel": "score_kernel", "bound": "hbm", "achieved": ach, "peak": hbm_peak,
+                        "unit": "GB/s", "frac": ach / hbm_peak, "traffic": None},
+           "clocks": clk}
+    del dev, K, V, Q, bufs
+    plan.close()
+    torch.cuda.synchronize()
+    return out
 
 
 def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_ranks,
@@ -534,6 +651,8 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
     from paper_2606_15157_gb300 import kvev
     scoring = [int(wl.route[l]) in (gen.SNAPKV, gen.H2O) for l in range(wl.L)]
     pinned = lambda t: None if t is None else torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t)
+    rt = cudart()
+    H2D = 1  # cudaMemcpyHostToDevice
     V_arg = []
     K_set, Q_set, copy_set = [[], []], [[], []], [[], []]
     for l in range(wl.L):
@@ -546,13 +665,16 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
                 Qb = Qd if b == 0 else torch.empty_like(Qd)
                 K_set[b].append(Kb)
                 Q_set[b].append(Qb)
-                # the prompt rows of each (sequence, KV head): a contiguous slice of
-                # [B][H_kv][S_cap][d]; rows past a sequence's length are never read
+                # the prompt rows of a sequence's KV heads: H_kv blocks of n rows,
+                # S_cap rows apart in [B][H_kv][S_cap][d], as one 2-D copy (rows
+                # past a sequence's length are never read)
+                pitch = wl.S_cap * wl.d * Kh.element_size()
                 for s in range(wl.B):
                     n = int(wl.lens[s])
                     if n > 0:
-                        copy_set[b] += [(Kh[s, h, :n], Kb[s, h, :n]) for h in range(wl.H_kv)]
-                copy_set[b].append((Qh, Qb))
+                        copy_set[b].append(("2d", Kb[s].data_ptr(), Kh[s].data_ptr(), pitch,
+                                            n * wl.d * Kh.element_size(), wl.H_kv))
+                copy_set[b].append(("1d", Qh, Qb))
             else:
                 K_set[b].append(Kh)
                 Q_set[b].append(None)
@@ -560,7 +682,8 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
     bufs = plan.buffers(wl.B, wl.S_cap)
     idx_h = torch.empty(bufs["out_idx"].shape, dtype=torch.int32, pin_memory=True)
     cnt_h = torch.empty(bufs["out_count"].shape, dtype=torch.int32, pin_memory=True)
-    copied = sum(h.numel() * h.element_size() for h, _ in copy_set[0]) + lens_h.numel() * 4
+    copied = sum(c[4] * c[5] if c[0] == "2d" else c[1].numel() * c[1].element_size()
+                 for c in copy_set[0]) + lens_h.numel() * 4
     d2h = idx_h.numel() * 4 + cnt_h.numel() * 4
     copy_streams = [torch.cuda.Stream() for _ in range(4)]
     released = [torch.cuda.Event(), torch.cuda.Event()]  # last eviction that read input set b is done
@@ -575,8 +698,13 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
         for i, cs in enumerate(copy_streams):
             cs.wait_event(released[b])
             with torch.cuda.stream(cs):
-                for h, d in copy_set[b][i::len(copy_streams)]:
-                    d.copy_(h, non_blocking=True)
+                for c in copy_set[b][i::len(copy_streams)]:
+                    if c[0] == "2d":
+                        _, dst, src, pitch, width, height = c
+                        rc = rt.cudaMemcpy2DAsync(dst, pitch, src, pitch, width, height, H2D, cs.cuda_stream)
+                        assert rc == 0, f"cudaMemcpy2DAsync failed ({rc})"
+                    else:
+                        c[2].copy_(c[1], non_blocking=True)
             ev = torch.cuda.Event()
             ev.record(cs)
             evs.append(ev)
@@ -621,6 +749,7 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
             "h2d_bytes_per_step": int(copied + host_read), "d2h_bytes_per_step": int(d2h),
             "ms_per_step": ms, "steps": n,
             "host_resident": "V of every layer and K of the StreamingLLM layers, read in place",
+            "copies_per_step": len(copy_set[0]) + 3,
             "pipelining": "two device copies of the streamed inputs; uploads overlap the previous step"}
 
 
@@ -650,6 +779,14 @@ def decode_step_bytes(wl, counts, supplied_attention=False):
 def run_decode(args, rank, world, local_rank):
     """Decode workload: batch 16, 16K-token caches compacted to 2048 slots by the
     prefill eviction (not timed), then one kvev_decode_step per generated token."""
+    out = decode_measure(args, rank, world, local_rank, B=args.batch or 16, steps=args.steps,
+                         warmup=args.warmup, attn_supplied=args.decode_attn)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def decode_measure(args, rank, world, local_rank, B, steps, warmup, attn_supplied):
+    """The decode step's JSON record (see run_decode)."""
     import torch
     from paper_2606_15157_gb300 import kvev
 
@@ -657,8 +794,8 @@ def run_decode(args, rank, world, local_rank):
     dist = world > 1
     if dist:
         import torch.distributed as td
-    wl = gen.config_decode(seed=rank, B=args.batch or 16)
-    total = args.warmup + args.steps
+    wl = gen.config_decode(seed=rank, B=B)
+    total = warmup + steps
     growth = total
     plan = kvev.Plan.from_workload(wl)
     lens = torch.from_numpy(np.asarray(wl.lens, np.int32)).cuda()
@@ -675,10 +812,10 @@ def run_decode(args, rank, world, local_rank):
     toks = [[gen.device_decode_tokens(wl, t, l) for l in range(wl.L)] for t in range(total)]
     torch.cuda.synchronize()
     counts = [int(wl.budget[l]) for l in range(wl.L)]
-    step_bytes = decode_step_bytes(wl, counts, args.decode_attn)
+    step_bytes = decode_step_bytes(wl, counts, attn_supplied)
     stream = torch.cuda.current_stream()
     attn = None
-    if args.decode_attn:
+    if attn_supplied:
         # the caller's decode attention would supply these every step; any valid
         # rows cost the same, so one seeded set of distributions is reused
         g = torch.Generator(device="cuda")
@@ -700,25 +837,25 @@ def run_decode(args, rank, world, local_rank):
         q = [x[2] for x in toks[t]]
         arena.step(k, v, q, stream)
 
-    for t in range(args.warmup):
+    for t in range(warmup):
         run(t)
     if dist:
         td.barrier()
     torch.cuda.synchronize()
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
     with ClockSampler(local_rank) as clk:
         if dist:
             td.barrier()
         torch.cuda.synchronize()
         evs[0].record(stream)
-        for i in range(args.steps):
-            run(args.warmup + i)
+        for i in range(steps):
+            run(warmup + i)
             evs[i + 1].record(stream)
         torch.cuda.synchronize()
         if dist:
             td.barrier()
-    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
-    ms = evs[0].elapsed_time(evs[-1]) / args.steps
+    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(steps)]
+    ms = evs[0].elapsed_time(evs[-1]) / steps
     max_over_ranks, sum_over_ranks = rank_reducers(dist, "cuda")
     ms = max_over_ranks(ms)
     all_bytes = sum_over_ranks(float(step_bytes))
@@ -731,15 +868,18 @@ def run_decode(args, rank, world, local_rank):
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     value = all_bytes / (ms / 1e3) / 1e9
     achieved = step_bytes / (statistics.median(per) / 1e3) / 1e9
-    if rank == 0:
+    del toks, arena, bufs
+    plan.close()
+    torch.cuda.synchronize()
+    if True:
         out = {
             "metric": "KV decode-step GB/s (retained-cache update per generated token)",
-            "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "value": value, "unit": "GB/s", "n_gpus": world, "steps": steps,
+            "warmup": warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded; shapes of LLaMA-3.1-8B decode with compacted caches)",
             "config": {"workload": wl.name, "layers": wl.L, "batch": wl.B, "cache_slots": 2048,
-                       "attention": "supplied by the caller (kvev_decode_step_attn)" if args.decode_attn
+                       "attention": "supplied by the caller (kvev_decode_step_attn)" if attn_supplied
                        else "computed from q_new and the retained K",
                        "route_decode": {"h2o": int((wl.route_decode == gen.H2O).sum()),
                                         "streaming": int((wl.route_decode == gen.STREAMING).sum()),
@@ -752,10 +892,10 @@ def run_decode(args, rank, world, local_rank):
                          "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                          "traffic": None},
             "clocks": clk.summary(),
-            "gpu_launches": args.steps,  # one decode_step_kernel per token (it also advances lens)
+            "gpu_launches": steps,  # one decode_step_kernel per token (it also advances lens)
             "e2e": None, "cpu_baseline": None,
         }
-        print(json.dumps(out), flush=True)
+    return out
 
 
 def main():
@@ -778,6 +918,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-units", type=int, default=16)
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the sustained run, the fixed-32K variant, the decode step and the "
+                         "host-link peak (profiling runs)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
