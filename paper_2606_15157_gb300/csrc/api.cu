@@ -956,6 +956,12 @@ int dec_params(const kvev_plan& P, int B, const DecLayout& d, DecodeParams& dp) 
     y.pre_slots = P.slots[l];
     y.pre_row_off = pre_off;
     pre_off += rows_per_layer(P, B, l);
+    if (y.cap > 0 && (md == KVEV_H2O || md == KVEV_TOVA))
+      dp.n_att += B * P.H_kv;
+    else if (y.cap > 0)
+      dp.n_cheap += B * P.H_kv;
+    y.att_end = dp.n_att;
+    y.cheap_end = dp.n_cheap;
     if (y.cap == 0) continue;
     if (md == KVEV_H2O || md == KVEV_TOVA) {
       y.r = md == KVEV_TOVA ? 0 : (P.h2o_recent < 0 ? b / 2 : P.h2o_recent);

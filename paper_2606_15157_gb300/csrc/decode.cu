@@ -12,7 +12,8 @@
 // the last step's attention).  Slot order carries no meaning: an evicted
 // slot is overwritten by the new token.
 //
-// One CTA per unit.  H2O / TOVA: the G query rows of the new token attend to
+// One CTA per H2O / TOVA unit, and one warp per StreamingLLM or append-only
+// unit (eight per CTA).  H2O / TOVA: the G query rows of the new token attend to
 // every retained slot and to the new token, p_j = (1/G) sum_g softmax_j(q_g .
 // k_j / sqrt(d)); acc += p (H2O) or acc = p (TOVA).  When the unit already
 // holds b slots, the slot with the smallest acc among positions older than
@@ -255,9 +256,15 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       zg[g] = 0.f;
-      for (int j = threadIdx.x; j < cnt; j += blockDim.x) zg[g] += exp2f(lg[g * ld + j] - mg[g]);
+      for (int j = threadIdx.x; j < cnt; j += blockDim.x) {  // each thread keeps its own exponentials
+        const float e = exp2f(lg[g * ld + j] - mg[g]);
+        lg[g * ld + j] = e;
+        zg[g] += e;
+      }
     }
     block_reduce_heads<G, false>(zg, sh);
+#pragma unroll
+    for (int g = 0; g < G; ++g) zg[g] = 1.0f / (static_cast<float>(G) * zg[g]);
   }
   // group-mean attention -> new keys (each thread overwrites row 0 at its own j only)
   const float* accr = p.acc + r.rows0;
@@ -265,22 +272,35 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
   const int limit = n + 1 - ly.r;  // positions >= limit are protected
   float ba = INFINITY;
   int bp = -1, bs = -1;
-  for (int j = threadIdx.x; j < cnt; j += blockDim.x) {
-    float pj = 0.f;
-    if (at != nullptr) {
-      pj = at[j];
-    } else {
+  constexpr int kU = 4;  // slots per thread whose global loads are issued together
+  for (int j0 = threadIdx.x; j0 < cnt; j0 += kU * kDecodeThreads) {
+    float accv[kU], atv[kU];
+    int posv[kU];
 #pragma unroll
-      for (int g = 0; g < G; ++g) pj += exp2f(lg[g * ld + j] - mg[g]) / zg[g];
-      pj *= 1.0f / static_cast<float>(G);
+    for (int q = 0; q < kU; ++q) {
+      const int j = j0 + q * kDecodeThreads;
+      accv[q] = (ly.method == KVEV_H2O && j < c) ? accr[j] : 0.f;
+      posv[q] = j < c ? posr[j] : n;
+      atv[q] = (at != nullptr && j < cnt) ? at[j] : 0.f;
     }
-    const float a = (ly.method == KVEV_H2O && j < c) ? accr[j] + pj : pj;
-    lg[j] = a;
-    const int pos = j < c ? posr[j] : n;
-    if (pos >= 0 && pos < limit && (bp < 0 || evict_before(a, pos, ba, bp))) {
-      ba = a;
-      bp = pos;
-      bs = j;
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int j = j0 + q * kDecodeThreads;
+      if (j >= cnt) break;
+      float pj = atv[q];
+      if (at == nullptr) {  // group mean of the kept exponentials times 1 / (G z_g)
+        pj = 0.f;
+#pragma unroll
+        for (int g = 0; g < G; ++g) pj += lg[g * ld + j] * zg[g];
+      }
+      const float a = accv[q] + pj;
+      lg[j] = a;
+      const int pos = posv[q];
+      if (pos >= 0 && pos < limit && (bp < 0 || evict_before(a, pos, ba, bp))) {
+        ba = a;
+        bp = pos;
+        bs = j;
+      }
     }
   }
   const bool full = c >= ly.b;
@@ -303,75 +323,132 @@ __device__ void attend_unit(const DecodeParams& p, const DecLayer& ly, const Uni
   }
 }
 
-// StreamingLLM unit: the oldest non-sink slot makes room once sink + recent
-// slots are held; positions are read from the state, no attention.
-__device__ void stream_unit(const DecodeParams& p, const DecLayer& ly, const UnitRef& r, int D, int n, int c,
-                            DecShared& sh) {
-  const int capacity = ly.sink + ly.recent;
-  if (c + 1 <= capacity) {
-    if (c >= ly.cap) {
-      if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
-      return;
-    }
-    place_new(p, r, D, c, n, 0.f, c + 1, -1);
-    return;
+constexpr int kDecodeWarps = kDecodeThreads / 32;
+
+// The first layer whose prefix end (att_end or cheap_end) exceeds i: the
+// layer holding the i-th unit of that kind.
+template <bool kAttend>
+__device__ __forceinline__ int find_kind_layer(const DecodeParams& p, int i) {
+  int lo = 0, hi = p.L - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if ((kAttend ? p.layer[mid].att_end : p.layer[mid].cheap_end) > i) hi = mid;
+    else lo = mid + 1;
   }
-  // smallest position >= sink among the slots and the new token (eviction key = position)
-  float ba = INFINITY;
-  int bp = -1, bs = -1;
-  for (int j = threadIdx.x; j <= c; j += blockDim.x) {
-    const int pos = j < c ? p.pos[r.rows0 + j] : n;
-    const float key = static_cast<float>(pos);  // exact: positions < 2^24
-    if (pos >= ly.sink && (bp < 0 || key < ba)) {
-      ba = key;
-      bp = pos;
-      bs = j;
-    }
-  }
-  // positions are distinct, so "smallest key" decides alone
-  const int ev = block_evict_choice(ba, bp, bs, sh);
-  __syncthreads();
-  const int evicted_pos = ev < 0 ? -1 : (ev < c ? p.pos[r.rows0 + ev] : n);
-  __syncthreads();
-  if (ev < 0) {
-    if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
-    return;
-  }
-  place_new(p, r, D, ev < c ? ev : -1, n, 0.f, c, evicted_pos);
+  return lo;
 }
 
-// The step of unit blockIdx.x (called by the whole block; returns early on
-// an inconsistent state, which it records in the status word).
-template <int D, int G>
-__device__ __forceinline__ void step_unit(const DecodeParams& p, float* lg, DecShared& sh) {
-  const int u = blockIdx.x;
-  const int l = find_dec_layer(p, u);
+__device__ __forceinline__ UnitRef unit_ref(const DecodeParams& p, int l, int rem) {
   const DecLayer& ly = p.layer[l];
-  const int rem = u - ly.unit_off;
   UnitRef r;
   r.l = l;
   r.s = rem / p.H_kv;
   r.h = rem - r.s * p.H_kv;
-  r.u = u;
+  r.u = ly.unit_off + rem;
   r.rows0 = static_cast<size_t>(ly.row_off) + static_cast<size_t>(rem) * ly.cap;
+  return r;
+}
+
+// The step of the a-th H2O / TOVA unit (called by the whole block; returns
+// early on an inconsistent state, which it records in the status word).
+template <int D, int G>
+__device__ __forceinline__ void step_attend(const DecodeParams& p, int a, float* lg, DecShared& sh) {
+  const int l = find_kind_layer<true>(p, a);
+  const DecLayer& ly = p.layer[l];
+  const UnitRef r = unit_ref(p, l, a - (ly.att_end - p.B * p.H_kv));
   const int n = p.lens[r.s];
-  const int c = p.count[u];
+  const int c = p.count[r.u];
   if (c < 0 || c > ly.cap) {
     if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
     return;
   }
-  if (ly.method == KVEV_H2O || ly.method == KVEV_TOVA) attend_unit<D, G>(p, ly, r, n, c, lg, sh);
-  else if (ly.method == KVEV_STREAMING) stream_unit(p, ly, r, D, n, c, sh);
-  else if (c < ly.cap) place_new(p, r, D, c, n, 0.f, c + 1, -1);  // append only
-  else if (threadIdx.x == 0) atomicOr(p.status, kStatusDevice);
+  attend_unit<D, G>(p, ly, r, n, c, lg, sh);
+}
+
+// place_new by one warp: the new token's K/V row (16-byte vectors over the
+// lanes), then its bookkeeping by lane 0.
+__device__ __forceinline__ void place_new_warp(const DecodeParams& p, const UnitRef& r, int D, int dst, int n,
+                                               float acc_new, int new_count, int evicted_pos) {
+  const int lane = threadIdx.x & 31;
+  if (dst >= 0) {
+    const int vec = D / 8;
+    const size_t src = static_cast<size_t>(r.s) * p.H_kv + r.h;
+    for (int i = lane; i < 2 * vec; i += 32) {
+      const bool isv = i >= vec;
+      const int e = isv ? i - vec : i;
+      uint4* drow = reinterpret_cast<uint4*>(isv ? p.V : p.K) + (r.rows0 + dst) * vec + e;
+      const uint4* srow = reinterpret_cast<const uint4*>(isv ? p.v_new[r.l] : p.k_new[r.l]) + src * vec + e;
+      *drow = *srow;
+    }
+  }
+  if (lane == 0) {
+    if (dst >= 0) {
+      p.pos[r.rows0 + dst] = n;
+      p.acc[r.rows0 + dst] = acc_new;
+    }
+    p.count[r.u] = new_count;
+    p.evicted[r.u] = evicted_pos;
+  }
+}
+
+// The step of the i-th StreamingLLM or append-only unit, by one warp (no
+// block barrier): StreamingLLM evicts the smallest position >= sink once
+// sink + recent slots are held; an append-only unit takes the next slot.
+__device__ void step_cheap_warp(const DecodeParams& p, int i, int D) {
+  const int lane = threadIdx.x & 31;
+  const int l = find_kind_layer<false>(p, i);
+  const DecLayer& ly = p.layer[l];
+  const UnitRef r = unit_ref(p, l, i - (ly.cheap_end - p.B * p.H_kv));
+  const int n = p.lens[r.s];
+  const int c = p.count[r.u];
+  const bool streaming = ly.method == KVEV_STREAMING;
+  if (c < 0 || c > ly.cap || (!streaming && c >= ly.cap) ||
+      (streaming && c + 1 <= ly.sink + ly.recent && c >= ly.cap)) {
+    if (lane == 0) atomicOr(p.status, kStatusDevice);
+    return;
+  }
+  if (!streaming || c + 1 <= ly.sink + ly.recent) {  // append
+    place_new_warp(p, r, D, c, n, 0.f, c + 1, -1);
+    return;
+  }
+  // smallest position >= sink among the slots and the new token (positions are distinct)
+  int bp = 0x7FFFFFFF, bs = -1;
+  for (int j = lane; j <= c; j += 32) {
+    const int pos = j < c ? p.pos[r.rows0 + j] : n;
+    if (pos >= ly.sink && pos < bp) {
+      bp = pos;
+      bs = j;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const int bp2 = __shfl_xor_sync(0xffffffffu, bp, o);
+    const int bs2 = __shfl_xor_sync(0xffffffffu, bs, o);
+    if (bp2 < bp) {
+      bp = bp2;
+      bs = bs2;
+    }
+  }
+  __syncwarp();  // every lane has read the positions before slot bs is rewritten
+  if (bs < 0) {
+    if (lane == 0) atomicOr(p.status, kStatusDevice);
+    return;
+  }
+  place_new_warp(p, r, D, bs < c ? bs : -1, n, 0.f, c, bp);
 }
 
 template <int D, int G>
 __global__ void __launch_bounds__(kDecodeThreads) decode_step_kernel(const __grid_constant__ DecodeParams p) {
   extern __shared__ float lg[];
   __shared__ DecShared sh;
-  step_unit<D, G>(p, lg, sh);
-  // The last unit of the step to finish advances every sequence by one token:
+  // CTAs [0, n_att): one H2O / TOVA unit each; then eight cheap units per CTA
+  if (static_cast<int>(blockIdx.x) < p.n_att) {
+    step_attend<D, G>(p, blockIdx.x, lg, sh);
+  } else {
+    const int i = (blockIdx.x - p.n_att) * kDecodeWarps + (threadIdx.x >> 5);
+    if (i < p.n_cheap) step_cheap_warp(p, i, D);
+  }
+  // The last CTA of the step to finish advances every sequence by one token:
   // every other CTA has read lens before it counted itself done.
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -432,7 +509,8 @@ cudaError_t launch_step_dg(const DecodeParams& p, size_t smem, cudaStream_t st) 
                                                static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  decode_step_kernel<D, G><<<p.units, kDecodeThreads, smem, st>>>(p);
+  const int grid = p.n_att + (p.n_cheap + kDecodeWarps - 1) / kDecodeWarps;
+  decode_step_kernel<D, G><<<grid, kDecodeThreads, smem, st>>>(p);
   return cudaGetLastError();
 }
 

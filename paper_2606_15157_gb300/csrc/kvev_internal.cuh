@@ -141,6 +141,8 @@ struct DecLayer {
   int pre_method;     // prefill operator (its packed rows seed the arena)
   int pre_slots;      // prefill slots per unit (b_l)
   int unit_off;       // first unit of the layer
+  int att_end;        // H2O / TOVA units of layers 0..l (one CTA each in the step kernel)
+  int cheap_end;      // StreamingLLM and append-only units of layers 0..l (one warp each)
   long long row_off;  // first arena slot row of the layer
   long long pre_row_off;  // first packed prefill row of the layer
 };
@@ -152,6 +154,7 @@ struct DecodeParams {
   const void* q_new[kMaxLayers];  // [B][H_q][d]
   const float* attn[kMaxLayers];  // [B][H_kv][cap + 1] caller-supplied attention, or null
   int L, B, H_kv, H_q, G, d, units;
+  int n_att, n_cheap; // attending units; StreamingLLM and append-only units
   float scale_log2;   // log2(e) / sqrt(d)
   void* K;            // arena rows [rows][d] bf16
   void* V;
