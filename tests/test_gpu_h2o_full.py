@@ -142,8 +142,9 @@ def _run_full_prompt(torch, wl, rng):
 
 def test_h2o_full_prompt_8k_properties(torch):
     # The geometry the full-prompt bench measures (8,192 positions, 32/8 heads,
-    # d = 128: 128 query blocks and 32 key super-tiles per unit).  Two sampled
-    # H2O units against the oracle, and every H2O unit: each query row's softmax sums to 1, so the scores of a KV head
+    # d = 128: 128 query blocks and 32 key super-tiles per unit).  Every H2O
+    # unit against the oracle (all host cores), and every H2O unit against
+    # properties: each query row's softmax sums to 1, so the scores of a KV head
     # (averaged over its G query heads) sum to n and are positive; the kept
     # set is the recent window plus the top (b - r) of the unit's own scores
     # before it (ties to the lower position); the H2O state holds the kept
@@ -167,10 +168,11 @@ def test_h2o_full_prompt_8k_properties(torch):
             expect = set(order[:b - r].tolist()) | set(range(n - r, n))
             assert set(kept.tolist()) == expect
             np.testing.assert_array_equal(gpu.state[base: base + cnt], gpu.scores[l][0, h, kept])
-    # and two sampled units against the oracle
+    # and every H2O unit against the oracle
+    import os
     import oracle
     specs, meta = [], []
-    for (l, h) in ((0, 5), (2, 1)):
+    for (l, h) in [(l, h) for l in (0, 2) for h in range(wl.H_kv)]:
         Kh = parity.to_host_u16(dev[l][0][0])
         Vh = parity.to_host_u16(dev[l][1][0])
         spec = parity.oracle_spec(wl, l, 0, h, Kh[h][:n],
@@ -179,20 +181,21 @@ def test_h2o_full_prompt_8k_properties(torch):
         spec["n"] = n
         specs.append(spec)
         meta.append((l, 0, h, n, Kh[h], Vh[h]))
-    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=2)
+    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=os.cpu_count())
     for (l, s, h, n_, Kr, Vr), res in zip(meta, results):
         parity.check_unit(wl, l, s, h, n_, res, gpu, Kr, Vr)
 
 
 def test_h2o_full_prompt_2k_oracle(torch):
     # The same geometry at 2,048 positions (32 query blocks, 8 key super-tiles):
-    # two sampled H2O units against the oracle with the whole prompt as the window.
+    # every H2O unit against the oracle with the whole prompt as the window.
+    import os
     import oracle
     wl = _full_prompt_workload(2048, 22)
     n = int(wl.lens[0])
     plan, bufs, dev, q_full, gpu = _run_full_prompt(torch, wl, np.random.default_rng(9))
     specs, meta = [], []
-    for (l, h) in ((0, 3), (2, 6)):
+    for (l, h) in [(l, h) for l in (0, 2) for h in range(wl.H_kv)]:
         Kh = parity.to_host_u16(dev[l][0][0])
         Vh = parity.to_host_u16(dev[l][1][0])
         spec = parity.oracle_spec(wl, l, 0, h, Kh[h][:n],
@@ -201,7 +204,7 @@ def test_h2o_full_prompt_2k_oracle(torch):
         spec["n"] = n
         specs.append(spec)
         meta.append((l, 0, h, n, Kh[h], Vh[h]))
-    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=2)
+    results = oracle.evict_units(specs, d=wl.d, G=wl.G, nthreads=os.cpu_count())
     for (l, s, h, n_, Kr, Vr), res in zip(meta, results):
         parity.check_unit(wl, l, s, h, n_, res, gpu, Kr, Vr)
 
