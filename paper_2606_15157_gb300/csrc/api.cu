@@ -25,7 +25,7 @@ struct DevCtx {
   int device = -1;
   int num_sms = 0;
   int smem_optin = 0;
-  size_t score_smem_set = 0, select_smem_set = 0, h2o_full_smem_set = 0;
+  size_t score_smem_set = 0, h2o_full_smem_set = 0;
   int* status = nullptr;
 };
 
@@ -63,6 +63,9 @@ struct WsLayout {
          lam = 0, raw = 0, lse = 0, sel_keys = 0, total = 0;
 };
 
+// Entries of a selection key row: S_cap rounded up to whole 16-byte vectors.
+int sel_key_stride(int S_cap) { return (S_cap + 3) & ~3; }
+
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   WsLayout w;
   w.n_units = static_cast<int>(p.score_layers.size()) * B * p.H_kv;
@@ -85,8 +88,8 @@ WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   w.part = take(sizeof(float2) * static_cast<size_t>(w.max_items) * w.R_pad);  // one per chunk
   w.lam = take(sizeof(float) * static_cast<size_t>(w.n_units) * w.R_pad);
   w.raw = take(sizeof(float) * static_cast<size_t>(w.n_units) * S_cap);
-  if (S_cap > kSelectSmemCapMax)  // the selection's keys and candidates, per scoring unit
-    w.sel_keys = take(sizeof(uint32_t) * 2 * static_cast<size_t>(w.n_units) * S_cap);
+  // the selection's keys, one 16-byte aligned row per scoring unit
+  w.sel_keys = take(sizeof(uint32_t) * static_cast<size_t>(w.n_units) * sel_key_stride(S_cap));
   if (p.h2o_full) {  // base-2 log-sum-exp of every prompt row of every H2O unit
     for (int l : p.score_layers) w.n_h2o_units += p.route_pre[l] == KVEV_H2O ? B * p.H_kv : 0;
     w.lse = take(sizeof(float) * static_cast<size_t>(w.n_h2o_units) * p.G * S_cap);
@@ -159,7 +162,7 @@ int query_device(DevCtx& c, int dev) {
     return KVEV_ECUDA;
   if (major < 10) return KVEV_ENOTSUP;
   c.device = dev;
-  c.score_smem_set = c.select_smem_set = c.h2o_full_smem_set = 0;
+  c.score_smem_set = c.h2o_full_smem_set = 0;
   return KVEV_OK;
 }
 
@@ -842,25 +845,10 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.lens = lens_ok;
   sel.out_idx = out_idx;
   sel.out_count = out_count;
-  // dynamic shared memory of the selection: the unit's keys, then as many
-  // candidate positions (at most S_cap) as fit next to the static part
-  size_t sel_smem = 0;
-  if (ws.n_units > 0 && S_cap > kSelectSmemCapMax) {
-    sel.keys_g = reinterpret_cast<uint32_t*>(wsb + ws.sel_keys);
-    sel.cand_cap = S_cap;
-  } else if (ws.n_units > 0) {
-    const size_t keys_b = sizeof(uint32_t) * static_cast<size_t>(S_cap);
-    if (keys_b + kSelectStaticSmem + 1024 > static_cast<size_t>(D.smem_optin)) return KVEV_ENOTSUP;
-    const size_t room = static_cast<size_t>(D.smem_optin) - kSelectStaticSmem - 1024 - keys_b;
-    sel.cand_cap = static_cast<int>(std::min<size_t>(room / sizeof(int), static_cast<size_t>(S_cap)));
-    sel_smem = keys_b + sizeof(int) * static_cast<size_t>(sel.cand_cap);
-  }
-  if (sel_smem > 48 * 1024 && D.select_smem_set < sel_smem) {
-    if (select_set_smem(sel_smem) != cudaSuccess) return KVEV_ECUDA;
-    D.select_smem_set = sel_smem;
-  }
+  sel.keys = reinterpret_cast<uint32_t*>(wsb + ws.sel_keys);
+  sel.key_stride = sel_key_stride(S_cap);
   mark(KVEV_K_SELECT, 0);
-  if (launch_select(sel, P.L * B * P.H_kv, sel_smem, s) != cudaSuccess) return KVEV_ECUDA;
+  if (launch_select(sel, P.L * B * P.H_kv, s) != cudaSuccess) return KVEV_ECUDA;
   mark(KVEV_K_SELECT, 1);
 
   // ---- gather-compaction ---------------------------------------------------

@@ -41,12 +41,8 @@ constexpr int kSlotCols = 128;        // fp32 columns per slot (4 x 128 = all 51
 constexpr int kRegsControl = 64;
 constexpr int kRegsSoftmax = 104;
 constexpr int kRegsNeeded = 128 * kRegsControl + 128 * kSoftmaxWGs * kRegsSoftmax;
-constexpr int kSelectThreads = 1024;
-constexpr int kSelectStaticSmem = 17 * 1024;  // bound on the select kernel's static shared memory
-// Largest capacity whose selection keys fit a CTA's shared memory next to the
-// static part (227 KiB opt-in per block on GB300); above it the keys and the
-// candidate positions live in a workspace region instead.
-constexpr int kSelectSmemCapMax = (227 * 1024 - kSelectStaticSmem - 1024) / 4;
+constexpr int kSelectThreads = 256;    // one selection CTA per unit
+constexpr int kSelectCtasPerSm = 4;    // resident selection CTAs an SM should hold
 constexpr int kWsAlign = 256;
 
 // Bits of the device status word.
@@ -126,9 +122,8 @@ struct SelectParams {
   const int* lens;
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
-  int cand_cap;       // candidate positions that fit after the keys in dynamic shared memory
-  uint32_t* keys_g;   // capacities above kSelectSmemCapMax: [scoring unit][2][S_cap] keys, then
-                      // candidate positions, in the workspace (null: shared memory)
+  uint32_t* keys;     // workspace: [scoring unit][key_stride] selection keys
+  int key_stride;     // S_cap rounded up to a multiple of 4 (16-byte aligned rows)
 };
 
 // Per-layer description of the decode arena.
@@ -578,7 +573,6 @@ int h2o_full_smem_bytes(int d);
 int h2o_full_kernel_regs(int d);
 cudaError_t h2o_full_set_smem(int d, size_t smem);
 cudaError_t launch_h2o_full(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
-cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s);
-cudaError_t select_set_smem(size_t smem);
+cudaError_t launch_select(const SelectParams& p, int grid, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s, int num_sms);
 }  // namespace kvev

@@ -3,8 +3,10 @@
 //
 //   SnapKV   : E = n - W prefix positions; keys = 1-D pooled window scores
 //              (stride 1, width p, same length; max ignores out-of-range
-//              entries, avg pads with zeros and divides by p); keep the
-//              top (b - W) prefix positions plus the window [E, n).
+//              entries, avg pads with zeros and divides by p -- a division
+//              by the same p for every key, so the window sum ranks the keys
+//              alike and is used instead); keep the top (b - W) prefix
+//              positions plus the window [E, n).
 //   H2O      : E = n - r (r = protected recent window); keys = raw window
 //              scores; keep the top (b - r) of [0, E) plus [E, n).
 //   Streaming: keep [0, sink) plus the last `recent` positions (closed form).
@@ -12,15 +14,27 @@
 // Top-k order: larger score first, equal scores keep the lower position.
 // Output indices are ascending; unused slots hold -1.
 //
-// The k-th largest key is found over an order-preserving uint32 image of the
-// fp32 scores held in shared memory.  The pass that builds the keys also
-// histograms their top 12 bits; the bin holding the k-th key is then the only
-// one that matters: each warp counts, then gathers in position order, that
-// bin's positions in its segment (counting the keys above it), two 10-bit
-// radix passes over those candidates alone fix the threshold key, and one
-// ordered pass (ballot/popc prefix counts) writes the kept positions.  Four
-// light passes over the unit's keys in all, none through a shared counter; a
-// first bin too crowded for the candidate buffer takes four 8-bit radix
+// A unit takes a CTA of 256 threads, so that several units share an SM and
+// one unit's barriers and round trips overlap another's passes.  The keys (an
+// order-preserving uint32 image of the fp32 scores) go to the unit's row of a
+// workspace array, which stays in L2 between the passes:
+//   1. build the keys and find their range [lo, hi];
+//   2. histogram the first digit (key - lo) >> s, which splits the range into
+//      at most 8192 bins of 2^s keys (a unit's scores may crowd into a few
+//      per cent of one octave, or spread over many octaves: the range adapts
+//      the bins to either);
+//   3. find the bin holding the k-th largest key; each warp counts the keys
+//      of higher bins in its segment and appends that bin's keys (the
+//      candidates) to a shared list that reuses the histogram's space; radix
+//      passes of up to 9 bits over the candidates' s low bits fix the
+//      threshold key T and how many keys equal to T to keep, and the
+//      candidates' tallies give every warp segment its counts above and equal
+//      to T;
+//   4. one ordered pass writes the kept positions: a warp's slots follow those
+//      of the warps before it, and within a warp lanes hold four consecutive
+//      keys each, ranked by warp scans.
+// Equal keys everywhere take the first k positions directly; a candidate bin
+// with more keys than the list holds (many equal keys) takes four 8-bit radix
 // passes over every key instead.
 #include "kvev_internal.cuh"
 
@@ -28,25 +42,27 @@ namespace kvev {
 
 namespace {
 
-// Bulk prefetch of [src, src + bytes) into L2 (src 16-byte aligned, bytes a
-// multiple of 16).
-__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
+constexpr int kSW = kSelectThreads / 32;   // warps of a selection CTA
+constexpr int kBins0 = 8192;               // first digit: the keys' range in at most 8192 bins
+constexpr int kCandCap = kBins0 / 2;       // (position, key) pairs in the histogram's space
+constexpr int kBins1 = 512;                // candidate digits: up to 9 bits a pass
+constexpr int kSegKeys = 128;              // a warp block: four keys per lane
+constexpr int kSelectUnroll = 4;           // key blocks whose loads are in flight together
 
-constexpr int kHistBits = 12;              // first radix digit: the top 12 bits of a key
-constexpr int kHistBins = 1 << kHistBits;
-constexpr int kSelWarps = kSelectThreads / 32;
-
-static_assert(kSelWarps == 32, "find_bin scans the warp totals with one warp");
-
-struct SelShared {
-  int hist[kHistBins];
-  int wsum[kSelWarps];
-  int wcnt[2][kSelWarps];  // per warp segment: keys above T, keys equal to T
+struct __align__(16) SelShared {
+  union {
+    int hist[kBins0];
+    uint2 cand[kCandCap];
+  } u;
+  int hist1[kBins1];
+  int wsum[kSW];
+  int wgt[kSW];   // per warp segment: keys above T
+  int weq[kSW];   // per warp segment: keys equal to T
   int bcast[2];
   int ncand;
 };
+
+static_assert(sizeof(SelShared) <= 48 * 1024, "the selection's shared memory is static");
 
 // Adds each valid lane's digit to the histogram, one shared-memory atomic per
 // distinct digit of the warp (the scores of a unit crowd into few bins).
@@ -57,50 +73,96 @@ __device__ __forceinline__ void hist_add(int* hist, bool valid, uint32_t digit) 
   if (valid && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
 }
 
-// Per-unit scores (or pooled scores) into order-preserving keys in shared
-// memory, and the histogram of their top kHistBits bits.  Every load of a
-// key's window is issued before any is used, four keys per thread at a time
-// (the window reads of neighbouring keys overlap and are served by L1), so the
-// latency of the score reads is paid once per group of keys rather than once
-// per window element.  The loop bounds are uniform over the block so that all
-// lanes reach the warp-wide match in hist_add.
-template <int P>
-__device__ __forceinline__ void build_keys_pooled(uint32_t* keys, int* hist, const float* raw, int E,
-                                                  bool is_max) {
-  constexpr int h = P / 2;
-  constexpr int U = 4;
-  for (int b0 = 0; b0 < E; b0 += U * kSelectThreads) {
-    float w[U][P];
+// Inclusive warp scan.
+__device__ __forceinline__ int warp_incl(int x) {
+  const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = b0 + u * kSelectThreads + threadIdx.x;
-#pragma unroll
-      for (int j = 0; j < P; ++j) {
-        const int q = i - h + j;
-        w[u][j] = (i < E && q >= 0 && q < E) ? raw[q] : (is_max ? -INFINITY : 0.f);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = b0 + u * kSelectThreads + threadIdx.x;
-      float v = w[u][0];
-#pragma unroll
-      for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[u][j]) : v + w[u][j];
-      const uint32_t key = float_key(is_max ? v : v / static_cast<float>(P));
-      if (i < E) keys[i] = key;
-      hist_add(hist, i < E, key >> (32 - kHistBits));
-    }
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
   }
+  return x;
 }
 
-// The same with 16-byte loads, for a 16-byte aligned score row: thread t of a
-// round takes keys 4t .. 4t+3, whose windows (P <= 9) lie in the three
-// aligned 4-float chunks starting at 4t - 4, 4t and 4t + 4.  Only chunks that
-// start before E are read (E <= S_cap, a multiple of 4, so none leaves the
-// row); entries outside [0, E) count as -inf (max) or 0 (avg).
+__device__ __forceinline__ int warp_sum(int x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// The bin of a histogram of `nbins` digits (a multiple of the block size)
+// that holds the kk-th largest key (1 <= kk <= keys counted), and the number
+// of keys in higher bins.  Thread t owns the q = nbins / 256 bins
+// nbins-1-q*t down to nbins-q*(t+1).
+__device__ void find_bin(const int* hist, int nbins, int kk, SelShared& sh, int& digit, int& above) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int q = nbins / kSelectThreads;
+  const int lo = nbins - q * (threadIdx.x + 1);  // this thread's lowest bin
+  int s = 0;
+  if (q % 4 == 0) {
+    const int4* h4 = reinterpret_cast<const int4*>(hist + lo);
+    for (int j = 0; j < q / 4; ++j) {
+      const int4 v = h4[j];
+      s += (v.x + v.y) + (v.z + v.w);
+    }
+  } else {
+    for (int j = 0; j < q; ++j) s += hist[lo + j];
+  }
+  int incl = warp_incl(s);
+  if (lane == 31) sh.wsum[warp] = incl;
+  __syncthreads();
+  for (int w = 0; w < warp; ++w) incl += sh.wsum[w];
+  const int before = incl - s;
+  if (before < kk && kk <= incl) {
+    int acc = before, b = lo + q - 1;
+    while (b > lo && acc + hist[b] < kk) acc += hist[b--];
+    sh.bcast[0] = b;
+    sh.bcast[1] = acc;
+  }
+  __syncthreads();
+  digit = sh.bcast[0];
+  above = sh.bcast[1];
+  __syncthreads();  // wsum and bcast are reused by the next call
+}
+
+// Warp segments of [0, E): contiguous, whole 128-key iterations, in warp
+// order, so that a warp's kept positions follow those of the warps before it.
+__device__ __forceinline__ int seg_len(int E) {
+  return ((E + kSW - 1) / kSW + kSegKeys - 1) / kSegKeys * kSegKeys;
+}
+
+// Four consecutive keys from a 16-byte aligned key row (the row is padded to
+// a multiple of four entries, so the load never leaves it).
+__device__ __forceinline__ uint4 ld_keys4(const uint32_t* keys, int i0) {
+  return __ldcg(reinterpret_cast<const uint4*>(keys + i0));
+}
+
+__device__ __forceinline__ uint32_t pick(const uint4& v, int u) {
+  return u == 0 ? v.x : u == 1 ? v.y : u == 2 ? v.z : v.w;
+}
+
+// ---------------------------------------------------------------------------
+// Pass 1: the keys and their range.  Keys past E in the last group of four are
+// written too (the row is padded); no later pass reads them.
+// ---------------------------------------------------------------------------
+struct KeyRange {
+  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+  __device__ __forceinline__ void add(uint32_t k, bool valid) {
+    if (valid) {
+      lo = min(lo, k);
+      hi = max(hi, k);
+    }
+  }
+};
+
+// Pooled keys from a 16-byte aligned score row: thread t of a round takes keys
+// 4t .. 4t+3, whose windows (P <= 9) lie in the three aligned 4-float chunks
+// starting at 4t - 4, 4t and 4t + 4.  Only chunks that start before E are read
+// (E <= S_cap, a multiple of 4, so none leaves the row); entries outside
+// [0, E) count as -inf (max) or 0 (avg).
 template <int P>
-__device__ __forceinline__ void build_keys_pooled4(uint32_t* keys, int* hist, const float* raw, int E,
-                                                   bool is_max) {
+__device__ __forceinline__ void build_pooled4(uint32_t* keys, const float* raw, int E, bool is_max,
+                                              KeyRange& kr) {
   constexpr int h = P / 2;
   static_assert(h <= 4, "the three chunks cover windows of up to 9");
   const float fill = is_max ? -INFINITY : 0.f;
@@ -111,273 +173,313 @@ __device__ __forceinline__ void build_keys_pooled4(uint32_t* keys, int* hist, co
     for (int c = 0; c < 3; ++c) {
       const int st = i0 - 4 + 4 * c;
       float4 v = make_float4(fill, fill, fill, fill);
-      if (st >= 0 && st < E) v = *reinterpret_cast<const float4*>(raw + st);
+      if (st >= 0 && st < E) v = __ldg(reinterpret_cast<const float4*>(raw + st));  // neighbours' chunks: L1 hits
       w[4 * c + 0] = st + 0 < E ? v.x : fill;
       w[4 * c + 1] = st + 1 < E ? v.y : fill;
       w[4 * c + 2] = st + 2 < E ? v.z : fill;
       w[4 * c + 3] = st + 3 < E ? v.w : fill;
     }
+    uint32_t kq[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const int i = i0 + u;
       float v = w[4 + u - h];
 #pragma unroll
       for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[4 + u - h + j]) : v + w[4 + u - h + j];
-      const uint32_t key = float_key(is_max ? v : v / static_cast<float>(P));
-      if (i < E) keys[i] = key;
-      hist_add(hist, i < E, key >> (32 - kHistBits));
+      kq[u] = float_key(v);
+      kr.add(kq[u], i0 + u < E);
+    }
+    if (i0 < E) *reinterpret_cast<uint4*>(keys + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+  }
+}
+
+// Raw keys (no pooling) from a 16-byte aligned score row.
+__device__ __forceinline__ void build_raw4(uint32_t* keys, const float* raw, int E, KeyRange& kr) {
+  for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
+    const int i0 = b0 + 4 * threadIdx.x;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i0 < E) v = __ldg(reinterpret_cast<const float4*>(raw + i0));
+    const uint32_t kq[4] = {float_key(v.x), float_key(v.y), float_key(v.z), float_key(v.w)};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) kr.add(kq[u], i0 + u < E);
+    if (i0 < E) *reinterpret_cast<uint4*>(keys + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+  }
+}
+
+// Any alignment and any odd pooling width: one key per thread at a time.
+__device__ void build_scalar(uint32_t* keys, const float* raw, int E, int pool, bool do_pool, bool is_max,
+                             KeyRange& kr) {
+  const int h = pool / 2;
+  for (int i = threadIdx.x; i < E; i += kSelectThreads) {
+    float v;
+    if (!do_pool) {
+      v = raw[i];
+    } else if (is_max) {
+      v = -INFINITY;
+      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
+      for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
+    } else {
+      v = 0.f;
+      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
+      for (int j = lo; j <= hi; ++j) v += raw[j];
+    }
+    keys[i] = float_key(v);
+    kr.add(keys[i], true);
+  }
+}
+
+// Builds the keys of [0, E) and returns their range in sh.bcast (lo, hi).
+__device__ void build_keys(uint32_t* keys, const float* raw, int E, int pool, int pool_type, bool do_pool,
+                           bool aligned4, SelShared& sh) {
+  const bool is_max = pool_type == KVEV_POOL_MAX;
+  KeyRange kr;
+  bool done = false;
+  if (aligned4) {
+    done = true;
+    if (!do_pool) build_raw4(keys, raw, E, kr);
+    else if (pool == 3) build_pooled4<3>(keys, raw, E, is_max, kr);
+    else if (pool == 5) build_pooled4<5>(keys, raw, E, is_max, kr);
+    else if (pool == 7) build_pooled4<7>(keys, raw, E, is_max, kr);
+    else if (pool == 9) build_pooled4<9>(keys, raw, E, is_max, kr);
+    else done = false;
+  }
+  if (!done) build_scalar(keys, raw, E, pool, do_pool, is_max, kr);
+  const uint32_t lo = __reduce_min_sync(0xffffffffu, kr.lo), hi = __reduce_max_sync(0xffffffffu, kr.hi);
+  if ((threadIdx.x & 31) == 0) {
+    atomicMin(reinterpret_cast<unsigned*>(&sh.bcast[0]), lo);
+    atomicMax(reinterpret_cast<unsigned*>(&sh.bcast[1]), hi);
+  }
+}
+
+// Pass 2: histogram of the first digit (key - lo) >> s, which splits the keys'
+// range into at most kBins0 bins of 2^s keys each (plain atomics: keys spread
+// over the bins).
+__device__ void range_hist(const uint32_t* keys, int E, uint32_t lo, int s, int* hist) {
+  constexpr int R = kSelectUnroll;
+  for (int b0 = 0; b0 < E; b0 += 4 * R * kSelectThreads) {
+    uint4 kv[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + (r * kSelectThreads + threadIdx.x) * 4;
+      kv[r] = i0 < E ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + (r * kSelectThreads + threadIdx.x) * 4;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u < E) atomicAdd(&hist[(pick(kv[r], u) - lo) >> s], 1);
     }
   }
 }
 
-__device__ void build_keys(uint32_t* keys, int* hist, const float* raw, int E, int pool, int pool_type,
-                           bool do_pool, bool aligned4) {
-  const bool is_max = pool_type == KVEV_POOL_MAX;
-  if (do_pool && aligned4) {
-    switch (pool) {
-      case 3: build_keys_pooled4<3>(keys, hist, raw, E, is_max); return;
-      case 5: build_keys_pooled4<5>(keys, hist, raw, E, is_max); return;
-      case 7: build_keys_pooled4<7>(keys, hist, raw, E, is_max); return;
-      case 9: build_keys_pooled4<9>(keys, hist, raw, E, is_max); return;
-      default: break;
+// ---------------------------------------------------------------------------
+// Pass 2 and the candidate radix passes.
+// ---------------------------------------------------------------------------
+
+// Each warp counts its segment's keys of first-digit bins above d (into wgt)
+// and appends the keys of bin d, with their positions, to the candidate list
+// (in no particular order; at most kCandCap are stored, ncand counts them all).
+__device__ void collect_candidates(const uint32_t* keys, int E, uint32_t lo_key, int s, uint32_t d,
+                                   SelShared& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int seg = seg_len(E);
+  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
+  int gt = 0;
+  constexpr int R = kSelectUnroll;
+  for (int b0 = lo; b0 < hi; b0 += R * kSegKeys) {
+    uint4 kv[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + r * kSegKeys + 4 * lane;
+      kv[r] = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
     }
-  }
-  if (do_pool) {
-    switch (pool) {  // common widths with fully unrolled windows
-      case 3: build_keys_pooled<3>(keys, hist, raw, E, is_max); return;
-      case 5: build_keys_pooled<5>(keys, hist, raw, E, is_max); return;
-      case 7: build_keys_pooled<7>(keys, hist, raw, E, is_max); return;
-      case 9: build_keys_pooled<9>(keys, hist, raw, E, is_max); return;
-      default: break;
-    }
-  }
-  const int h = pool / 2;
-  for (int b0 = 0; b0 < E; b0 += kSelectThreads) {
-    const int i = b0 + threadIdx.x;
-    float v = 0.f;
-    if (i < E) {
-      if (!do_pool) {
-        v = raw[i];
-      } else if (is_max) {
-        v = -INFINITY;
-        const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-        for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
-      } else {
-        float sum = 0.f;
-        const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-        for (int j = lo; j <= hi; ++j) sum += raw[j];
-        v = sum / static_cast<float>(pool);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + r * kSegKeys + 4 * lane;
+      int c = 0;
+      uint32_t cmask = 0;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const bool valid = i0 + u < hi;
+        const uint32_t q = (pick(kv[r], u) - lo_key) >> s;
+        gt += valid && q > d;
+        const bool in = valid && q == d;
+        cmask |= static_cast<uint32_t>(in) << u;
+        c += in;
+      }
+      if (__any_sync(0xffffffffu, c)) {
+        const int incl = warp_incl(c);
+        int base = 0;
+        if (lane == 31) base = atomicAdd(&sh.ncand, incl);
+        base = __shfl_sync(0xffffffffu, base, 31) + incl - c;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          if (cmask & (1u << u)) {
+            if (base < kCandCap) sh.u.cand[base] = make_uint2(static_cast<uint32_t>(i0 + u), pick(kv[r], u));
+            ++base;
+          }
+        }
       }
     }
-    const uint32_t key = float_key(v);
-    if (i < E) keys[i] = key;
-    hist_add(hist, i < E, key >> (32 - kHistBits));
+  }
+  gt = warp_sum(gt);
+  if (lane == 0) {
+    sh.wgt[warp] = gt;
+    sh.weq[warp] = 0;
   }
 }
 
-// The bin of a histogram of `nbins` digits (a multiple of the block size)
-// that holds the kk-th largest key (kk >= 1), and the number of keys in
-// higher bins.  Thread t owns bins nbins-1-q*t .. nbins-q*t-q (descending).
-__device__ void find_bin(SelShared& sh, int nbins, int kk, int& digit, int& above) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int q = nbins / kSelectThreads;
-  const int top = nbins - 1 - q * threadIdx.x;
-  int s = 0;
-  for (int j = 0; j < q; ++j) s += sh.hist[top - j];
-  int incl = s;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += y;
-  }
-  if (lane == 31) sh.wsum[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    int w = sh.wsum[lane], wi = w;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, wi, o);
-      if (lane >= o) wi += y;
+// Threshold key T (the kk-th largest of the candidates, the keys of first-digit
+// bin d) and how many keys equal to T to keep, by radix passes of up to 9 bits
+// over the s low bits of key - lo_key; then each candidate above or equal to
+// T is tallied to its warp segment.
+__device__ void select_candidates(int E, uint32_t lo_key, int s, uint32_t d, int kk, SelShared& sh,
+                                  uint32_t& T, int& need) {
+  const int nc = sh.ncand;
+  uint32_t prefix = 0, mask = 0;  // over the s low bits
+  for (int r = s; r > 0;) {
+    const int nb = min(9, r), shift = r - nb;
+    const uint32_t dm = (1u << nb) - 1u;
+    for (int i = threadIdx.x; i < kBins1; i += kSelectThreads) sh.hist1[i] = 0;
+    __syncthreads();
+    for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
+      const uint32_t v = sh.u.cand[c].y - lo_key;
+      if ((v & mask) == prefix) atomicAdd(&sh.hist1[(v >> shift) & dm], 1);
     }
-    sh.wsum[lane] = wi - w;  // exclusive prefix over warps
+    __syncthreads();
+    int digit, above;
+    find_bin(sh.hist1, kBins1, kk, sh, digit, above);
+    kk -= above;
+    prefix |= static_cast<uint32_t>(digit) << shift;
+    mask |= dm << shift;
+    r = shift;
   }
-  __syncthreads();
-  incl += sh.wsum[warp];
-  const int before = incl - s;
-  if (before < kk && kk <= incl) {
-    int acc = before, j = 0;
-    while (j < q - 1 && acc + sh.hist[top - j] < kk) acc += sh.hist[top - j++];
-    sh.bcast[0] = top - j;
-    sh.bcast[1] = acc;
+  T = lo_key + ((d << s) | prefix);
+  need = kk;
+  const int seg = seg_len(E);
+  for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
+    const uint2 e = sh.u.cand[c];
+    const int w = static_cast<int>(e.x) / seg;
+    if (e.y > T) atomicAdd(&sh.wgt[w], 1);
+    else if (e.y == T) atomicAdd(&sh.weq[w], 1);
   }
-  __syncthreads();
-  digit = sh.bcast[0];
-  above = sh.bcast[1];
   __syncthreads();
 }
 
-// Threshold key T (the k-th largest) and how many keys equal to T to keep,
-// by 8-bit radix passes over every key (the general path).
-__device__ void radix_select(const uint32_t* keys, int E, int k, SelShared& sh, uint32_t& T,
-                             int& need) {
+// The general path: four 8-bit radix passes over every key, then each warp
+// counts its segment's keys above and equal to T.
+__device__ void select_all_keys(const uint32_t* keys, int E, int k, SelShared& sh, uint32_t& T, int& need) {
   uint32_t prefix = 0, mask = 0;
   int kk = k;
   for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
+    for (int i = threadIdx.x; i < 256; i += kSelectThreads) sh.hist1[i] = 0;
     __syncthreads();
-    for (int base = 0; base < E; base += kSelectThreads) {
-      const int i = base + threadIdx.x;
-      const bool in = i < E && (keys[i] & mask) == prefix;
-      hist_add(sh.hist, in, in ? (keys[i] >> shift) & 255u : 0u);
+    for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
+      const int i0 = b0 + 4 * threadIdx.x;
+      const uint4 kv = i0 < E ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t key = pick(kv, u);
+        const bool in = i0 + u < E && (key & mask) == prefix;
+        hist_add(sh.hist1, in, (key >> shift) & 255u);
+      }
     }
     __syncthreads();
-    int digit, above;  // bins 256 .. 1023 are empty: the 1024-bin search ends in 255 .. 0
-
-    find_bin(sh, 1024, kk, digit, above);
+    int digit, above;
+    find_bin(sh.hist1, 256, kk, sh, digit, above);
     kk -= above;
     prefix |= static_cast<uint32_t>(digit) << shift;
     mask |= 255u << shift;
   }
   T = prefix;
   need = kk;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int seg = seg_len(E);
+  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
+  int gt = 0, eq = 0;
+  for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
+    const int i0 = b0 + 4 * lane;
+    const uint4 kv = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const bool valid = i0 + u < hi;
+      gt += valid && pick(kv, u) > T;
+      eq += valid && pick(kv, u) == T;
+    }
+  }
+  gt = warp_sum(gt);
+  eq = warp_sum(eq);
+  if (lane == 0) {
+    sh.wgt[warp] = gt;
+    sh.weq[warp] = eq;
+  }
+  __syncthreads();
 }
 
-// Warp segments of [0, E): contiguous, 32-aligned, in warp order, so that a
-// warp's kept positions follow those of the warps before it.
-__device__ __forceinline__ int seg_len(int E) { return (((E + kSelWarps - 1) / kSelWarps) + 31) & ~31; }
-
-// Ordered write of the kept positions of [0, E) to out[0..k): keys above T,
-// and the first `need` keys equal to T in position order.  sh.wcnt holds each
-// warp segment's counts of both.
-__device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int need, SelShared& sh,
+// ---------------------------------------------------------------------------
+// Pass 4: ordered write of the kept positions of [0, E) to out[0..k): keys
+// above T, and the first `need` keys equal to T in position order.
+// ---------------------------------------------------------------------------
+__device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int need, const SelShared& sh,
                            int* out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   int eq_base = 0, sel_base = 0;
   for (int w = 0; w < warp; ++w) {
-    const int e = sh.wcnt[1][w];
-    const int take = min(max(need - eq_base, 0), e);
-    sel_base += sh.wcnt[0][w] + take;
+    const int e = sh.weq[w];
+    sel_base += sh.wgt[w] + min(max(need - eq_base, 0), e);
     eq_base += e;
   }
-  const uint32_t lt = (1u << lane) - 1u;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int i = b0 + lane;
-    const uint32_t key = i < hi ? keys[i] : 0u;
-    const bool g = i < hi && key > T;
-    const bool e = i < hi && key == T;
-    const uint32_t eb = __ballot_sync(0xffffffffu, e);
-    const int rank = eq_base + __popc(eb & lt);
-    const bool sel = g || (e && rank < need);
-    const uint32_t sb = __ballot_sync(0xffffffffu, sel);
-    const int slot = sel_base + __popc(sb & lt);
-    if (sel && slot < k) out[slot] = i;
-    eq_base += __popc(eb);
-    sel_base += __popc(sb);
-  }
-}
-
-// Per-warp-segment counts of keys above and equal to T over all of [0, E).
-__device__ void count_segments(const uint32_t* keys, int E, uint32_t T, SelShared& sh) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int seg = seg_len(E);
-  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
-  int gt = 0, eq = 0;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int i = b0 + lane;
-    const uint32_t key = i < hi ? keys[i] : 0u;
-    gt += __popc(__ballot_sync(0xffffffffu, i < hi && key > T));
-    eq += __popc(__ballot_sync(0xffffffffu, i < hi && key == T));
-  }
-  if (lane == 0) {
-    sh.wcnt[0][warp] = gt;
-    sh.wcnt[1][warp] = eq;
-  }
-  __syncthreads();
-}
-
-// The fast path once the first digit's bin (digit d0, kk-th within it) holds
-// at most `cap` keys.  Each warp counts its segment's keys of that bin and of
-// higher bins; a block prefix over the warps gives each warp its own range of
-// cand[], which it fills in position order (no shared counter).  The remaining
-// 20 bits are resolved by two 10-bit radix passes over the candidates alone
-// (their digits are spread out, so plain shared-memory atomics), and each warp
-// then counts its own candidates above and equal to T.
-__device__ void select_by_candidates(const uint32_t* keys, int E, uint32_t d0, int kk, SelShared& sh,
-                                     int* cand, uint32_t& T, int& need) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int seg = seg_len(E);
-  const int lo = min(warp * seg, E), hi = min(lo + seg, E);
-  const uint32_t lt = (1u << lane) - 1u;
-  int gt = 0, mine = 0;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int i = b0 + lane;
-    const uint32_t d = i < hi ? keys[i] >> (32 - kHistBits) : 0u;
-    gt += __popc(__ballot_sync(0xffffffffu, i < hi && d > d0));
-    mine += __popc(__ballot_sync(0xffffffffu, i < hi && d == d0));
-  }
-  if (lane == 0) sh.wsum[warp] = mine;
-  __syncthreads();
-  if (warp == 0) {  // exclusive prefix of the per-warp candidate counts
-    const int v = sh.wsum[lane];
-    int incl = v;
+  constexpr int R = kSelectUnroll;
+  for (int b0 = lo; b0 < hi; b0 += R * kSegKeys) {
+    uint4 kr[R];
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + r * kSegKeys + 4 * lane;
+      kr[r] = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
     }
-    sh.wsum[lane] = incl - v;
-    if (lane == 31) sh.ncand = incl;
-  }
-  __syncthreads();
-  const int first = sh.wsum[warp];  // this warp's range of cand[]: [first, first + mine)
-  int at = first;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int i = b0 + lane;
-    const bool in = i < hi && (keys[i] >> (32 - kHistBits)) == d0;
-    const uint32_t b = __ballot_sync(0xffffffffu, in);
-    if (in) cand[at + __popc(b & lt)] = i;
-    at += __popc(b);
-  }
-  __syncthreads();
-  const int nc = sh.ncand;
-  uint32_t prefix = d0 << (32 - kHistBits), mask = ~0u << (32 - kHistBits);
-  for (int shift = 10; shift >= 0; shift -= 10) {
-    for (int i = threadIdx.x; i < 1024; i += kSelectThreads) sh.hist[i] = 0;
-    __syncthreads();
-    for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
-      const uint32_t key = keys[cand[c]];
-      if ((key & mask) == prefix) atomicAdd(&sh.hist[(key >> shift) & 1023u], 1);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i0 = b0 + r * kSegKeys + 4 * lane;
+      const uint4 kv = kr[r];
+      uint32_t gm = 0, em = 0;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const bool valid = i0 + u < hi;
+        gm |= static_cast<uint32_t>(valid && pick(kv, u) > T) << u;
+        em |= static_cast<uint32_t>(valid && pick(kv, u) == T) << u;
+      }
+      if (!__any_sync(0xffffffffu, gm | em)) continue;
+      // ranks of the keys equal to T, in position order
+      const int ce = __popc(em);
+      const int ie = warp_incl(ce);
+      int rank = eq_base + ie - ce;
+      uint32_t sm = gm;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (em & (1u << u)) {
+          if (rank < need) sm |= 1u << u;
+          ++rank;
+        }
+      }
+      const int cs = __popc(sm);
+      const int is = warp_incl(cs);
+      int slot = sel_base + is - cs;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (sm & (1u << u)) {
+          if (slot < k) out[slot] = i0 + u;
+          ++slot;
+        }
+      }
+      eq_base += __shfl_sync(0xffffffffu, ie, 31);
+      sel_base += __shfl_sync(0xffffffffu, is, 31);
     }
-    __syncthreads();
-    int digit, above;
-    find_bin(sh, 1024, kk, digit, above);
-    kk -= above;
-    prefix |= static_cast<uint32_t>(digit) << shift;
-    mask |= 1023u << shift;
   }
-  T = prefix;
-  need = kk;
-  int eq = 0;
-  for (int c0 = 0; c0 < mine; c0 += 32) {
-    const bool v = c0 + lane < mine;
-    const uint32_t key = v ? keys[cand[first + c0 + lane]] : 0u;
-    gt += __popc(__ballot_sync(0xffffffffu, v && key > T));
-    eq += __popc(__ballot_sync(0xffffffffu, v && key == T));
-  }
-  if (lane == 0) {
-    sh.wcnt[0][warp] = gt;
-    sh.wcnt[1][warp] = eq;
-  }
-  __syncthreads();
 }
 
-static_assert(sizeof(SelShared) <= kSelectStaticSmem, "select kernel's static shared memory");
-
-template <bool kKeysInWorkspace>
-__global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_constant__ SelectParams p) {
-  extern __shared__ uint32_t keys_smem[];
+__global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kernel(const __grid_constant__ SelectParams p) {
   __shared__ SelShared sh;
   const int per_layer = p.B * p.H_kv;
   const int l = blockIdx.x / per_layer;
@@ -426,51 +528,44 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const __grid_con
     return;
   }
   const float* raw = ld.scores + static_cast<size_t>(rem) * p.S_cap;
-  // the unit's keys, then its candidate positions: shared memory, or the
-  // workspace for capacities whose keys do not fit
-  uint32_t* keys = kKeysInWorkspace
-                       ? p.keys_g + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * 2 * p.S_cap
-                       : keys_smem;
-  // pull the unit's scores into L2 in 16 KiB pieces (16-byte aligned, whole
-  // 16-byte blocks: the score array is one 256-byte aligned workspace region)
-  {
-    const uintptr_t a0 = reinterpret_cast<uintptr_t>(raw) & ~uintptr_t(15);
-    const uintptr_t a1 = (reinterpret_cast<uintptr_t>(raw + E) + 15) & ~uintptr_t(15);
-    const uintptr_t a = a0 + static_cast<uintptr_t>(threadIdx.x) * 16384;
-    if (a < a1) prefetch_l2_bulk(reinterpret_cast<const void*>(a), static_cast<uint32_t>(a1 - a < 16384 ? a1 - a : 16384));
+  uint32_t* keys = p.keys + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * p.key_stride;
+  for (int i = threadIdx.x; i < kBins0; i += kSelectThreads) sh.u.hist[i] = 0;
+  if (threadIdx.x == 0) {
+    sh.bcast[0] = static_cast<int>(0xFFFFFFFFu);  // key range, as unsigned
+    sh.bcast[1] = 0;
+    sh.ncand = 0;
   }
-  for (int i = threadIdx.x; i < kHistBins; i += kSelectThreads) sh.hist[i] = 0;
   __syncthreads();
   const bool aligned4 = (reinterpret_cast<uintptr_t>(raw) & 15u) == 0 && (p.S_cap & 3) == 0;
-  build_keys(keys, sh.hist, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV, aligned4);
+  build_keys(keys, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV, aligned4, sh);
   __syncthreads();
-  int d0, above;
-  find_bin(sh, kHistBins, k, d0, above);
+  const uint32_t klo = static_cast<uint32_t>(sh.bcast[0]), khi = static_cast<uint32_t>(sh.bcast[1]);
+  if (klo == khi) {  // every key equal: the lowest positions win the ties
+    for (int j = threadIdx.x; j < k; j += blockDim.x) idx[j] = j;
+    return;
+  }
+  // first digit: (key - klo) >> s, at most kBins0 bins over the keys' range
+  const int s_bits = max(0, 32 - __clz(static_cast<int>(khi - klo)) - 13);
+  range_hist(keys, E, klo, s_bits, sh.u.hist);
+  __syncthreads();
+  int d, above;
+  find_bin(sh.u.hist, kBins0, k, sh, d, above);  // ends with a barrier: hist may be overwritten
+  collect_candidates(keys, E, klo, s_bits, static_cast<uint32_t>(d), sh);
+  __syncthreads();
   uint32_t T;
   int need;
-  if (sh.hist[d0] <= p.cand_cap) {
-    select_by_candidates(keys, E, static_cast<uint32_t>(d0), k - above, sh,
-                         reinterpret_cast<int*>(keys + p.S_cap), T, need);
-  } else {  // a crowded first bin (e.g. many equal scores): radix passes over every key
-    radix_select(keys, E, k, sh, T, need);
-    count_segments(keys, E, T, sh);
-  }
+  if (sh.ncand <= kCandCap)
+    select_candidates(E, klo, s_bits, static_cast<uint32_t>(d), k - above, sh, T, need);
+  else  // a crowded bin: many equal keys
+    select_all_keys(keys, E, k, sh, T, need);
   write_kept(keys, E, k, T, need, sh, idx);
 }
 
 }  // namespace
 
-cudaError_t select_set_smem(size_t smem) {
-  return cudaFuncSetAttribute(select_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(smem));
-}
-
-cudaError_t launch_select(const SelectParams& p, int grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_select(const SelectParams& p, int grid, cudaStream_t s) {
   if (grid == 0) return cudaSuccess;
-  if (p.keys_g != nullptr)
-    select_kernel<true><<<grid, kSelectThreads, 0, s>>>(p);
-  else
-    select_kernel<false><<<grid, kSelectThreads, smem, s>>>(p);
+  select_kernel<<<grid, kSelectThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

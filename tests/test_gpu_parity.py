@@ -221,11 +221,10 @@ def test_h2o_recent_override_and_ties(torch, orc):
 
 
 def test_select_crowded_first_bin(torch, orc):
-    # At a 40K capacity the selection's candidate buffer holds fewer positions
-    # than these units have keys.  Layer 0 has zero queries, so all of its
-    # prefix scores tie and its units take the radix passes over every key
-    # (lower positions win the ties); layer 1 keeps live queries and takes the
-    # candidate path at full length.
+    # Long units whose candidate bin can hold more keys than the selection's
+    # candidate list.  Layer 0 has zero queries, so all of its prefix scores
+    # tie (lower positions win the ties); layer 1 keeps live queries and takes
+    # the candidate path at full length.
     wl = _custom([gen.SNAPKV, gen.H2O], [2048, 1024], [38000, 30000], W=8, H_q=4, H_kv=2, S_cap=40000, d=64)
     dev = device_workload(wl)
     dev[0][2].zero_()
@@ -233,9 +232,9 @@ def test_select_crowded_first_bin(torch, orc):
 
 
 def test_capacity_beyond_shared_memory(torch, orc):
-    # Up to 53,504 positions the selection holds a unit's keys in shared memory;
-    # past it, in the workspace.  Both sides of the bound, with sequences that
-    # fill the capacity, against the oracle.
+    # Capacities past what one CTA's shared memory could hold as keys (53,504
+    # positions at 4 bytes): the selection keeps them in the workspace at any
+    # capacity.  Sequences that fill the capacity, against the oracle.
     for s_cap in (53504, 65536):
         wl = _custom([gen.SNAPKV, gen.H2O], [512, 300], [s_cap, s_cap - 777], W=8, H_q=4, H_kv=2,
                      S_cap=s_cap, d=64)
