@@ -15,27 +15,27 @@
 // Output indices are ascending; unused slots hold -1.
 //
 // A unit takes a CTA of 256 threads, so that several units share an SM and
-// one unit's barriers and round trips overlap another's passes.  The keys (an
-// order-preserving uint32 image of the fp32 scores) go to the unit's row of a
-// workspace array, which stays in L2 between the passes:
-//   1. build the keys and find their range [lo, hi];
-//   2. histogram the first digit (key - lo) >> s, which splits the range into
-//      at most 8192 bins of 2^s keys (a unit's scores may crowd into a few
-//      per cent of one octave, or spread over many octaves: the range adapts
-//      the bins to either);
-//   3. find the bin holding the k-th largest key; each warp counts the keys
-//      of higher bins in its segment and appends that bin's keys (the
-//      candidates) to a shared list that reuses the histogram's space; radix
-//      passes of up to 9 bits over the candidates' s low bits fix the
-//      threshold key T and how many keys equal to T to keep, and the
-//      candidates' tallies give every warp segment its counts above and equal
-//      to T;
-//   4. one ordered pass writes the kept positions: a warp's slots follow those
-//      of the warps before it, and within a warp lanes hold four consecutive
-//      keys each, ranked by warp scans.
-// Equal keys everywhere take the first k positions directly; a candidate bin
-// with more keys than the list holds (many equal keys) takes four 8-bit radix
-// passes over every key instead.
+// one unit's barriers and round trips overlap another's passes.  Keys are an
+// order-preserving uint32 image of the fp32 (pooled) scores; they go to the
+// unit's row of a workspace array, which stays in L2 between the two passes:
+//   0. 1024 keys sampled at even strides give the bins: their range, widened
+//      by half on either side, split into 8192 bins of 2^s keys (a unit's
+//      scores may crowd into a few per cent of one octave, or spread over
+//      many octaves: the range adapts the bins to either);
+//   1. build the keys and histogram their bins (the two end bins also take
+//      every key outside the range);
+//   2. with the bin d holding the k-th largest key found, each warp walks its
+//      segment of the keys in order: keys of higher bins are kept for sure
+//      and their positions are staged, in order, at the start of the
+//      segment's row; keys of bin d (the candidates) go to the warp's list in
+//      shared memory with the count of sure positions before them;
+//   3. radix passes of up to 9 bits over the candidates fix the threshold key
+//      T and how many keys equal to T to keep (ties keep the lower position);
+//   4. every warp merges its staged positions and its kept candidates into
+//      its share of the output, after the shares of the warps before it.
+// An end bin, or a candidate list that overflows (many equal keys), takes the
+// general path instead: the keys are rebuilt, four 8-bit radix passes over
+// every key fix T, and one ordered pass writes the kept positions.
 #include "kvev_internal.cuh"
 
 namespace kvev {
@@ -43,35 +43,55 @@ namespace kvev {
 namespace {
 
 constexpr int kSW = kSelectThreads / 32;   // warps of a selection CTA
-constexpr int kBins0 = 8192;               // first digit: the keys' range in at most 8192 bins
-constexpr int kCandCap = kBins0 / 2;       // (position, key) pairs in the histogram's space
+constexpr int kBins0 = 8192;               // bins of the sampled range
+constexpr int kCandPerWarp = 320;          // candidates a warp's list holds
 constexpr int kBins1 = 512;                // candidate digits: up to 9 bits a pass
 constexpr int kSegKeys = 128;              // a warp block: four keys per lane
 constexpr int kSelectUnroll = 4;           // key blocks whose loads are in flight together
 
+struct CandLists {
+  uint32_t pos[kSW][kCandPerWarp];
+  uint32_t key[kSW][kCandPerWarp];
+  int sure[kSW][kCandPerWarp];  // sure positions of the segment before the candidate
+};
+
 struct __align__(16) SelShared {
   union {
     int hist[kBins0];
-    uint2 cand[kCandCap];
+    CandLists c;
   } u;
   int hist1[kBins1];
   int wsum[kSW];
-  int wgt[kSW];   // per warp segment: keys above T
-  int weq[kSW];   // per warp segment: keys equal to T
+  int wS[kSW];    // per warp segment: sure positions staged
+  int wC[kSW];    // per warp segment: candidates
+  int wgt[kSW];   // per warp segment: keys above T (general path) / candidates above T
+  int weq[kSW];   // per warp segment: keys (candidates) equal to T
   int bcast[2];
-  int ncand;
+  uint32_t rlo, rhi;  // sampled key range, then the candidates' key range
+  int overflow;
 };
 
 static_assert(sizeof(SelShared) <= 48 * 1024, "the selection's shared memory is static");
+static_assert(sizeof(CandLists) <= sizeof(int) * kBins0, "the candidate lists reuse the histogram");
 
 // Adds each valid lane's digit to the histogram, one shared-memory atomic per
-// distinct digit of the warp (the scores of a unit crowd into few bins).
-// Every lane of the warp must call it.
+// distinct digit of the warp (for digits that crowd into few bins).  Every
+// lane of the warp must call it.
 __device__ __forceinline__ void hist_add(int* hist, bool valid, uint32_t digit) {
   const uint32_t d = valid ? digit : 0xFFFFFFFFu;
   const uint32_t peers = __match_any_sync(0xffffffffu, d);
   if (valid && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[d], __popc(peers));
 }
+
+// The first digit: the bin of the key within [lo, lo + 8192 * 2^s); keys
+// below or above the range fall into the end bins.
+struct Binning {
+  uint32_t lo;
+  int s;
+  __device__ __forceinline__ uint32_t bin(uint32_t key) const {
+    return key < lo ? 0u : min((key - lo) >> s, static_cast<uint32_t>(kBins0 - 1));
+  }
+};
 
 // Inclusive warp scan.
 __device__ __forceinline__ int warp_incl(int x) {
@@ -142,209 +162,279 @@ __device__ __forceinline__ uint32_t pick(const uint4& v, int u) {
 }
 
 // ---------------------------------------------------------------------------
-// Pass 1: the keys and their range.  Keys past E in the last group of four are
-// written too (the row is padded); no later pass reads them.
+// Key generators: four consecutive keys of [0, E) from position i0 (a multiple
+// of four, i0 < E), in two halves -- load() issues the reads, keys() computes
+// -- so that a pass can have the next block's reads in flight while it works
+// on the current one.  Keys past E are computed but never used.
 // ---------------------------------------------------------------------------
-struct KeyRange {
-  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
-  __device__ __forceinline__ void add(uint32_t k, bool valid) {
-    if (valid) {
-      lo = min(lo, k);
-      hi = max(hi, k);
-    }
-  }
-};
 
-// Pooled keys from a 16-byte aligned score row: thread t of a round takes keys
-// 4t .. 4t+3, whose windows (P <= 9) lie in the three aligned 4-float chunks
-// starting at 4t - 4, 4t and 4t + 4.  Only chunks that start before E are read
-// (E <= S_cap, a multiple of 4, so none leaves the row); entries outside
-// [0, E) count as -inf (max) or 0 (avg).
+// Pooled keys from a 16-byte aligned score row (S_cap a multiple of 4): keys
+// i0 .. i0+3 have windows (P <= 9) inside the three aligned 4-float chunks
+// starting at i0 - 4, i0 and i0 + 4.  Only chunks that start before E are
+// read (none leaves the row); entries outside [0, E) count as -inf (max) or 0
+// (avg).  Avg pooling divides every window sum by the same p, so the sum
+// ranks the keys alike and is used instead.
 template <int P>
-__device__ __forceinline__ void build_pooled4(uint32_t* keys, const float* raw, int E, bool is_max,
-                                              KeyRange& kr) {
-  constexpr int h = P / 2;
-  static_assert(h <= 4, "the three chunks cover windows of up to 9");
-  const float fill = is_max ? -INFINITY : 0.f;
-  for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
-    const int i0 = b0 + 4 * threadIdx.x;  // first of this thread's four keys
-    float w[12];
+struct Pooled4 {
+  const float* raw;
+  int E;
+  bool is_max;
+  struct Regs {
+    float4 c[3];
+  };
+  __device__ __forceinline__ void load(int i0, Regs& r) const {
+    const float fill = is_max ? -INFINITY : 0.f;
 #pragma unroll
     for (int c = 0; c < 3; ++c) {
       const int st = i0 - 4 + 4 * c;
-      float4 v = make_float4(fill, fill, fill, fill);
-      if (st >= 0 && st < E) v = __ldg(reinterpret_cast<const float4*>(raw + st));  // neighbours' chunks: L1 hits
-      w[4 * c + 0] = st + 0 < E ? v.x : fill;
-      w[4 * c + 1] = st + 1 < E ? v.y : fill;
-      w[4 * c + 2] = st + 2 < E ? v.z : fill;
-      w[4 * c + 3] = st + 3 < E ? v.w : fill;
+      r.c[c] = make_float4(fill, fill, fill, fill);
+      if (st >= 0 && st < E) r.c[c] = __ldg(reinterpret_cast<const float4*>(raw + st));  // neighbours': L1
     }
-    uint32_t kq[4];
+  }
+  __device__ __forceinline__ void keys(int i0, const Regs& r, uint32_t (&kq)[4]) const {
+    constexpr int h = P / 2;
+    static_assert(h <= 4, "the three chunks cover windows of up to 9");
+    float w[12];
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+      w[4 * c + 0] = r.c[c].x;
+      w[4 * c + 1] = r.c[c].y;
+      w[4 * c + 2] = r.c[c].z;
+      w[4 * c + 3] = r.c[c].w;
+    }
+    if (i0 + 8 > E) {  // the last chunk may run past E
+      const float fill = is_max ? -INFINITY : 0.f;
+#pragma unroll
+      for (int j = 0; j < 12; ++j)
+        if (i0 - 4 + j >= E) w[j] = fill;
+    }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       float v = w[4 + u - h];
 #pragma unroll
       for (int j = 1; j < P; ++j) v = is_max ? fmaxf(v, w[4 + u - h + j]) : v + w[4 + u - h + j];
       kq[u] = float_key(v);
-      kr.add(kq[u], i0 + u < E);
     }
-    if (i0 < E) *reinterpret_cast<uint4*>(keys + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
   }
-}
+};
 
 // Raw keys (no pooling) from a 16-byte aligned score row.
-__device__ __forceinline__ void build_raw4(uint32_t* keys, const float* raw, int E, KeyRange& kr) {
-  for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
-    const int i0 = b0 + 4 * threadIdx.x;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (i0 < E) v = __ldg(reinterpret_cast<const float4*>(raw + i0));
-    const uint32_t kq[4] = {float_key(v.x), float_key(v.y), float_key(v.z), float_key(v.w)};
+struct Raw4 {
+  const float* raw;
+  int E;
+  struct Regs {
+    float4 v;
+  };
+  __device__ __forceinline__ void load(int i0, Regs& r) const {
+    r.v = __ldg(reinterpret_cast<const float4*>(raw + i0));
+  }
+  __device__ __forceinline__ void keys(int, const Regs& r, uint32_t (&kq)[4]) const {
+    kq[0] = float_key(r.v.x);
+    kq[1] = float_key(r.v.y);
+    kq[2] = float_key(r.v.z);
+    kq[3] = float_key(r.v.w);
+  }
+};
+
+// Any alignment and any odd pooling width: scalar loads, all in keys().
+struct Scalar4 {
+  const float* raw;
+  int E, h;
+  bool do_pool, is_max;
+  struct Regs {};
+  __device__ __forceinline__ uint32_t one(int i) const {
+    if (!do_pool) return float_key(raw[i]);
+    const int lo = max(i - h, 0), hi = min(i + h, E - 1);
+    float v = is_max ? -INFINITY : 0.f;
+    for (int j = lo; j <= hi; ++j) v = is_max ? fmaxf(v, raw[j]) : v + raw[j];
+    return float_key(v);
+  }
+  __device__ __forceinline__ void load(int, Regs&) const {}
+  __device__ __forceinline__ void keys(int i0, const Regs&, uint32_t (&kq)[4]) const {
 #pragma unroll
-    for (int u = 0; u < 4; ++u) kr.add(kq[u], i0 + u < E);
-    if (i0 < E) *reinterpret_cast<uint4*>(keys + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+    for (int u = 0; u < 4; ++u) kq[u] = i0 + u < E ? one(i0 + u) : 0u;
   }
+};
+
+template <class Gen>
+__device__ __forceinline__ void gen_keys(const Gen& gen, int i0, uint32_t (&kq)[4]) {
+  typename Gen::Regs r;
+  gen.load(i0, r);
+  gen.keys(i0, r, kq);
 }
 
-// Any alignment and any odd pooling width: one key per thread at a time.
-__device__ void build_scalar(uint32_t* keys, const float* raw, int E, int pool, bool do_pool, bool is_max,
-                             KeyRange& kr) {
-  const int h = pool / 2;
-  for (int i = threadIdx.x; i < E; i += kSelectThreads) {
-    float v;
-    if (!do_pool) {
-      v = raw[i];
-    } else if (is_max) {
-      v = -INFINITY;
-      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-      for (int j = lo; j <= hi; ++j) v = fmaxf(v, raw[j]);
-    } else {
-      v = 0.f;
-      const int lo = max(i - h, 0), hi = min(i + h, E - 1);
-      for (int j = lo; j <= hi; ++j) v += raw[j];
+// ---------------------------------------------------------------------------
+// Step 0: the bracket.  Sample keys: thread t takes the group of four at
+// 4 * floor(t * ceil(E / 4) / 256).  Their range is widened by half of it on
+// either side (at least 4096 key steps) and split into 8192 bins.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ Binning make_binning(uint32_t a, uint32_t b) {
+  const uint32_t m = max((b - a) / 2u, 4096u);
+  const uint32_t lo = a > m ? a - m : 0u;
+  const uint32_t hi = 0xFFFFFFFFu - b > m ? b + m : 0xFFFFFFFFu;
+  Binning bn;
+  bn.lo = lo;
+  bn.s = max(0, 32 - __clz(static_cast<int>(hi - lo)) - 13);  // (hi - lo) >> s < 8192
+  return bn;
+}
+
+struct Bracket {
+  Binning bn;
+  uint32_t lo_bin, hi_bin;  // candidates: bins lo_bin .. hi_bin; sure: bins above hi_bin
+};
+
+// The binning of the unit's keys from its sample.  Needs sh.rlo / sh.rhi
+// initialised.
+template <class Gen>
+__device__ Binning sample_binning(const Gen& gen, int E, SelShared& sh) {
+  const int groups = (E + 3) / 4;
+  const int i0 = 4 * static_cast<int>((static_cast<long long>(threadIdx.x) * groups) / kSelectThreads);
+  uint32_t kq[4];
+  gen_keys(gen, i0, kq);
+  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    if (i0 + u < E) {
+      lo = min(lo, kq[u]);
+      hi = max(hi, kq[u]);
     }
-    keys[i] = float_key(v);
-    kr.add(keys[i], true);
   }
-}
-
-// Builds the keys of [0, E) and returns their range in sh.bcast (lo, hi).
-__device__ void build_keys(uint32_t* keys, const float* raw, int E, int pool, int pool_type, bool do_pool,
-                           bool aligned4, SelShared& sh) {
-  const bool is_max = pool_type == KVEV_POOL_MAX;
-  KeyRange kr;
-  bool done = false;
-  if (aligned4) {
-    done = true;
-    if (!do_pool) build_raw4(keys, raw, E, kr);
-    else if (pool == 3) build_pooled4<3>(keys, raw, E, is_max, kr);
-    else if (pool == 5) build_pooled4<5>(keys, raw, E, is_max, kr);
-    else if (pool == 7) build_pooled4<7>(keys, raw, E, is_max, kr);
-    else if (pool == 9) build_pooled4<9>(keys, raw, E, is_max, kr);
-    else done = false;
-  }
-  if (!done) build_scalar(keys, raw, E, pool, do_pool, is_max, kr);
-  const uint32_t lo = __reduce_min_sync(0xffffffffu, kr.lo), hi = __reduce_max_sync(0xffffffffu, kr.hi);
+  lo = __reduce_min_sync(0xffffffffu, lo);
+  hi = __reduce_max_sync(0xffffffffu, hi);
   if ((threadIdx.x & 31) == 0) {
-    atomicMin(reinterpret_cast<unsigned*>(&sh.bcast[0]), lo);
-    atomicMax(reinterpret_cast<unsigned*>(&sh.bcast[1]), hi);
+    atomicMin(&sh.rlo, lo);
+    atomicMax(&sh.rhi, hi);
+  }
+  __syncthreads();
+  return make_binning(sh.rlo, sh.rhi);
+}
+
+// Step 1: every key of [0, E) into the unit's workspace row, and the
+// histogram of their bins.
+template <class Gen>
+__device__ void build_row_hist(const Gen& gen, uint32_t* row, int E, Binning bn, int* hist) {
+  typename Gen::Regs nxt;
+  int i0 = 4 * threadIdx.x;
+  if (i0 < E) gen.load(i0, nxt);
+  for (; i0 < E; i0 += 4 * kSelectThreads) {
+    const typename Gen::Regs cur = nxt;
+    if (i0 + 4 * kSelectThreads < E) gen.load(i0 + 4 * kSelectThreads, nxt);  // next reads go out first
+    uint32_t kq[4];
+    gen.keys(i0, cur, kq);
+    *reinterpret_cast<uint4*>(row + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (i0 + u < E) atomicAdd(&hist[bn.bin(kq[u])], 1);
   }
 }
 
-// Pass 2: histogram of the first digit (key - lo) >> s, which splits the keys'
-// range into at most kBins0 bins of 2^s keys each (plain atomics: keys spread
-// over the bins).
-__device__ void range_hist(const uint32_t* keys, int E, uint32_t lo, int s, int* hist) {
-  constexpr int R = kSelectUnroll;
-  for (int b0 = 0; b0 < E; b0 += 4 * R * kSelectThreads) {
-    uint4 kv[R];
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + (r * kSelectThreads + threadIdx.x) * 4;
-      kv[r] = i0 < E ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + (r * kSelectThreads + threadIdx.x) * 4;
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + u < E) atomicAdd(&hist[(pick(kv[r], u) - lo) >> s], 1);
-    }
+// Keys read back from the unit's workspace row.
+struct Stored4 {
+  const uint32_t* row;
+  struct Regs {
+    uint4 v;
+  };
+  __device__ __forceinline__ void load(int i0, Regs& r) const { r.v = ld_keys4(row, i0); }
+  __device__ __forceinline__ void keys(int, const Regs& r, uint32_t (&kq)[4]) const {
+    kq[0] = r.v.x;
+    kq[1] = r.v.y;
+    kq[2] = r.v.z;
+    kq[3] = r.v.w;
   }
-}
+};
 
 // ---------------------------------------------------------------------------
-// Pass 2 and the candidate radix passes.
+// Step 2: each warp walks its segment [lo, hi) of the keys in order.  Keys of
+// bins above the bracket are kept for sure: their positions are staged, in
+// order, at the start of the segment's row (a warp only overwrites entries of
+// positions it has passed, and has the next block's keys in registers).  Keys
+// inside the bracket (the candidates) go to the warp's list with the count of
+// sure positions before them.  A list that fills up sets sh.overflow.
 // ---------------------------------------------------------------------------
-
-// Each warp counts its segment's keys of first-digit bins above d (into wgt)
-// and appends the keys of bin d, with their positions, to the candidate list
-// (in no particular order; at most kCandCap are stored, ncand counts them all).
-__device__ void collect_candidates(const uint32_t* keys, int E, uint32_t lo_key, int s, uint32_t d,
-                                   SelShared& sh) {
+template <class Gen>
+__device__ void classify_pass(const Gen& gen, uint32_t* row, int E, const Bracket& br, SelShared& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
-  int gt = 0;
-  constexpr int R = kSelectUnroll;
-  for (int b0 = lo; b0 < hi; b0 += R * kSegKeys) {
-    uint4 kv[R];
+  int ns = 0, nc = 0;  // sure positions staged, candidates listed
+  typename Gen::Regs nxt;
+  if (lo + 4 * lane < hi) gen.load(lo + 4 * lane, nxt);
+  for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
+    const int i0 = b0 + 4 * lane;
+    const typename Gen::Regs cur = nxt;
+    if (i0 + kSegKeys < hi) gen.load(i0 + kSegKeys, nxt);  // the next block's reads go out first
+    uint32_t kq[4] = {0u, 0u, 0u, 0u};
+    if (i0 < hi) gen.keys(i0, cur, kq);
+    uint32_t sm = 0, cm = 0;
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + r * kSegKeys + 4 * lane;
-      kv[r] = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t q = br.bn.bin(kq[u]);
+      const bool valid = i0 + u < hi;
+      sm |= static_cast<uint32_t>(valid && q > br.hi_bin) << u;
+      cm |= static_cast<uint32_t>(valid && q >= br.lo_bin && q <= br.hi_bin) << u;
     }
+    if (!__any_sync(0xffffffffu, (sm | cm) != 0)) continue;
+    const int cs = __popc(sm), cc = __popc(cm);
+    const int is = warp_incl(cs), ic = warp_incl(cc);
+    int js = ns + is - cs, jc = nc + ic - cc;
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + r * kSegKeys + 4 * lane;
-      int c = 0;
-      uint32_t cmask = 0;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const bool valid = i0 + u < hi;
-        const uint32_t q = (pick(kv[r], u) - lo_key) >> s;
-        gt += valid && q > d;
-        const bool in = valid && q == d;
-        cmask |= static_cast<uint32_t>(in) << u;
-        c += in;
-      }
-      if (__any_sync(0xffffffffu, c)) {
-        const int incl = warp_incl(c);
-        int base = 0;
-        if (lane == 31) base = atomicAdd(&sh.ncand, incl);
-        base = __shfl_sync(0xffffffffu, base, 31) + incl - c;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          if (cmask & (1u << u)) {
-            if (base < kCandCap) sh.u.cand[base] = make_uint2(static_cast<uint32_t>(i0 + u), pick(kv[r], u));
-            ++base;
-          }
+    for (int u = 0; u < 4; ++u) {
+      if (sm & (1u << u)) row[lo + js++] = static_cast<uint32_t>(i0 + u);
+      if (cm & (1u << u)) {
+        if (jc < kCandPerWarp) {
+          sh.u.c.pos[warp][jc] = static_cast<uint32_t>(i0 + u);
+          sh.u.c.key[warp][jc] = kq[u];
+          sh.u.c.sure[warp][jc] = js;
         }
+        ++jc;
       }
     }
+    ns += __shfl_sync(0xffffffffu, is, 31);
+    nc += __shfl_sync(0xffffffffu, ic, 31);
   }
-  gt = warp_sum(gt);
   if (lane == 0) {
-    sh.wgt[warp] = gt;
-    sh.weq[warp] = 0;
+    sh.wS[warp] = ns;
+    sh.wC[warp] = nc;
+    if (nc > kCandPerWarp) sh.overflow = 1;
   }
 }
 
-// Threshold key T (the kk-th largest of the candidates, the keys of first-digit
-// bin d) and how many keys equal to T to keep, by radix passes of up to 9 bits
-// over the s low bits of key - lo_key; then each candidate above or equal to
-// T is tallied to its warp segment.
-__device__ void select_candidates(int E, uint32_t lo_key, int s, uint32_t d, int kk, SelShared& sh,
-                                  uint32_t& T, int& need) {
-  const int nc = sh.ncand;
-  uint32_t prefix = 0, mask = 0;  // over the s low bits
-  for (int r = s; r > 0;) {
+// Step 3: threshold key T (the kk-th largest candidate) and how many keys
+// equal to T to keep, by radix passes of up to 9 bits over key - (least
+// candidate key); then each warp counts its candidates above and equal to T.
+__device__ void select_candidates(int kk, SelShared& sh, uint32_t& T, int& need) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    sh.rlo = 0xFFFFFFFFu;
+    sh.rhi = 0u;
+  }
+  __syncthreads();
+  uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+  for (int i = lane; i < sh.wC[warp]; i += 32) {
+    lo = min(lo, sh.u.c.key[warp][i]);
+    hi = max(hi, sh.u.c.key[warp][i]);
+  }
+  lo = __reduce_min_sync(0xffffffffu, lo);
+  hi = __reduce_max_sync(0xffffffffu, hi);
+  if (lane == 0) {
+    atomicMin(&sh.rlo, lo);
+    atomicMax(&sh.rhi, hi);
+  }
+  __syncthreads();
+  const uint32_t clo = sh.rlo, span = sh.rhi - sh.rlo;
+  const int bits = span == 0 ? 0 : 32 - __clz(static_cast<int>(span));
+  uint32_t prefix = 0, mask = 0;  // over the low `bits` bits of key - clo
+  for (int r = bits; r > 0;) {
     const int nb = min(9, r), shift = r - nb;
     const uint32_t dm = (1u << nb) - 1u;
     for (int i = threadIdx.x; i < kBins1; i += kSelectThreads) sh.hist1[i] = 0;
     __syncthreads();
-    for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
-      const uint32_t v = sh.u.cand[c].y - lo_key;
-      if ((v & mask) == prefix) atomicAdd(&sh.hist1[(v >> shift) & dm], 1);
+    for (int c = threadIdx.x; c < kSW * kCandPerWarp; c += kSelectThreads) {
+      const int w = c / kCandPerWarp, i = c - w * kCandPerWarp;
+      if (i < sh.wC[w]) {
+        const uint32_t v = sh.u.c.key[w][i] - clo;
+        if ((v & mask) == prefix) atomicAdd(&sh.hist1[(v >> shift) & dm], 1);
+      }
     }
     __syncthreads();
     int digit, above;
@@ -354,16 +444,75 @@ __device__ void select_candidates(int E, uint32_t lo_key, int s, uint32_t d, int
     mask |= dm << shift;
     r = shift;
   }
-  T = lo_key + ((d << s) | prefix);
+  T = clo + prefix;
   need = kk;
-  const int seg = seg_len(E);
-  for (int c = threadIdx.x; c < nc; c += kSelectThreads) {
-    const uint2 e = sh.u.cand[c];
-    const int w = static_cast<int>(e.x) / seg;
-    if (e.y > T) atomicAdd(&sh.wgt[w], 1);
-    else if (e.y == T) atomicAdd(&sh.weq[w], 1);
+  int gt = 0, eq = 0;
+  for (int i = lane; i < sh.wC[warp]; i += 32) {
+    const uint32_t key = sh.u.c.key[warp][i];
+    gt += key > T;
+    eq += key == T;
+  }
+  gt = warp_sum(gt);
+  eq = warp_sum(eq);
+  if (lane == 0) {
+    sh.wgt[warp] = gt;
+    sh.weq[warp] = eq;
   }
   __syncthreads();
+}
+
+// Step 4: warp w's output share starts after the shares (sure positions plus
+// kept candidates) of the warps before it.  Its kept candidates go to
+// base + (sure positions before it) + (kept candidates before it); its sure
+// position j to base + j + (kept candidates with at most j sure positions
+// before them).
+__device__ void merge_write(const uint32_t* keys, int E, int k, int need, SelShared& sh, uint32_t T, int* out) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
+  int base = 0, eq_base = 0;
+  for (int w = 0; w < warp; ++w) {
+    base += sh.wS[w] + sh.wgt[w] + min(max(need - eq_base, 0), sh.weq[w]);
+    eq_base += sh.weq[w];
+  }
+  const int nc = sh.wC[warp];
+  int* sure = sh.u.c.sure[warp];
+  int nk = 0;  // kept candidates so far; their sure counts are compacted into sure[0 .. nk)
+  for (int i0 = 0; i0 < nc; i0 += 32) {
+    const int i = i0 + lane;
+    uint32_t key = 0, pos = 0;
+    int sb = 0;
+    if (i < nc) {
+      key = sh.u.c.key[warp][i];
+      pos = sh.u.c.pos[warp][i];
+      sb = sure[i];
+    }
+    const bool e = i < nc && key == T;
+    const uint32_t eb = __ballot_sync(0xffffffffu, e);
+    const bool keep = i < nc && (key > T || (e && eq_base + __popc(eb & lt) < need));
+    const uint32_t kb = __ballot_sync(0xffffffffu, keep);
+    const int ki = nk + __popc(kb & lt);
+    __syncwarp();  // every lane has read its entry before the compaction overwrites it
+    if (keep) {
+      if (base + sb + ki < k) out[base + sb + ki] = static_cast<int>(pos);
+      sure[ki] = sb;
+    }
+    __syncwarp();
+    nk += __popc(kb);
+    eq_base += __popc(eb);
+  }
+  const int seg = seg_len(E);
+  const int lo = min(warp * seg, E);
+  const int ns = sh.wS[warp];
+  for (int j = lane; j < ns; j += 32) {
+    const int pos = static_cast<int>(__ldcg(keys + lo + j));
+    int a = 0, b = nk;  // kept candidates with sure[] <= j: the first index with sure[] > j
+    while (a < b) {
+      const int m = (a + b) >> 1;
+      if (sure[m] <= j) a = m + 1;
+      else b = m;
+    }
+    if (base + j + a < k) out[base + j + a] = pos;
+  }
 }
 
 // The general path: four 8-bit radix passes over every key, then each warp
@@ -479,6 +628,58 @@ __device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int n
   }
 }
 
+// Every key of [0, E) into the unit's workspace row (the general path).
+template <class Gen>
+__device__ void build_row(const Gen& gen, uint32_t* row, int E) {
+  for (int i0 = 4 * threadIdx.x; i0 < E; i0 += 4 * kSelectThreads) {
+    uint32_t kq[4];
+    gen_keys(gen, i0, kq);
+    *reinterpret_cast<uint4*>(row + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+  }
+}
+
+// Top-k of the keys of [0, E) (1 <= k < E) into out[0 .. k), ascending.
+template <class Gen>
+__device__ void select_unit(const Gen& gen, uint32_t* row, int E, int k, SelShared& sh, int* out) {
+  for (int i = threadIdx.x; i < kBins0; i += kSelectThreads) sh.u.hist[i] = 0;
+  if (threadIdx.x == 0) {
+    sh.rlo = 0xFFFFFFFFu;
+    sh.rhi = 0u;
+    sh.overflow = 0;
+  }
+  __syncthreads();
+  const Binning bn = sample_binning(gen, E, sh);
+  build_row_hist(gen, row, E, bn, sh.u.hist);
+  __syncthreads();
+  int d, above;
+  find_bin(sh.u.hist, kBins0, k, sh, d, above);  // ends with a barrier
+  const int nd = sh.u.hist[d];
+  __syncthreads();  // every thread has read it before the candidate lists overwrite the histogram
+  // the end bins also hold keys outside the sampled range: not one prefix
+  bool fast = d > 0 && d < kBins0 - 1 && nd <= kSW * kCandPerWarp;
+  const bool staged = fast;
+  if (fast) {
+    const Bracket br{bn, static_cast<uint32_t>(d), static_cast<uint32_t>(d)};
+    classify_pass(Stored4{row}, row, E, br, sh);
+    __syncthreads();
+    fast = !sh.overflow;
+  }
+  uint32_t T;
+  int need;
+  if (fast) {
+    select_candidates(k - above, sh, T, need);
+    merge_write(row, E, k, need, sh, T, out);
+    return;
+  }
+  // the general path: many equal keys, or a sample that missed the k-th key
+  if (staged) {
+    build_row(gen, row, E);
+    __syncthreads();
+  }
+  select_all_keys(row, E, k, sh, T, need);
+  write_kept(row, E, k, T, need, sh, out);
+}
+
 __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kernel(const __grid_constant__ SelectParams p) {
   __shared__ SelShared sh;
   const int per_layer = p.B * p.H_kv;
@@ -528,37 +729,20 @@ __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kerne
     return;
   }
   const float* raw = ld.scores + static_cast<size_t>(rem) * p.S_cap;
-  uint32_t* keys = p.keys + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * p.key_stride;
-  for (int i = threadIdx.x; i < kBins0; i += kSelectThreads) sh.u.hist[i] = 0;
-  if (threadIdx.x == 0) {
-    sh.bcast[0] = static_cast<int>(0xFFFFFFFFu);  // key range, as unsigned
-    sh.bcast[1] = 0;
-    sh.ncand = 0;
-  }
-  __syncthreads();
+  uint32_t* row = p.keys + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * p.key_stride;
+  const bool do_pool = ld.method == KVEV_SNAPKV, is_max = p.pool_type == KVEV_POOL_MAX;
   const bool aligned4 = (reinterpret_cast<uintptr_t>(raw) & 15u) == 0 && (p.S_cap & 3) == 0;
-  build_keys(keys, raw, E, p.pool_kernel, p.pool_type, ld.method == KVEV_SNAPKV, aligned4, sh);
-  __syncthreads();
-  const uint32_t klo = static_cast<uint32_t>(sh.bcast[0]), khi = static_cast<uint32_t>(sh.bcast[1]);
-  if (klo == khi) {  // every key equal: the lowest positions win the ties
-    for (int j = threadIdx.x; j < k; j += blockDim.x) idx[j] = j;
-    return;
+  if (aligned4 && !do_pool) return select_unit(Raw4{raw, E}, row, E, k, sh, idx);
+  if (aligned4) {
+    switch (p.pool_kernel) {
+      case 3: return select_unit(Pooled4<3>{raw, E, is_max}, row, E, k, sh, idx);
+      case 5: return select_unit(Pooled4<5>{raw, E, is_max}, row, E, k, sh, idx);
+      case 7: return select_unit(Pooled4<7>{raw, E, is_max}, row, E, k, sh, idx);
+      case 9: return select_unit(Pooled4<9>{raw, E, is_max}, row, E, k, sh, idx);
+      default: break;
+    }
   }
-  // first digit: (key - klo) >> s, at most kBins0 bins over the keys' range
-  const int s_bits = max(0, 32 - __clz(static_cast<int>(khi - klo)) - 13);
-  range_hist(keys, E, klo, s_bits, sh.u.hist);
-  __syncthreads();
-  int d, above;
-  find_bin(sh.u.hist, kBins0, k, sh, d, above);  // ends with a barrier: hist may be overwritten
-  collect_candidates(keys, E, klo, s_bits, static_cast<uint32_t>(d), sh);
-  __syncthreads();
-  uint32_t T;
-  int need;
-  if (sh.ncand <= kCandCap)
-    select_candidates(E, klo, s_bits, static_cast<uint32_t>(d), k - above, sh, T, need);
-  else  // a crowded bin: many equal keys
-    select_all_keys(keys, E, k, sh, T, need);
-  write_kept(keys, E, k, T, need, sh, idx);
+  select_unit(Scalar4{raw, E, p.pool_kernel / 2, do_pool, is_max}, row, E, k, sh, idx);
 }
 
 }  // namespace
