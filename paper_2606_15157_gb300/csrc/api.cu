@@ -63,8 +63,8 @@ struct WsLayout {
          lam = 0, raw = 0, lse = 0, sel_keys = 0, total = 0;
 };
 
-// Entries of a selection key row: S_cap rounded up to whole 16-byte vectors.
-int sel_key_stride(int S_cap) { return (S_cap + 3) & ~3; }
+// Entries of a selection key row: S_cap rounded up to whole 128-key blocks.
+int sel_key_stride(int S_cap) { return (S_cap + 127) & ~127; }
 
 WsLayout ws_layout(const kvev_plan& p, int B, int S_cap) {
   WsLayout w;

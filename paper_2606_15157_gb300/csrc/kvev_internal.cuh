@@ -123,7 +123,7 @@ struct SelectParams {
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
   uint32_t* keys;     // workspace: [scoring unit][key_stride] selection keys
-  int key_stride;     // S_cap rounded up to a multiple of 4 (16-byte aligned rows)
+  int key_stride;     // S_cap rounded up to a multiple of 128 (whole transposed key blocks)
 };
 
 // Per-layer description of the decode arena.

@@ -17,7 +17,9 @@
 // A unit takes a CTA of 256 threads, so that several units share an SM and
 // one unit's barriers and round trips overlap another's passes.  Keys are an
 // order-preserving uint32 image of the fp32 (pooled) scores; they go to the
-// unit's row of a workspace array, which stays in L2 between the two passes:
+// unit's row of a workspace array (transposed in 128-key blocks, so that a
+// warp's ballots rank them by position), which stays in L2 between the two
+// passes:
 //   0. 1024 keys sampled at even strides give the bins: their range, widened
 //      by half on either side, split into 8192 bins of 2^s keys (a unit's
 //      scores may crowd into a few per cent of one octave, or spread over
@@ -46,8 +48,7 @@ constexpr int kSW = kSelectThreads / 32;   // warps of a selection CTA
 constexpr int kBins0 = 8192;               // bins of the sampled range
 constexpr int kCandPerWarp = 320;          // candidates a warp's list holds
 constexpr int kBins1 = 512;                // candidate digits: up to 9 bits a pass
-constexpr int kSegKeys = 128;              // a warp block: four keys per lane
-constexpr int kSelectUnroll = 4;           // key blocks whose loads are in flight together
+constexpr int kSegKeys = 128;              // a key block: four keys per lane
 
 struct CandLists {
   uint32_t pos[kSW][kCandPerWarp];
@@ -151,14 +152,31 @@ __device__ __forceinline__ int seg_len(int E) {
   return ((E + kSW - 1) / kSW + kSegKeys - 1) / kSegKeys * kSegKeys;
 }
 
-// Four consecutive keys from a 16-byte aligned key row (the row is padded to
-// a multiple of four entries, so the load never leaves it).
-__device__ __forceinline__ uint4 ld_keys4(const uint32_t* keys, int i0) {
-  return __ldcg(reinterpret_cast<const uint4*>(keys + i0));
+// A key row holds 128-key blocks, each transposed: the key of position
+// b + 32u + L (b a multiple of 128, L < 32, u < 4) sits at b + 4L + u, so that
+// one 16-byte load gives lane L its four keys of the block in position order
+// and a ballot per u ranks a warp's keys by position.  Rows are padded to
+// whole blocks.
+__device__ __forceinline__ int tpos(int i) { return (i & ~127) | ((i & 31) << 2) | ((i >> 5) & 3); }
+
+// Lane L's four keys of the block at b0: positions b0 + L + 32u.
+__device__ __forceinline__ uint4 ld_block_keys(const uint32_t* keys, int b0) {
+  return __ldcg(reinterpret_cast<const uint4*>(keys + b0 + 4 * (threadIdx.x & 31)));
 }
 
 __device__ __forceinline__ uint32_t pick(const uint4& v, int u) {
   return u == 0 ? v.x : u == 1 ? v.y : u == 2 ? v.z : v.w;
+}
+
+// Bulk prefetch of the floats [src, src + n) into L2, in 16 KiB pieces, one
+// per thread (the row is 16-byte aligned and padded to whole 16-byte blocks).
+__device__ __forceinline__ void prefetch_row_l2(const float* src, int n) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(src);
+  const uintptr_t a1 = (reinterpret_cast<uintptr_t>(src + n) + 15) & ~uintptr_t(15);
+  for (uintptr_t a = a0 + static_cast<uintptr_t>(threadIdx.x) * 16384; a < a1; a += 16384u * kSelectThreads) {
+    const uint32_t bytes = static_cast<uint32_t>(a1 - a < 16384 ? a1 - a : 16384);
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a), "r"(bytes) : "memory");
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -309,8 +327,8 @@ __device__ Binning sample_binning(const Gen& gen, int E, SelShared& sh) {
   return make_binning(sh.rlo, sh.rhi);
 }
 
-// Step 1: every key of [0, E) into the unit's workspace row, and the
-// histogram of their bins.
+// Step 1: every key of [0, E) into the unit's workspace row (transposed
+// blocks), and the histogram of their bins.
 template <class Gen>
 __device__ void build_row_hist(const Gen& gen, uint32_t* row, int E, Binning bn, int* hist) {
   typename Gen::Regs nxt;
@@ -321,27 +339,15 @@ __device__ void build_row_hist(const Gen& gen, uint32_t* row, int E, Binning bn,
     if (i0 + 4 * kSelectThreads < E) gen.load(i0 + 4 * kSelectThreads, nxt);  // next reads go out first
     uint32_t kq[4];
     gen.keys(i0, cur, kq);
-    *reinterpret_cast<uint4*>(row + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (i0 + u < E) atomicAdd(&hist[bn.bin(kq[u])], 1);
+    for (int u = 0; u < 4; ++u) {
+      if (i0 + u < E) {
+        row[tpos(i0 + u)] = kq[u];
+        atomicAdd(&hist[bn.bin(kq[u])], 1);
+      }
+    }
   }
 }
-
-// Keys read back from the unit's workspace row.
-struct Stored4 {
-  const uint32_t* row;
-  struct Regs {
-    uint4 v;
-  };
-  __device__ __forceinline__ void load(int i0, Regs& r) const { r.v = ld_keys4(row, i0); }
-  __device__ __forceinline__ void keys(int, const Regs& r, uint32_t (&kq)[4]) const {
-    kq[0] = r.v.x;
-    kq[1] = r.v.y;
-    kq[2] = r.v.z;
-    kq[3] = r.v.w;
-  }
-};
 
 // ---------------------------------------------------------------------------
 // Step 2: each warp walks its segment [lo, hi) of the keys in order.  Keys of
@@ -351,46 +357,38 @@ struct Stored4 {
 // inside the bracket (the candidates) go to the warp's list with the count of
 // sure positions before them.  A list that fills up sets sh.overflow.
 // ---------------------------------------------------------------------------
-template <class Gen>
-__device__ void classify_pass(const Gen& gen, uint32_t* row, int E, const Bracket& br, SelShared& sh) {
+__device__ void classify_pass(uint32_t* row, int E, const Bracket& br, SelShared& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   int ns = 0, nc = 0;  // sure positions staged, candidates listed
-  typename Gen::Regs nxt;
-  if (lo + 4 * lane < hi) gen.load(lo + 4 * lane, nxt);
+  uint4 nxt = make_uint4(0, 0, 0, 0);
+  if (lo < hi) nxt = ld_block_keys(row, lo);
   for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
-    const int i0 = b0 + 4 * lane;
-    const typename Gen::Regs cur = nxt;
-    if (i0 + kSegKeys < hi) gen.load(i0 + kSegKeys, nxt);  // the next block's reads go out first
-    uint32_t kq[4] = {0u, 0u, 0u, 0u};
-    if (i0 < hi) gen.keys(i0, cur, kq);
-    uint32_t sm = 0, cm = 0;
+    const uint4 cur = nxt;
+    if (b0 + kSegKeys < hi) nxt = ld_block_keys(row, b0 + kSegKeys);  // the next block's keys go out first
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const uint32_t q = br.bn.bin(kq[u]);
-      const bool valid = i0 + u < hi;
-      sm |= static_cast<uint32_t>(valid && q > br.hi_bin) << u;
-      cm |= static_cast<uint32_t>(valid && q >= br.lo_bin && q <= br.hi_bin) << u;
-    }
-    if (!__any_sync(0xffffffffu, (sm | cm) != 0)) continue;
-    const int cs = __popc(sm), cc = __popc(cm);
-    const int is = warp_incl(cs), ic = warp_incl(cc);
-    int js = ns + is - cs, jc = nc + ic - cc;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (sm & (1u << u)) row[lo + js++] = static_cast<uint32_t>(i0 + u);
-      if (cm & (1u << u)) {
+      const int p = b0 + 32 * u + lane;
+      const uint32_t q = br.bn.bin(pick(cur, u));
+      const bool valid = p < hi;
+      const bool sure = valid && q > br.hi_bin;
+      const bool cand = valid && q >= br.lo_bin && q <= br.hi_bin;
+      const uint32_t bs = __ballot_sync(0xffffffffu, sure), bc = __ballot_sync(0xffffffffu, cand);
+      const int js = ns + __popc(bs & lt);
+      if (sure) row[lo + js] = static_cast<uint32_t>(p);
+      if (cand) {
+        const int jc = nc + __popc(bc & lt);
         if (jc < kCandPerWarp) {
-          sh.u.c.pos[warp][jc] = static_cast<uint32_t>(i0 + u);
-          sh.u.c.key[warp][jc] = kq[u];
+          sh.u.c.pos[warp][jc] = static_cast<uint32_t>(p);
+          sh.u.c.key[warp][jc] = pick(cur, u);
           sh.u.c.sure[warp][jc] = js;
         }
-        ++jc;
       }
+      ns += __popc(bs);
+      nc += __popc(bc);
     }
-    ns += __shfl_sync(0xffffffffu, is, 31);
-    nc += __shfl_sync(0xffffffffu, ic, 31);
   }
   if (lane == 0) {
     sh.wS[warp] = ns;
@@ -518,18 +516,18 @@ __device__ void merge_write(const uint32_t* keys, int E, int k, int need, SelSha
 // The general path: four 8-bit radix passes over every key, then each warp
 // counts its segment's keys above and equal to T.
 __device__ void select_all_keys(const uint32_t* keys, int E, int k, SelShared& sh, uint32_t& T, int& need) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t prefix = 0, mask = 0;
   int kk = k;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += kSelectThreads) sh.hist1[i] = 0;
     __syncthreads();
-    for (int b0 = 0; b0 < E; b0 += 4 * kSelectThreads) {
-      const int i0 = b0 + 4 * threadIdx.x;
-      const uint4 kv = i0 < E ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+    for (int b0 = 128 * warp; b0 < E; b0 += 128 * kSW) {  // blocks dealt to the warps in turn
+      const uint4 kv = ld_block_keys(keys, b0);
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const uint32_t key = pick(kv, u);
-        const bool in = i0 + u < E && (key & mask) == prefix;
+        const bool in = b0 + 32 * u + lane < E && (key & mask) == prefix;
         hist_add(sh.hist1, in, (key >> shift) & 255u);
       }
     }
@@ -542,16 +540,14 @@ __device__ void select_all_keys(const uint32_t* keys, int E, int k, SelShared& s
   }
   T = prefix;
   need = kk;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   int gt = 0, eq = 0;
   for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
-    const int i0 = b0 + 4 * lane;
-    const uint4 kv = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
+    const uint4 kv = ld_block_keys(keys, b0);
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const bool valid = i0 + u < hi;
+      const bool valid = b0 + 32 * u + lane < hi;
       gt += valid && pick(kv, u) > T;
       eq += valid && pick(kv, u) == T;
     }
@@ -566,12 +562,14 @@ __device__ void select_all_keys(const uint32_t* keys, int E, int k, SelShared& s
 }
 
 // ---------------------------------------------------------------------------
-// Pass 4: ordered write of the kept positions of [0, E) to out[0..k): keys
-// above T, and the first `need` keys equal to T in position order.
+// The general path's ordered write of the kept positions of [0, E) to
+// out[0..k): keys above T, and the first `need` keys equal to T in position
+// order.
 // ---------------------------------------------------------------------------
 __device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int need, const SelShared& sh,
                            int* out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   int eq_base = 0, sel_base = 0;
@@ -580,61 +578,34 @@ __device__ void write_kept(const uint32_t* keys, int E, int k, uint32_t T, int n
     sel_base += sh.wgt[w] + min(max(need - eq_base, 0), e);
     eq_base += e;
   }
-  constexpr int R = kSelectUnroll;
-  for (int b0 = lo; b0 < hi; b0 += R * kSegKeys) {
-    uint4 kr[R];
+  for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
+    const uint4 kv = ld_block_keys(keys, b0);
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + r * kSegKeys + 4 * lane;
-      kr[r] = i0 < hi ? ld_keys4(keys, i0) : make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int i0 = b0 + r * kSegKeys + 4 * lane;
-      const uint4 kv = kr[r];
-      uint32_t gm = 0, em = 0;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const bool valid = i0 + u < hi;
-        gm |= static_cast<uint32_t>(valid && pick(kv, u) > T) << u;
-        em |= static_cast<uint32_t>(valid && pick(kv, u) == T) << u;
-      }
-      if (!__any_sync(0xffffffffu, gm | em)) continue;
-      // ranks of the keys equal to T, in position order
-      const int ce = __popc(em);
-      const int ie = warp_incl(ce);
-      int rank = eq_base + ie - ce;
-      uint32_t sm = gm;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        if (em & (1u << u)) {
-          if (rank < need) sm |= 1u << u;
-          ++rank;
-        }
-      }
-      const int cs = __popc(sm);
-      const int is = warp_incl(cs);
-      int slot = sel_base + is - cs;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        if (sm & (1u << u)) {
-          if (slot < k) out[slot] = i0 + u;
-          ++slot;
-        }
-      }
-      eq_base += __shfl_sync(0xffffffffu, ie, 31);
-      sel_base += __shfl_sync(0xffffffffu, is, 31);
+    for (int u = 0; u < 4; ++u) {
+      const int p = b0 + 32 * u + lane;
+      const bool valid = p < hi;
+      const bool g = valid && pick(kv, u) > T, e = valid && pick(kv, u) == T;
+      const uint32_t be = __ballot_sync(0xffffffffu, e);
+      const bool sel = g || (e && eq_base + __popc(be & lt) < need);
+      const uint32_t bsel = __ballot_sync(0xffffffffu, sel);
+      const int slot = sel_base + __popc(bsel & lt);
+      if (sel && slot < k) out[slot] = p;
+      eq_base += __popc(be);
+      sel_base += __popc(bsel);
     }
   }
 }
 
-// Every key of [0, E) into the unit's workspace row (the general path).
+// Every key of [0, E) into the unit's workspace row, transposed blocks (the
+// general path).
 template <class Gen>
 __device__ void build_row(const Gen& gen, uint32_t* row, int E) {
   for (int i0 = 4 * threadIdx.x; i0 < E; i0 += 4 * kSelectThreads) {
     uint32_t kq[4];
     gen_keys(gen, i0, kq);
-    *reinterpret_cast<uint4*>(row + i0) = make_uint4(kq[0], kq[1], kq[2], kq[3]);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (i0 + u < E) row[tpos(i0 + u)] = kq[u];
   }
 }
 
@@ -660,7 +631,7 @@ __device__ void select_unit(const Gen& gen, uint32_t* row, int E, int k, SelShar
   const bool staged = fast;
   if (fast) {
     const Bracket br{bn, static_cast<uint32_t>(d), static_cast<uint32_t>(d)};
-    classify_pass(Stored4{row}, row, E, br, sh);
+    classify_pass(row, E, br, sh);
     __syncthreads();
     fast = !sh.overflow;
   }
@@ -732,6 +703,7 @@ __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kerne
   uint32_t* row = p.keys + (static_cast<size_t>(ld.score_slot) * per_layer + rem) * p.key_stride;
   const bool do_pool = ld.method == KVEV_SNAPKV, is_max = p.pool_type == KVEV_POOL_MAX;
   const bool aligned4 = (reinterpret_cast<uintptr_t>(raw) & 15u) == 0 && (p.S_cap & 3) == 0;
+  if (aligned4) prefetch_row_l2(raw, E);  // the passes' score reads become L2 hits
   if (aligned4 && !do_pool) return select_unit(Raw4{raw, E}, row, E, k, sh, idx);
   if (aligned4) {
     switch (p.pool_kernel) {
