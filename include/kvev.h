@@ -240,10 +240,9 @@ KVEV_API int kvev_plan_scores_offset(const kvev_plan *plan, int B, int S_cap, in
  *   Any rule with b_l >= lens[s] keeps every position.
  * Top-k ties keep the lower position.
  * EINVAL on null/misaligned pointers or B < 0, S_cap < 1; ENOMEM if the
- * workspace is smaller than kvev_plan_query() reports.  The selection keeps
- * a unit's keys in shared memory up to S_cap = 53,504 (GB300's opt-in limit
- * per block); larger capacities keep them in the workspace, which then grows
- * by 8 bytes per position per (scoring layer, sequence, KV head). */
+ * workspace is smaller than kvev_plan_query() reports.  The workspace holds,
+ * among the rest, 4 bytes per position per (scoring layer, sequence, KV head)
+ * for the selection's keys (rows padded to whole 128-position blocks). */
 KVEV_API int kvev_evict_prefill(kvev_plan *plan, const void *const *K, const void *const *V,
                        const void *const *Q_win, const int32_t *lens_dev, int B, int S_cap,
                        void *out_K, void *out_V, int32_t *out_idx, int32_t *out_count,
@@ -267,6 +266,30 @@ KVEV_API int kvev_evict_prefill_scored(kvev_plan *plan, const void *const *K, co
                                        void *out_V, int32_t *out_idx, int32_t *out_count,
                                        float *h2o_state, void *workspace, size_t workspace_bytes,
                                        void *stream);
+
+/* kvev_evict_prefill with the window rows' softmax normalisers supplied by
+ * the caller: the fused form, where the caller's own prefill attention has
+ * already formed every query row's log-sum-exp (flash-attention-style kernels
+ * return it).  The window scores of Sec. 2.1's rules need each window row's
+ * normaliser over every visible key before any key's score is final; given
+ * them, the library's score kernel makes one pass over K instead of two.
+ *   lse_win[L]  host array of device pointers; for every SnapKV and H2O
+ *               layer fp32 [B][H_q][W]: entry (s, q, i) is
+ *               ln sum_{k <= t} exp(q_row . K[s][q / G][k] / sqrt(d)) for
+ *               the window row of query head q at position t = lens[s] - W + i
+ *               (the same scale and causal range as the scores; rows with
+ *               t < 0 are not read).  Entries of other layers are ignored.
+ *               4-byte aligned.
+ * Q_win is still read (the scores need the rows' logits).  Everything else
+ * as kvev_evict_prefill.  EINVAL if lse_win or an entry of a SnapKV / H2O
+ * layer is NULL or misaligned, or if the plan scores H2O layers over the
+ * whole prompt (kvev_plan_set_h2o_full_prompt). */
+KVEV_API int kvev_evict_prefill_lse(kvev_plan *plan, const void *const *K, const void *const *V,
+                                    const void *const *Q_win, const float *const *lse_win,
+                                    const int32_t *lens_dev, int B, int S_cap, void *out_K,
+                                    void *out_V, int32_t *out_idx, int32_t *out_count,
+                                    float *h2o_state, void *workspace, size_t workspace_bytes,
+                                    void *stream);
 
 /* Sec. 2.1 (H2O's original scoring): with on = 1, the prefill scores of the
  * plan's H2O layers accumulate the attention of every prompt query row,

@@ -557,13 +557,13 @@ int check_prefill_args(const kvev_plan& P, const void* const* K, const void* con
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
                const void* const* Q_win, const float* const* scores, const int32_t* lens_dev, int B,
                int S_cap, void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count,
-               float* h2o_state, void* workspace, cudaStream_t s);
+               float* h2o_state, void* workspace, cudaStream_t s, const float* const* lse_win = nullptr);
 
 int evict_prefill_impl(kvev_plan* plan, const void* const* K, const void* const* V,
                        const void* const* Q_win, const float* const* scores, const int32_t* lens_dev,
                        int B, int S_cap, void* out_K, void* out_V, int32_t* out_idx,
                        int32_t* out_count, float* h2o_state, void* workspace, size_t workspace_bytes,
-                       void* stream) {
+                       void* stream, const float* const* lse_win = nullptr) {
   if (!plan || B < 0 || S_cap < 1) return KVEV_EINVAL;
   kvev_plan& P = *plan;
   if (B == 0) return KVEV_OK;
@@ -576,8 +576,15 @@ int evict_prefill_impl(kvev_plan* plan, const void* const* K, const void* const*
   if (rc != KVEV_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   P.last_stream = s;
+  if (lse_win) {  // every scored layer needs its window rows' log-sum-exp
+    if (P.h2o_full) return KVEV_EINVAL;
+    for (int l = 0; l < P.L; ++l)
+      if (is_scoring(P.route_pre[l]) &&
+          (!lse_win[l] || (reinterpret_cast<uintptr_t>(lse_win[l]) & 3u)))
+        return KVEV_EINVAL;
+  }
   return evict_impl(P, P.ctx, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
-                    out_count, h2o_state, workspace, s);
+                    out_count, h2o_state, workspace, s, lse_win);
 }
 
 }  // namespace
@@ -600,6 +607,17 @@ extern "C" int kvev_evict_prefill_scored(kvev_plan* plan, const void* const* K, 
   if (!scores) return KVEV_EINVAL;
   return evict_prefill_impl(plan, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
                             out_count, h2o_state, workspace, workspace_bytes, stream);
+}
+
+extern "C" int kvev_evict_prefill_lse(kvev_plan* plan, const void* const* K, const void* const* V,
+                                      const void* const* Q_win, const float* const* lse_win,
+                                      const int32_t* lens_dev, int B, int S_cap, void* out_K,
+                                      void* out_V, int32_t* out_idx, int32_t* out_count,
+                                      float* h2o_state, void* workspace, size_t workspace_bytes,
+                                      void* stream) {
+  if (!lse_win) return KVEV_EINVAL;
+  return evict_prefill_impl(plan, K, V, Q_win, nullptr, lens_dev, B, S_cap, out_K, out_V, out_idx,
+                            out_count, h2o_state, workspace, workspace_bytes, stream, lse_win);
 }
 
 namespace {
@@ -632,7 +650,7 @@ int h2o_full_regs_ok(int d) {
 int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const* V,
                const void* const* Q_win, const float* const* scores, const int32_t* lens_dev, int B,
                int S_cap, void* out_K, void* out_V, int32_t* out_idx, int32_t* out_count,
-               float* h2o_state, void* workspace, cudaStream_t s) {
+               float* h2o_state, void* workspace, cudaStream_t s, const float* const* lse_win) {
   auto supplied = [&](int l) { return scores != nullptr && scores[l] != nullptr; };
   if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
   int64_t total_rows = 0;
@@ -764,12 +782,31 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
     sp.raw = reinterpret_cast<float*>(wsb + ws.raw);
     sp.wait_ns = P.wait_ns;
     sp.stall_unit = P.stall_unit;
+    sp.single = lse_win ? 1 : 0;
     score_grid = grid;
     score_smem = smem;
   }
   mark(KVEV_K_PROLOGUE, 0);
   pp.mode = full_prompt ? kScoreNoH2O : kScoreAll;
   if (launch_prologue(pp, s) != cudaSuccess) return KVEV_ECUDA;
+  if (lse_win && ws.n_units > 0) {  // the caller's normalisers: the score kernel makes one sweep
+    LseParams lp;
+    std::memset(&lp, 0, sizeof(lp));
+    for (int i = 0; i < n_slayers; ++i)
+      lp.lse[i] = supplied(P.score_layers[i]) ? nullptr : lse_win[P.score_layers[i]];
+    lp.n_units = ws.n_units;
+    lp.B = B;
+    lp.H_kv = P.H_kv;
+    lp.H_q = P.H_q;
+    lp.G = P.G;
+    lp.W = P.W;
+    lp.R = ws.R;
+    lp.R_pad = ws.R_pad;
+    lp.lens = lens_ok;
+    lp.lam = reinterpret_cast<float*>(wsb + ws.lam);
+    lp.ready = reinterpret_cast<int*>(wsb + ws.ready);
+    if (launch_lse_fill(lp, s) != cudaSuccess) return KVEV_ECUDA;
+  }
   mark(KVEV_K_PROLOGUE, 1);
   if (ws.n_units > 0) mark(KVEV_K_SCORE, 0);
   if (ws.n_units > 0 &&

@@ -105,6 +105,7 @@ struct ScoreParams {
   float* raw;         // [n_units][S_cap] window scores
   long long wait_ns;
   int stall_unit;
+  int single;         // 1: the normalisers are supplied (lse_fill_kernel); sweep 2 only
   // ---- whole-prompt H2O scoring (h2o_full.cu) ----
   int phase;          // 0: row pass (lse2 of every prompt row), 1: key pass (scores)
   int Pb;             // prompt positions per query block (G * Pb <= 256 rows)
@@ -114,6 +115,16 @@ struct ScoreParams {
   int nkt_max;        // 256-key super-tiles of a full-capacity unit
   int n_items;        // items of the pass: (nb_max or nkt_max) x H2O units
   float* lse;         // [H2O unit][G][S_cap] base-2 log-sum-exp of every prompt row
+};
+
+// The caller's window-row log-sum-exp (natural log, softmax scale included)
+// of each scoring layer, fp32 [B][H_q][W], into the units' normaliser rows.
+struct LseParams {
+  const float* lse[kMaxScoreLayers];  // null: the layer's scores are supplied instead
+  int n_units, B, H_kv, H_q, G, W, R, R_pad;
+  const int* lens;
+  float* lam;         // [n_units][R_pad] lse2 of the rows (+inf: no row)
+  int* ready;
 };
 
 struct SelectParams {
@@ -573,6 +584,7 @@ int h2o_full_smem_bytes(int d);
 int h2o_full_kernel_regs(int d);
 cudaError_t h2o_full_set_smem(int d, size_t smem);
 cudaError_t launch_h2o_full(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
+cudaError_t launch_lse_fill(const LseParams& p, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int grid, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s, int num_sms);
 }  // namespace kvev

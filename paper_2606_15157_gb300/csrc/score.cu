@@ -143,14 +143,22 @@ __device__ __forceinline__ void prefetch_item(const ScoreParams& p, int first, i
 // item j (j < J), then sweep 2 of item j - kLag (j >= kLag).  Sweep 2 of an
 // item runs kLag sweep-1 items after its own sweep 1, so the unit's row
 // normalisers (which need every chunk of the unit, some of them on other
-// CTAs) are almost always published by then.  Every entry loads its own Q
-// (buffer e mod 2 for entry e).
+// CTAs) are almost always published by then.  With the normalisers supplied
+// (single sweep), the entries are sweep 2 of items 0 .. J-1.  Every entry
+// loads its own Q (buffer e mod 2 for entry e).
 constexpr int kLag = 2;
 struct EntryIter {
   int J, j = 0, sweep = -1;
-  __device__ __forceinline__ explicit EntryIter(int J_) : J(J_) {}
+  bool single;
+  __device__ __forceinline__ EntryIter(int J_, bool single_) : J(J_), single(single_) {}
   // Next entry: item index jj (of this CTA) and sweep; false at the end.
   __device__ __forceinline__ bool next(int& jj, int& sw) {
+    if (single) {
+      if (++sweep >= J) return false;
+      jj = sweep;
+      sw = 1;
+      return true;
+    }
     for (;;) {
       if (++sweep == 2) {
         sweep = 0;
@@ -192,7 +200,7 @@ __device__ __forceinline__ void producer(const ScoreParams& p, const Smem& sm, i
   // Q of entry x goes into buffer x mod nq once entry x - nq has released it
   auto q_free = [&](uint32_t x) { return mbar_try_wait(&sm.qempty[x % nq], ((x / nq) & 1) ^ 1); };
   bool ok = true;
-  EntryIter ei(J);
+  EntryIter ei(J, p.single != 0);
   int jj, sw;
   for (uint32_t e = 0; ok && ei.next(jj, sw); ++e) {
     const int t = first + jj * stride;
@@ -267,7 +275,7 @@ __device__ __forceinline__ void mma_issuer(const ScoreParams& p, const Smem& sm,
   uint32_t st = 0, kph = 0;  // K stage ring: position and phase of the next super-tile
   uint32_t sl = 0, tph = 0;  // TMEM ring of two 256-column units: first slot and phase
   bool ok = true;
-  EntryIter ei(J);
+  EntryIter ei(J, p.single != 0);
   int jj, sw;
   for (uint32_t e = 0; ok && ei.next(jj, sw); ++e) {
     const int t = first + jj * stride;
@@ -394,7 +402,7 @@ __device__ __forceinline__ void softmax_wg(const ScoreParams& p, const Smem& sm,
   uint32_t q1 = 0, q2 = 0;  // sweep-1 / sweep-2 entries done
   bool ok = true;
 
-  EntryIter ei(J);
+  EntryIter ei(J, p.single != 0);
   int jj, sw;
   while (ei.next(jj, sw)) {
     // ---------------- sweep 1 ----------------
@@ -515,7 +523,7 @@ __device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, 
   const int lane = threadIdx.x & 31;
   const int nr = p.R_pad >> 5;
   uint32_t q1 = 0;
-  EntryIter ei(J);
+  EntryIter ei(J, p.single != 0);
   int jj, sw;
   while (ei.next(jj, sw)) {
     if (sw != 0) continue;
@@ -596,7 +604,7 @@ __device__ __forceinline__ void publisher(const ScoreParams& p, const Smem& sm, 
 __device__ __forceinline__ void lam_loader(const ScoreParams& p, const Smem& sm, int first, int stride, int J) {
   const int lane = threadIdx.x & 31;
   uint32_t q2 = 0;
-  EntryIter ei(J);
+  EntryIter ei(J, p.single != 0);
   int jj, sw;
   while (ei.next(jj, sw)) {
     if (sw != 1) continue;
@@ -775,7 +783,41 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
   if (tid == 0) p.chunk_start[p.n_units] = carry;
 }
 
+// ---------------------------------------------------------------------------
+// Supplied normalisers: the caller's log-sum-exp of every window row (the
+// softmax_lse of its own prefill attention), as -base-2 values in each
+// scored unit's normaliser row, the unit then marked ready.  One CTA per
+// scoring unit; rows that lie before the sequence start get +inf (no key
+// sees them).  Runs after the prologue, which clears the ready flags.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) lse_fill_kernel(const __grid_constant__ LseParams p) {
+  const int u = blockIdx.x;
+  const int per_layer = p.B * p.H_kv;
+  const int ls = u / per_layer;
+  const int rem = u - ls * per_layer;
+  const int s = rem / p.H_kv, h = rem - s * p.H_kv;
+  const int n = p.lens[s];
+  const float* lse = p.lse[ls];
+  if (lse == nullptr) return;  // a layer whose scores the caller supplies
+  constexpr float kInvLn2 = 1.4426950408889634f;
+  for (int r = threadIdx.x; r < p.R_pad; r += blockDim.x) {
+    const int g = r / p.W, i = r - g * p.W;
+    const bool valid = r < p.R && n - p.W + i >= 0;
+    p.lam[static_cast<size_t>(u) * p.R_pad + r] =
+        valid ? lse[(static_cast<size_t>(s) * p.H_q + h * p.G + g) * p.W + i] * kInvLn2 : INFINITY;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) st_release(&p.ready[u], 1);
+}
+
 }  // namespace
+
+cudaError_t launch_lse_fill(const LseParams& p, cudaStream_t s) {
+  if (p.n_units == 0) return cudaSuccess;
+  lse_fill_kernel<<<p.n_units, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
 
 int score_smem_bytes(int d, int q_rows, int q_bufs, int R_pad, int stages) {
   size_t koff, loff, roff, poff, boff;

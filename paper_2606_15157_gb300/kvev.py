@@ -31,7 +31,8 @@ EXPORTS = ["kvev_alloc_from_scores", "kvev_alloc_rescale", "kvev_plan_create",
            "kvev_plan_debug_stall_unit", "kvev_plan_scores_offset", "kvev_plan_enable_timing",
            "kvev_plan_last_timings", "kvev_evict_prefill_noalloc", "kvev_decode_query",
            "kvev_decode_layer", "kvev_decode_state_offsets", "kvev_decode_init",
-           "kvev_decode_step", "kvev_decode_step_attn", "kvev_evict_prefill_scored", "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
+           "kvev_decode_step", "kvev_decode_step_attn", "kvev_evict_prefill_scored", "kvev_evict_prefill_lse",
+           "kvev_profile_cosine", "kvev_score_ppl", "kvev_score_entropy",
            "kvev_route_toprank", "kvev_route_install", "kvev_plan_save", "kvev_plan_load",
            "kvev_plan_set_h2o_full_prompt"]
 KERNEL_NAMES = ["prologue", "score", "select", "gather"]
@@ -70,6 +71,8 @@ def load(path: str = LIB_PATH):
                                          vp, sz, vp]
         L.kvev_evict_prefill_scored.argtypes = [vp, vp, vp, vp, vp, vp, C.c_int, C.c_int, vp, vp, vp,
                                                 vp, vp, vp, sz, vp]
+        L.kvev_evict_prefill_lse.argtypes = [vp, vp, vp, vp, vp, vp, C.c_int, C.c_int, vp, vp, vp,
+                                             vp, vp, vp, sz, vp]
         L.kvev_status.argtypes = [vp, P(C.c_int)]
         L.kvev_plan_set_wait_limit.argtypes = [vp, i64]
         L.kvev_plan_debug_stall_unit.argtypes = [vp, C.c_int]
@@ -182,6 +185,19 @@ def kvev_evict_prefill_scored(handle, K_ptrs, V_ptrs, Q_ptrs, score_ptrs, lens_p
     return load().kvev_evict_prefill_scored(handle, Ka, Va, Qa, Sa, lens_ptr, B, S_cap, out_K, out_V,
                                             out_idx, out_count, h2o_state, workspace, workspace_bytes,
                                             stream)
+
+
+def kvev_evict_prefill_lse(handle, K_ptrs, V_ptrs, Q_ptrs, lse_ptrs, lens_ptr, B, S_cap, out_K, out_V,
+                           out_idx, out_count, h2o_state, workspace, workspace_bytes, stream) -> int:
+    """Pointer-level call with the caller's window-row log-sum-exp; returns the status code."""
+    Ln = len(K_ptrs)
+    arr = C.c_void_p * Ln
+    Ka, Va = arr(*K_ptrs), arr(*V_ptrs)
+    La = arr(*lse_ptrs) if lse_ptrs is not None else None
+    Qa = arr(*Q_ptrs) if Q_ptrs is not None else None
+    return load().kvev_evict_prefill_lse(handle, Ka, Va, Qa, La, lens_ptr, B, S_cap, out_K, out_V,
+                                         out_idx, out_count, h2o_state, workspace, workspace_bytes,
+                                         stream)
 
 
 NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -417,14 +433,27 @@ class Plan:
             "rows": rows,
         }
 
-    def evict_prefill(self, K, V, Q, lens, B, S_cap, bufs, stream=None, check=True, scores=None) -> int:
+    def evict_prefill(self, K, V, Q, lens, B, S_cap, bufs, stream=None, check=True, scores=None,
+                      lse=None) -> int:
         """K, V, Q: lists (per layer) of CUDA tensors or None; lens: int32 CUDA tensor.
         scores: optional per-layer fp32 [B][H_kv][S_cap] CUDA tensors (or None) that a
-        caller's own attention produced for SnapKV / H2O layers (kvev_evict_prefill_scored)."""
+        caller's own attention produced for SnapKV / H2O layers (kvev_evict_prefill_scored).
+        lse: optional per-layer fp32 [B][H_q][W] CUDA tensors (or None): the window rows'
+        log-sum-exp from the caller's prefill attention (kvev_evict_prefill_lse)."""
         import torch
         if stream is None:
             stream = torch.cuda.current_stream()
         ptr = lambda t: None if t is None else t.data_ptr()
+        if lse is not None:
+            rc = kvev_evict_prefill_lse(
+                self.handle, [ptr(k) for k in K], [ptr(v) for v in V],
+                [ptr(q) for q in Q] if Q is not None else None, [ptr(x) for x in lse], lens.data_ptr(),
+                B, S_cap, bufs["out_K"].data_ptr(), bufs["out_V"].data_ptr(), bufs["out_idx"].data_ptr(),
+                bufs["out_count"].data_ptr(), bufs["h2o_state"].data_ptr(), bufs["workspace"].data_ptr(),
+                bufs["workspace"].numel(), stream.cuda_stream)
+            if check:
+                _check(rc, "kvev_evict_prefill_lse")
+            return rc
         if scores is not None:
             rc = kvev_evict_prefill_scored(
                 self.handle, [ptr(k) for k in K], [ptr(v) for v in V],

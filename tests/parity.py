@@ -142,8 +142,9 @@ def check_unit(wl, l, s, h, n, res, gpu: GpuRun, K_rows, V_rows, stats=None):
         assert np.all(np.abs(st - ref) <= tol), f"{where}: H2O state off"
 
 
-def run_gpu(wl, layers_dev, lens_np, plan=None):
-    """Run kvev_evict_prefill on device tensors {l: (K, V, Q)}; returns (plan, bufs)."""
+def run_gpu(wl, layers_dev, lens_np, plan=None, lse=None):
+    """Run kvev_evict_prefill on device tensors {l: (K, V, Q)} (kvev_evict_prefill_lse
+    with the per-layer window-row log-sum-exp `lse`); returns (plan, bufs)."""
     import torch
     from paper_2606_15157_gb300 import kvev
     if plan is None:
@@ -153,7 +154,7 @@ def run_gpu(wl, layers_dev, lens_np, plan=None):
     K = [layers_dev[l][0] if l in layers_dev else None for l in range(wl.L)]
     V = [layers_dev[l][1] if l in layers_dev else None for l in range(wl.L)]
     Q = [layers_dev[l][2] if l in layers_dev else None for l in range(wl.L)]
-    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs)
+    plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, lse=lse)
     torch.cuda.synchronize()
     assert plan.status() == 0, "device status word set"
     return plan, bufs
@@ -164,10 +165,10 @@ def to_host_u16(t):
     return t.view(torch.int16).cpu().numpy().view(np.uint16)
 
 
-def check_workload(wl, layers_dev, lens_np, units=None, nthreads=0, stats=None):
+def check_workload(wl, layers_dev, lens_np, units=None, nthreads=0, stats=None, lse=None):
     """Run the GPU path on the whole workload and compare `units` (default: all)."""
     import oracle
-    plan, bufs = run_gpu(wl, layers_dev, lens_np)
+    plan, bufs = run_gpu(wl, layers_dev, lens_np, lse=lse)
     gpu = GpuRun(plan, wl, bufs, lens_np)
     if units is None:
         units = [(l, s, h) for l in range(wl.L) for s in range(wl.B) for h in range(wl.H_kv)]

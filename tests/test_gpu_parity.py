@@ -287,6 +287,57 @@ def test_supplied_scores(torch, orc):
         parity.check_unit(wl, l, s, h, n, res, gpu, Kr, Vr)
 
 
+def _window_lse(wl, dev, torch):
+    """The caller's prefill-attention normalisers: for every SnapKV / H2O layer,
+    fp32 [B][H_q][W] log-sum-exp of each window row over the keys it sees, from a
+    plain fp64 softmax of the same bf16 rows (the library never computes them in
+    this mode)."""
+    out = []
+    for l in range(wl.L):
+        if int(wl.route[l]) not in (gen.SNAPKV, gen.H2O):
+            out.append(None)
+            continue
+        lse = np.zeros((wl.B, wl.H_q, wl.W), np.float32)
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            if n == 0:
+                continue
+            Kh = gen.bf16_bits_to_f32(parity.to_host_u16(dev[l][0][s])).astype(np.float64)
+            Qh = gen.bf16_bits_to_f32(parity.to_host_u16(dev[l][2][s])).astype(np.float64)
+            t = n - wl.W + np.arange(wl.W)                     # positions of the window rows
+            for q in range(wl.H_q):
+                S = Qh[q] @ Kh[q // wl.G][:n].T / np.sqrt(wl.d)  # [W][n]
+                S[np.arange(n)[None, :] > t[:, None]] = -np.inf
+                m = S.max(axis=1)
+                ok = t >= 0
+                lse[s, q, ok] = (m[ok] + np.log(np.exp(S[ok] - m[ok, None]).sum(axis=1)))
+        out.append(torch.from_numpy(lse).cuda())
+    return out
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_supplied_lse(torch, orc, d):
+    # kvev_evict_prefill_lse: the window rows' log-sum-exp comes from the caller's
+    # own prefill attention, and the score kernel makes a single sweep over K.
+    # Ragged lengths (one shorter than the window, one not a multiple of the
+    # tile), SnapKV with max and avg pooling, H2O, a StreamingLLM and a FULL
+    # layer; every unit against the oracle, which forms its own normalisers.
+    routes = [gen.SNAPKV, gen.H2O, gen.STREAMING, gen.FULL, gen.SNAPKV]
+    for pool in ((7, gen.POOL_AVG), (5, gen.POOL_MAX)):
+        wl = _custom(routes, [64, 80, 64, 0, 100], [900, 1500, 11, 2100], W=16, d=d, pool=pool)
+        dev = device_workload(wl)
+        parity.check_workload(wl, dev, wl.lens, lse=_window_lse(wl, dev, torch))
+
+
+def test_supplied_lse_groups_and_windows(torch, orc):
+    # The same for R = G*W of 48 (a 16-column tail), 128 and 256 rows.
+    for (H_q, H_kv, W) in [(12, 4, 16), (8, 2, 32), (32, 8, 64)]:
+        wl = _custom([gen.SNAPKV, gen.H2O], [W + 37, 100], [700, 3000, 2 * W], W=W, H_q=H_q, H_kv=H_kv,
+                     pool=(7, gen.POOL_AVG))
+        dev = device_workload(wl)
+        parity.check_workload(wl, dev, wl.lens, lse=_window_lse(wl, dev, torch))
+
+
 def test_repeat_calls_identical(torch):
     wl = gen.config_tiny(1)
     dev = host_to_dev(torch, gen.host_tensors(wl))
