@@ -472,12 +472,16 @@ def run_ours(args, rank, world, local_rank):
     max_over_ranks, sum_over_ranks = rank_reducers(dist, "cuda")
 
     # ---- device-resident timed region ----
+    main_lse = None
+    if args.lse_supplied:  # the fused form's own line: no end-to-end or CPU arms
+        main_lse = window_lse_device(wl, K, Q)
+        args.no_e2e = args.no_cpu_baseline = True
     kvev.kvev_plan_enable_timing(plan.handle, True)
     for _ in range(args.warmup):
-        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream)
+        plan.evict_prefill(K, V, Q, lens, wl.B, wl.S_cap, bufs, stream, lse=main_lse)
     barrier()
     ms_local, kernel_ms, clocks, kernels_launched = time_prefill(plan, wl, K, V, Q, lens, bufs, stream,
-                                                                  args.steps, barrier, kvev)
+                                                                  args.steps, barrier, kvev, lse=main_lse)
     ms_step = max_over_ranks(ms_local)
     status = plan.status()
     assert status == kvev.OK, f"device status {status}"
@@ -539,14 +543,15 @@ def run_ours(args, rank, world, local_rank):
     sustained = None
     if not args.no_extras and not args.h2o_full_prompt:
         n_s = max(args.steps, int(np.ceil(500.0 / max(ms_step, 1e-3))))
-        ms_s, _, clk_s, _ = time_prefill(plan, wl, K, V, Q, lens, bufs, stream, n_s, barrier, kvev)
+        ms_s, _, clk_s, _ = time_prefill(plan, wl, K, V, Q, lens, bufs, stream, n_s, barrier, kvev,
+                                         lse=main_lse)
         ms_s = max_over_ranks(ms_s)
         assert plan.status() == kvev.OK
         sustained = {"value": all_bytes / (ms_s / 1e3) / 1e9, "unit": "GB/s", "ms_per_step": ms_s,
                      "steps": n_s, "device_seconds": n_s * ms_s / 1e3, "clocks": clk_s}
 
     extras = {}
-    if not args.no_extras and not args.h2o_full_prompt:
+    if not args.no_extras and not args.h2o_full_prompt and not args.lse_supplied:
         # the fused form: the window rows' normalisers come from the caller's own
         # prefill attention (kvev_evict_prefill_lse); one sweep over K
         lse = window_lse_device(wl, K, Q)
@@ -617,7 +622,8 @@ def run_ours(args, rank, world, local_rank):
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded; shapes of LLaMA-3.1-8B long-context workloads)",
-            "config": workload_config(wl, {"parallelism": f"independent batch per GPU x{world}"}),
+            "config": workload_config(wl, {"parallelism": f"independent batch per GPU x{world}",
+                                           **({"lse_supplied": True} if args.lse_supplied else {})}),
             "hbm_frac": {"of_measured": value / hbm_peak, "of_nominal_8TBs": value / NOMINAL_HBM_GBS},
             # tokens dropped from a layer's cache, counted once per (sequence,
             # layer) and once per (sequence, layer, KV head): every head keeps
@@ -968,6 +974,8 @@ def main():
                          "in the decode workload (profiling)")
     ap.add_argument("--h2o-full-prompt", action="store_true",
                     help="H2O layers score every prompt query row (reports causal-attention TFLOP/s)")
+    ap.add_argument("--lse-supplied", action="store_true",
+                    help="the window rows' log-sum-exp is supplied (kvev_evict_prefill_lse): one score sweep")
     ap.add_argument("--decode-attn", action="store_true",
                     help="decode workload: the caller supplies the attention (kvev_decode_step_attn)")
     ap.add_argument("--e2e-steps", type=int, default=8)
