@@ -176,6 +176,55 @@ def test_long_context_fixed_32k_sampled(torch, orc):
         assert np.all(np.diff(blk, axis=1) > 0)
 
 
+def _window_lse_device(wl, dev, torch):
+    """A caller's prefill-attention normalisers at full size: per SnapKV / H2O layer
+    fp32 [B][H_q][W] log-sum-exp of each window row over the keys it sees, from a
+    plain fp32 torch softmax on the device."""
+    import math
+    tf32 = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    out = []
+    for l in range(wl.L):
+        if int(wl.route[l]) not in (gen.SNAPKV, gen.H2O):
+            out.append(None)
+            continue
+        K, _, Q = dev[l]
+        lse = torch.zeros((wl.B, wl.H_q, wl.W), dtype=torch.float32, device="cuda")
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            t = n - wl.W + torch.arange(wl.W, device="cuda")
+            mask = torch.arange(n, device="cuda")[None, :] > t[:, None]
+            for h in range(wl.H_kv):
+                S = torch.matmul(Q[s, h * wl.G:(h + 1) * wl.G].float(), K[s, h, :n].float().T) / math.sqrt(wl.d)
+                S.masked_fill_(mask[None], float("-inf"))
+                lse[s, h * wl.G:(h + 1) * wl.G] = torch.logsumexp(S, dim=-1)
+        out.append(lse)
+    torch.backends.cuda.matmul.allow_tf32 = tf32
+    return out
+
+
+def test_long_context_supplied_lse_sampled(torch, orc):
+    # The headline workload through kvev_evict_prefill_lse (one score sweep), the
+    # window rows' log-sum-exp from the caller's attention (plain fp32 torch on the
+    # device): sampled units of every rule against the oracle, which forms its own
+    # normalisers, and every scored unit's window-row mass.
+    wl = gen.config_long(kvev_alloc, seed=0)
+    wl_o = gen.config_long(oracle_alloc, seed=0)
+    assert np.array_equal(wl.budget, wl_o.budget)
+    dev = device_workload(wl)
+    lse = _window_lse_device(wl, dev, torch)
+    stats = {}
+    plan, bufs, gpu = parity.check_workload(wl_o, dev, wl.lens, units=_sample_units(wl, 8, 2), stats=stats,
+                                            nthreads=os.cpu_count(), lse=lse)
+    print("long, supplied lse, sampled", stats)
+    for l in range(wl.L):
+        if wl.route[l] in (gen.SNAPKV, gen.H2O):
+            for s in range(wl.B):
+                n = int(wl.lens[s])
+                tot = gpu.scores[l][s, :, :n].astype(np.float64).sum(axis=1)
+                assert np.allclose(tot, wl.W, rtol=1e-3)  # each window row's softmax sums to 1
+
+
 def _custom(L_routes, budgets, lens, W=16, d=128, H_q=8, H_kv=2, S_cap=None, pool=(5, gen.POOL_MAX),
             seed=7, sink=4, h2o_recent=-1):
     lens = np.asarray(lens, np.int32)
