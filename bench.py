@@ -377,7 +377,7 @@ def window_lse_device(wl, K, Q):
     out = []
     scale = 1.0 / math.sqrt(wl.d)
     for l in range(wl.L):
-        if wl.route[l] not in (gen.SNAPKV, gen.H2O):
+        if wl.route[l] not in (gen.SNAPKV, gen.H2O) or Q[l] is None:
             out.append(None)
             continue
         lse = torch.zeros((wl.B, wl.H_q, wl.W), dtype=torch.float32, device="cuda")
@@ -391,6 +391,36 @@ def window_lse_device(wl, K, Q):
                 S.masked_fill_(mask[None], float("-inf"))
                 lse[s, h * wl.G:(h + 1) * wl.G] = torch.logsumexp(S, dim=-1)
         out.append(lse)
+    torch.backends.cuda.matmul.allow_tf32 = tf32
+    torch.cuda.synchronize()
+    return out
+
+
+def prompt_lse_device(wl, K, Q, rows=1024):
+    """Every prompt row's log-sum-exp for the H2O layers scored over the whole
+    prompt (Q[l] is then [B][H_q][S_cap][d]): fp32 [B][H_q][S_cap], the layout
+    a flash-attention prefill returns; plain fp32 torch, row blocks of `rows`."""
+    import torch
+    tf32 = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    scale = 1.0 / math.sqrt(wl.d)
+    out = {}
+    for l in range(wl.L):
+        if wl.route[l] != gen.H2O:
+            continue
+        lse = torch.zeros((wl.B, wl.H_q, wl.S_cap), dtype=torch.float32, device="cuda")
+        for s in range(wl.B):
+            n = int(wl.lens[s])
+            for h in range(wl.H_kv):
+                k = K[l][s, h, :n].float()
+                for t0 in range(0, n, rows):
+                    t1 = min(n, t0 + rows)
+                    q = Q[l][s, h * wl.G:(h + 1) * wl.G, t0:t1].float()        # [G][r][d]
+                    S = torch.matmul(q, k[:t1].T) * scale                      # [G][r][t1]
+                    t = torch.arange(t0, t1, device="cuda")
+                    S.masked_fill_(torch.arange(t1, device="cuda")[None, :] > t[:, None], float("-inf"))
+                    lse[s, h * wl.G:(h + 1) * wl.G, t0:t1] = torch.logsumexp(S, dim=-1)
+        out[l] = lse
     torch.backends.cuda.matmul.allow_tf32 = tf32
     torch.cuda.synchronize()
     return out
@@ -474,7 +504,16 @@ def run_ours(args, rank, world, local_rank):
     # ---- device-resident timed region ----
     main_lse = None
     if args.lse_supplied:  # the fused form's own line: no end-to-end or CPU arms
-        main_lse = window_lse_device(wl, K, Q)
+        if args.h2o_full_prompt:  # the window kernel's layers (SnapKV) need only the window rows
+            Q_win_snap = [Q[l] if wl.route[l] == gen.SNAPKV else None for l in range(wl.L)]
+            main_lse = [None] * wl.L
+            for l, x in enumerate(window_lse_device(wl, K, Q_win_snap)):
+                if wl.route[l] == gen.SNAPKV:
+                    main_lse[l] = x
+            for l, x in prompt_lse_device(wl, K, Q).items():
+                main_lse[l] = x
+        else:
+            main_lse = window_lse_device(wl, K, Q)
         args.no_e2e = args.no_cpu_baseline = True
     kvev.kvev_plan_enable_timing(plan.handle, True)
     for _ in range(args.warmup):

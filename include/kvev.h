@@ -278,12 +278,15 @@ KVEV_API int kvev_evict_prefill_scored(kvev_plan *plan, const void *const *K, co
  *               ln sum_{k <= t} exp(q_row . K[s][q / G][k] / sqrt(d)) for
  *               the window row of query head q at position t = lens[s] - W + i
  *               (the same scale and causal range as the scores; rows with
- *               t < 0 are not read).  Entries of other layers are ignored.
- *               4-byte aligned.
+ *               t < 0 are not read).  For the H2O layers of a plan that
+ *               scores them over the whole prompt
+ *               (kvev_plan_set_h2o_full_prompt): fp32 [B][H_q][S_cap], the
+ *               same for every prompt row t < lens[s] (the layout of a
+ *               flash-attention softmax_lse), and the row pass is skipped.
+ *               Entries of other layers are ignored.  4-byte aligned.
  * Q_win is still read (the scores need the rows' logits).  Everything else
  * as kvev_evict_prefill.  EINVAL if lse_win or an entry of a SnapKV / H2O
- * layer is NULL or misaligned, or if the plan scores H2O layers over the
- * whole prompt (kvev_plan_set_h2o_full_prompt). */
+ * layer is NULL or misaligned. */
 KVEV_API int kvev_evict_prefill_lse(kvev_plan *plan, const void *const *K, const void *const *V,
                                     const void *const *Q_win, const float *const *lse_win,
                                     const int32_t *lens_dev, int B, int S_cap, void *out_K,

@@ -576,8 +576,7 @@ int evict_prefill_impl(kvev_plan* plan, const void* const* K, const void* const*
   if (rc != KVEV_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   P.last_stream = s;
-  if (lse_win) {  // every scored layer needs its window rows' log-sum-exp
-    if (P.h2o_full) return KVEV_EINVAL;
+  if (lse_win) {  // every scored layer needs its rows' log-sum-exp
     for (int l = 0; l < P.L; ++l)
       if (is_scoring(P.route_pre[l]) &&
           (!lse_win[l] || (reinterpret_cast<uintptr_t>(lse_win[l]) & 3u)))
@@ -792,8 +791,10 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   if (lse_win && ws.n_units > 0) {  // the caller's normalisers: the score kernel makes one sweep
     LseParams lp;
     std::memset(&lp, 0, sizeof(lp));
-    for (int i = 0; i < n_slayers; ++i)
-      lp.lse[i] = supplied(P.score_layers[i]) ? nullptr : lse_win[P.score_layers[i]];
+    for (int i = 0; i < n_slayers; ++i) {  // H2O layers scored over the whole prompt: below
+      const int l = P.score_layers[i];
+      lp.lse[i] = supplied(l) || (full_prompt && P.route_pre[l] == KVEV_H2O) ? nullptr : lse_win[l];
+    }
     lp.n_units = ws.n_units;
     lp.B = B;
     lp.H_kv = P.H_kv;
@@ -837,7 +838,11 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
       if (h2o_full_set_smem(P.d, fsmem) != cudaSuccess) return KVEV_ECUDA;
       D.h2o_full_smem_set = fsmem;
     }
-    for (int phase = 0; phase < 2; ++phase) {
+    if (lse_win) {  // the caller's every-row normalisers replace the row pass
+      for (int j = 0; j < fp.n_h2o; ++j) fp.lse_src[j] = lse_win[P.score_layers[fp.h2o_slot[j]]];
+      if (launch_lse_rows_fill(fp, s) != cudaSuccess) return KVEV_ECUDA;
+    }
+    for (int phase = lse_win ? 1 : 0; phase < 2; ++phase) {
       fp.phase = phase;
       fp.n_items = static_cast<int>(units * (phase == 0 ? fp.nb_max : fp.nkt_max));
       if (launch_h2o_full(fp, P.d, std::min(D.num_sms, fp.n_items), fsmem, s) != cudaSuccess)

@@ -509,6 +509,24 @@ __global__ void __launch_bounds__(kScoreThreads, 1) h2o_full_kernel(const __grid
   }
 }
 
+// The caller's log-sum-exp of every prompt row (the softmax_lse its own
+// prefill attention returns, natural log, fp32 [B][H_q][S_cap]) into the key
+// pass's base-2 rows, in place of the row pass.  One CTA per H2O unit.
+__global__ void __launch_bounds__(256) lse_rows_fill_kernel(const __grid_constant__ ScoreParams p) {
+  const int per_layer = p.B * p.H_kv;
+  const int hu = blockIdx.x;
+  const int li = hu / per_layer;
+  const int rem = hu - li * per_layer;
+  const int s = rem / p.H_kv, h = rem - s * p.H_kv;
+  const int n = p.lens[s];
+  const float* src = p.lse_src[li] + (static_cast<size_t>(s) * p.H_q + static_cast<size_t>(h) * p.G) * p.S_cap;
+  float* dst = p.lse + static_cast<size_t>(hu) * p.G * p.S_cap;
+  constexpr float kInvLn2 = 1.4426950408889634f;
+  for (int g = 0; g < p.G; ++g)
+    for (int t = threadIdx.x; t < n; t += blockDim.x)
+      dst[static_cast<size_t>(g) * p.S_cap + t] = __ldg(src + static_cast<size_t>(g) * p.S_cap + t) * kInvLn2;
+}
+
 }  // namespace
 
 int h2o_full_smem_bytes(int d) {
@@ -530,6 +548,13 @@ cudaError_t h2o_full_set_smem(int d, size_t smem) {
                                 static_cast<int>(smem));
   return cudaFuncSetAttribute(h2o_full_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(smem));
+}
+
+cudaError_t launch_lse_rows_fill(const ScoreParams& p, cudaStream_t s) {
+  const int units = p.n_h2o * p.B * p.H_kv;
+  if (units == 0) return cudaSuccess;
+  lse_rows_fill_kernel<<<units, 256, 0, s>>>(p);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_h2o_full(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s) {

@@ -115,6 +115,8 @@ struct ScoreParams {
   int nkt_max;        // 256-key super-tiles of a full-capacity unit
   int n_items;        // items of the pass: (nb_max or nkt_max) x H2O units
   float* lse;         // [H2O unit][G][S_cap] base-2 log-sum-exp of every prompt row
+  const float* lse_src[kMaxScoreLayers];  // the caller's every-row log-sum-exp per H2O layer
+                      // (fp32 [B][H_q][S_cap], natural log), or null: the row pass computes it
 };
 
 // The caller's window-row log-sum-exp (natural log, softmax scale included)
@@ -585,6 +587,7 @@ int h2o_full_kernel_regs(int d);
 cudaError_t h2o_full_set_smem(int d, size_t smem);
 cudaError_t launch_h2o_full(const ScoreParams& p, int d, int grid, size_t smem, cudaStream_t s);
 cudaError_t launch_lse_fill(const LseParams& p, cudaStream_t s);
+cudaError_t launch_lse_rows_fill(const ScoreParams& p, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int grid, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s, int num_sms);
 }  // namespace kvev

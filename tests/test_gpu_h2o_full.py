@@ -40,8 +40,23 @@ GEOMETRIES = [
 ]
 
 
+def _rows_lse(Kh, Qh, n, t_rows, d):
+    """ln sum_{k <= t} exp(q_t . k / sqrt(d)) for the query rows Qh [rows][d] at
+    positions t_rows, from the bf16 bits in fp64 (a caller's attention)."""
+    Kf = gen.bf16_bits_to_f32(Kh[:n]).astype(np.float64)
+    Qf = gen.bf16_bits_to_f32(Qh).astype(np.float64)
+    S = Qf @ Kf.T / np.sqrt(d)
+    S[np.arange(n)[None, :] > t_rows[:, None]] = -np.inf
+    m = S.max(axis=1)
+    out = np.zeros(len(t_rows), np.float32)
+    ok = t_rows >= 0
+    out[ok] = m[ok] + np.log(np.exp(S[ok] - m[ok, None]).sum(axis=1))
+    return out
+
+
+@pytest.mark.parametrize("supplied_lse", [False, True])
 @pytest.mark.parametrize("H_q,H_kv,d,lens", GEOMETRIES)
-def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens):
+def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens, supplied_lse):
     from paper_2606_15157_gb300 import kvev
     import oracle
     route = [gen.H2O, gen.SNAPKV, gen.H2O]
@@ -63,10 +78,29 @@ def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens):
     V = [dev[l][1] for l in range(wl.L)]
     Q = [dev[l][2] for l in range(wl.L)]
 
+    lse = None
+    if supplied_lse:
+        # kvev_evict_prefill_lse: the caller's attention gives every prompt row's
+        # log-sum-exp for the H2O layers ([B][H_q][S_cap]; the row pass is
+        # skipped) and the window rows' for the SnapKV layer ([B][H_q][W])
+        lse = []
+        for l in range(wl.L):
+            rows = wl.S_cap if route[l] == gen.H2O else wl.W
+            x = np.zeros((wl.B, wl.H_q, rows), np.float32)
+            for s in range(wl.B):
+                n = int(lens[s])
+                if n == 0:
+                    continue
+                Kh = parity.to_host_u16(dev[l][0][s])
+                t = np.arange(n) if route[l] == gen.H2O else n - wl.W + np.arange(wl.W)
+                for q in range(wl.H_q):
+                    Qq = q_full[l][s, q, :n] if route[l] == gen.H2O else parity.to_host_u16(dev[l][2][s])[q]
+                    x[s, q, :len(t)] = _rows_lse(Kh[q // wl.G], Qq, n, t, wl.d)
+            lse.append(torch.from_numpy(x).cuda())
     plan = kvev.Plan(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel, wl.pool_type,
                      wl.sink, wl.recent, wl.h2o_recent, h2o_full_prompt=True)
     bufs = plan.buffers(wl.B, wl.S_cap)
-    plan.evict_prefill(K, V, Q, lens_dev, wl.B, wl.S_cap, bufs)
+    plan.evict_prefill(K, V, Q, lens_dev, wl.B, wl.S_cap, bufs, lse=lse)
     torch.cuda.synchronize()
     assert plan.status() == kvev.OK
     gpu = parity.GpuRun(plan, wl, bufs, np.asarray(lens))
@@ -93,6 +127,8 @@ def test_h2o_full_prompt_scores_and_selection(torch, H_q, H_kv, d, lens):
     for (l, s, h, n, Kr, Vr), res in zip(meta, results):
         parity.check_unit(wl, l, s, h, n, res, gpu, Kr, Vr)
 
+    if supplied_lse:
+        return  # the check below compares two library-formed normalisers bit for bit
     # the SnapKV layer's window scores do not depend on the option
     ref = kvev.Plan(wl.L, wl.H_q, wl.H_kv, wl.d, wl.route, wl.budget, wl.W, wl.pool_kernel, wl.pool_type,
                     wl.sink, wl.recent, wl.h2o_recent)
