@@ -16,28 +16,31 @@
 //
 // A unit takes a CTA of 256 threads, so that several units share an SM and
 // one unit's barriers and round trips overlap another's passes.  Keys are an
-// order-preserving uint32 image of the fp32 (pooled) scores; they go to the
-// unit's row of a workspace array (transposed in 128-key blocks, so that a
-// warp's ballots rank them by position), which stays in L2 between the two
-// passes:
+// order-preserving uint32 image of the fp32 (pooled) scores.  The unit's row
+// of a workspace array holds, between the two passes, each key's 16-bit bin
+// (transposed in 256-position blocks, so that one 16-byte load gives a lane
+// eight positions and a warp's ballots rank them by position); it stays in
+// L2:
 //   0. 1024 keys sampled at even strides give the bins: their range, widened
 //      by half on either side, split into 8192 bins of 2^s keys (a unit's
 //      scores may crowd into a few per cent of one octave, or spread over
 //      many octaves: the range adapts the bins to either);
-//   1. build the keys and histogram their bins (the two end bins also take
-//      every key outside the range);
+//   1. build the keys, store their bins and histogram them (the two end bins
+//      also take every key outside the range);
 //   2. with the bin d holding the k-th largest key found, each warp walks its
-//      segment of the keys in order: keys of higher bins are kept for sure
-//      and their positions are staged, in order, at the start of the
-//      segment's row; keys of bin d (the candidates) go to the warp's list in
-//      shared memory with the count of sure positions before them;
+//      segment of the bins in order: keys of higher bins are kept for sure
+//      and their positions are staged, in order, as 16-bit offsets at the
+//      start of the segment's row; keys of bin d (the candidates) go to the
+//      warp's list in shared memory with the count of sure positions before
+//      them, and their keys are recomputed from the scores;
 //   3. radix passes of up to 9 bits over the candidates fix the threshold key
 //      T and how many keys equal to T to keep (ties keep the lower position);
 //   4. every warp merges its staged positions and its kept candidates into
 //      its share of the output, after the shares of the warps before it.
 // An end bin, or a candidate list that overflows (many equal keys), takes the
-// general path instead: the keys are rebuilt, four 8-bit radix passes over
-// every key fix T, and one ordered pass writes the kept positions.
+// general path instead: the full keys are written to the row (transposed
+// 128-key blocks), four 8-bit radix passes over every key fix T, and one
+// ordered pass writes the kept positions.
 #include "kvev_internal.cuh"
 
 namespace kvev {
@@ -49,6 +52,7 @@ constexpr int kBins0 = 8192;               // bins of the sampled range
 constexpr int kCandPerWarp = 320;          // candidates a warp's list holds
 constexpr int kBins1 = 512;                // candidate digits: up to 9 bits a pass
 constexpr int kSegKeys = 128;              // a key block: four keys per lane
+constexpr int kBinBlock = 256;             // a bin block: eight positions per lane
 
 struct CandLists {
   uint32_t pos[kSW][kCandPerWarp];
@@ -146,10 +150,14 @@ __device__ void find_bin(const int* hist, int nbins, int kk, SelShared& sh, int&
   __syncthreads();  // wsum and bcast are reused by the next call
 }
 
-// Warp segments of [0, E): contiguous, whole 128-key iterations, in warp
+// Warp segments of [0, E): contiguous, whole 256-position blocks, in warp
 // order, so that a warp's kept positions follow those of the warps before it.
 __device__ __forceinline__ int seg_len(int E) {
-  return ((E + kSW - 1) / kSW + kSegKeys - 1) / kSegKeys * kSegKeys;
+  return ((E + kSW - 1) / kSW + kBinBlock - 1) / kBinBlock * kBinBlock;
+}
+
+__device__ __forceinline__ uint32_t pick(const uint4& v, int u) {
+  return u == 0 ? v.x : u == 1 ? v.y : u == 2 ? v.z : v.w;
 }
 
 // A key row holds 128-key blocks, each transposed: the key of position
@@ -164,9 +172,20 @@ __device__ __forceinline__ uint4 ld_block_keys(const uint32_t* keys, int b0) {
   return __ldcg(reinterpret_cast<const uint4*>(keys + b0 + 4 * (threadIdx.x & 31)));
 }
 
-__device__ __forceinline__ uint32_t pick(const uint4& v, int u) {
-  return u == 0 ? v.x : u == 1 ? v.y : u == 2 ? v.z : v.w;
+// The fast path keeps 16-bit bins instead of keys, in 256-position blocks
+// transposed the same way: the bin of position b + 32u + L (u < 8) sits at
+// 16-bit index b + 8L + u, so one 16-byte load gives lane L eight positions.
+__device__ __forceinline__ int tpos16(int i) { return (i & ~255) | ((i & 31) << 3) | ((i >> 5) & 7); }
+
+__device__ __forceinline__ uint4 ld_block_bins(const uint16_t* bins, int b0) {
+  return __ldcg(reinterpret_cast<const uint4*>(bins + b0 + 8 * (threadIdx.x & 31)));
 }
+
+__device__ __forceinline__ uint32_t pick16(const uint4& v, int u) {
+  const uint32_t w = pick(v, u >> 1);
+  return (u & 1) ? (w >> 16) : (w & 0xFFFFu);
+}
+
 
 // Bulk prefetch of the floats [src, src + n) into L2, in 16 KiB pieces, one
 // per thread (the row is 16-byte aligned and padded to whole 16-byte blocks).
@@ -327,10 +346,10 @@ __device__ Binning sample_binning(const Gen& gen, int E, SelShared& sh) {
   return make_binning(sh.rlo, sh.rhi);
 }
 
-// Step 1: every key of [0, E) into the unit's workspace row (transposed
-// blocks), and the histogram of their bins.
+// Step 1: the bin of every key of [0, E) into the unit's workspace row (16-bit
+// transposed blocks), and the histogram of the bins.
 template <class Gen>
-__device__ void build_row_hist(const Gen& gen, uint32_t* row, int E, Binning bn, int* hist) {
+__device__ void build_row_hist(const Gen& gen, uint16_t* bins, int E, Binning bn, int* hist) {
   typename Gen::Regs nxt;
   int i0 = 4 * threadIdx.x;
   if (i0 < E) gen.load(i0, nxt);
@@ -342,47 +361,50 @@ __device__ void build_row_hist(const Gen& gen, uint32_t* row, int E, Binning bn,
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       if (i0 + u < E) {
-        row[tpos(i0 + u)] = kq[u];
-        atomicAdd(&hist[bn.bin(kq[u])], 1);
+        const uint32_t b = bn.bin(kq[u]);
+        bins[tpos16(i0 + u)] = static_cast<uint16_t>(b);
+        atomicAdd(&hist[b], 1);
       }
     }
   }
 }
 
 // ---------------------------------------------------------------------------
-// Step 2: each warp walks its segment [lo, hi) of the keys in order.  Keys of
+// Step 2: each warp walks its segment [lo, hi) of the bins in order.  Keys of
 // bins above the bracket are kept for sure: their positions are staged, in
-// order, at the start of the segment's row (a warp only overwrites entries of
-// positions it has passed, and has the next block's keys in registers).  Keys
-// inside the bracket (the candidates) go to the warp's list with the count of
-// sure positions before them.  A list that fills up sets sh.overflow.
+// order, as 16-bit offsets at the start of the segment's row (a warp only
+// overwrites entries of positions it has passed, and has the next block's
+// bins in registers).  Keys inside the bracket (the candidates) go to the
+// warp's list with the count of sure positions before them; their keys are
+// recomputed from the scores afterwards.  A list that fills up sets
+// sh.overflow.
 // ---------------------------------------------------------------------------
-__device__ void classify_pass(uint32_t* row, int E, const Bracket& br, SelShared& sh) {
+__device__ void classify_pass(uint16_t* bins, int E, const Bracket& br, SelShared& sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint32_t lt = (1u << lane) - 1u;
   const int seg = seg_len(E);
   const int lo = min(warp * seg, E), hi = min(lo + seg, E);
   int ns = 0, nc = 0;  // sure positions staged, candidates listed
   uint4 nxt = make_uint4(0, 0, 0, 0);
-  if (lo < hi) nxt = ld_block_keys(row, lo);
-  for (int b0 = lo; b0 < hi; b0 += kSegKeys) {
+  if (lo < hi) nxt = ld_block_bins(bins, lo);
+  for (int b0 = lo; b0 < hi; b0 += kBinBlock) {
     const uint4 cur = nxt;
-    if (b0 + kSegKeys < hi) nxt = ld_block_keys(row, b0 + kSegKeys);  // the next block's keys go out first
+    if (b0 + kBinBlock < hi) nxt = ld_block_bins(bins, b0 + kBinBlock);  // the next block goes out first
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       const int p = b0 + 32 * u + lane;
-      const uint32_t q = br.bn.bin(pick(cur, u));
+      const uint32_t q = pick16(cur, u);
       const bool valid = p < hi;
       const bool sure = valid && q > br.hi_bin;
       const bool cand = valid && q >= br.lo_bin && q <= br.hi_bin;
       const uint32_t bs = __ballot_sync(0xffffffffu, sure), bc = __ballot_sync(0xffffffffu, cand);
       const int js = ns + __popc(bs & lt);
-      if (sure) row[lo + js] = static_cast<uint32_t>(p);
+      // staged as offsets from the segment start, behind the positions already read
+      if (sure) bins[lo + js] = static_cast<uint16_t>(p - lo);
       if (cand) {
         const int jc = nc + __popc(bc & lt);
         if (jc < kCandPerWarp) {
           sh.u.c.pos[warp][jc] = static_cast<uint32_t>(p);
-          sh.u.c.key[warp][jc] = pick(cur, u);
           sh.u.c.sure[warp][jc] = js;
         }
       }
@@ -395,6 +417,13 @@ __device__ void classify_pass(uint32_t* row, int E, const Bracket& br, SelShared
     sh.wC[warp] = nc;
     if (nc > kCandPerWarp) sh.overflow = 1;
   }
+}
+
+// The keys of each warp's listed candidates, from the scores.
+__device__ void candidate_keys(const Scalar4& sk, SelShared& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nc = min(sh.wC[warp], kCandPerWarp);
+  for (int i = lane; i < nc; i += 32) sh.u.c.key[warp][i] = sk.one(static_cast<int>(sh.u.c.pos[warp][i]));
 }
 
 // Step 3: threshold key T (the kk-th largest candidate) and how many keys
@@ -464,7 +493,7 @@ __device__ void select_candidates(int kk, SelShared& sh, uint32_t& T, int& need)
 // base + (sure positions before it) + (kept candidates before it); its sure
 // position j to base + j + (kept candidates with at most j sure positions
 // before them).
-__device__ void merge_write(const uint32_t* keys, int E, int k, int need, SelShared& sh, uint32_t T, int* out) {
+__device__ void merge_write(const uint16_t* bins, int E, int k, int need, SelShared& sh, uint32_t T, int* out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint32_t lt = (1u << lane) - 1u;
   int base = 0, eq_base = 0;
@@ -502,7 +531,7 @@ __device__ void merge_write(const uint32_t* keys, int E, int k, int need, SelSha
   const int lo = min(warp * seg, E);
   const int ns = sh.wS[warp];
   for (int j = lane; j < ns; j += 32) {
-    const int pos = static_cast<int>(__ldcg(keys + lo + j));
+    const int pos = lo + static_cast<int>(__ldcg(bins + lo + j));
     int a = 0, b = nk;  // kept candidates with sure[] <= j: the first index with sure[] > j
     while (a < b) {
       const int m = (a + b) >> 1;
@@ -611,7 +640,8 @@ __device__ void build_row(const Gen& gen, uint32_t* row, int E) {
 
 // Top-k of the keys of [0, E) (1 <= k < E) into out[0 .. k), ascending.
 template <class Gen>
-__device__ void select_unit(const Gen& gen, uint32_t* row, int E, int k, SelShared& sh, int* out) {
+__device__ void select_unit(const Gen& gen, const Scalar4& sk, uint32_t* row, int E, int k, SelShared& sh,
+                            int* out) {
   for (int i = threadIdx.x; i < kBins0; i += kSelectThreads) sh.u.hist[i] = 0;
   if (threadIdx.x == 0) {
     sh.rlo = 0xFFFFFFFFu;
@@ -620,33 +650,36 @@ __device__ void select_unit(const Gen& gen, uint32_t* row, int E, int k, SelShar
   }
   __syncthreads();
   const Binning bn = sample_binning(gen, E, sh);
-  build_row_hist(gen, row, E, bn, sh.u.hist);
+  uint16_t* bins = reinterpret_cast<uint16_t*>(row);
+  build_row_hist(gen, bins, E, bn, sh.u.hist);
   __syncthreads();
   int d, above;
   find_bin(sh.u.hist, kBins0, k, sh, d, above);  // ends with a barrier
   const int nd = sh.u.hist[d];
   __syncthreads();  // every thread has read it before the candidate lists overwrite the histogram
   // the end bins also hold keys outside the sampled range: not one prefix
-  bool fast = d > 0 && d < kBins0 - 1 && nd <= kSW * kCandPerWarp;
-  const bool staged = fast;
+  bool fast = d > 0 && d < kBins0 - 1 && nd <= kSW * kCandPerWarp && seg_len(E) <= 65536;
   if (fast) {
     const Bracket br{bn, static_cast<uint32_t>(d), static_cast<uint32_t>(d)};
-    classify_pass(row, E, br, sh);
+    classify_pass(bins, E, br, sh);
     __syncthreads();
     fast = !sh.overflow;
+    if (fast) {
+      candidate_keys(sk, sh);
+      __syncthreads();
+    }
   }
   uint32_t T;
   int need;
   if (fast) {
     select_candidates(k - above, sh, T, need);
-    merge_write(row, E, k, need, sh, T, out);
+    merge_write(bins, E, k, need, sh, T, out);
     return;
   }
-  // the general path: many equal keys, or a sample that missed the k-th key
-  if (staged) {
-    build_row(gen, row, E);
-    __syncthreads();
-  }
+  // the general path: many equal keys, or a sample that missed the k-th key:
+  // the row holds bins, so the keys are built now
+  build_row(gen, row, E);
+  __syncthreads();
   select_all_keys(row, E, k, sh, T, need);
   write_kept(row, E, k, T, need, sh, out);
 }
@@ -704,17 +737,18 @@ __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kerne
   const bool do_pool = ld.method == KVEV_SNAPKV, is_max = p.pool_type == KVEV_POOL_MAX;
   const bool aligned4 = (reinterpret_cast<uintptr_t>(raw) & 15u) == 0 && (p.S_cap & 3) == 0;
   if (aligned4) prefetch_row_l2(raw, E);  // the passes' score reads become L2 hits
-  if (aligned4 && !do_pool) return select_unit(Raw4{raw, E}, row, E, k, sh, idx);
+  const Scalar4 sk{raw, E, p.pool_kernel / 2, do_pool, is_max};  // one key at a time (candidates)
+  if (aligned4 && !do_pool) return select_unit(Raw4{raw, E}, sk, row, E, k, sh, idx);
   if (aligned4) {
     switch (p.pool_kernel) {
-      case 3: return select_unit(Pooled4<3>{raw, E, is_max}, row, E, k, sh, idx);
-      case 5: return select_unit(Pooled4<5>{raw, E, is_max}, row, E, k, sh, idx);
-      case 7: return select_unit(Pooled4<7>{raw, E, is_max}, row, E, k, sh, idx);
-      case 9: return select_unit(Pooled4<9>{raw, E, is_max}, row, E, k, sh, idx);
+      case 3: return select_unit(Pooled4<3>{raw, E, is_max}, sk, row, E, k, sh, idx);
+      case 5: return select_unit(Pooled4<5>{raw, E, is_max}, sk, row, E, k, sh, idx);
+      case 7: return select_unit(Pooled4<7>{raw, E, is_max}, sk, row, E, k, sh, idx);
+      case 9: return select_unit(Pooled4<9>{raw, E, is_max}, sk, row, E, k, sh, idx);
       default: break;
     }
   }
-  select_unit(Scalar4{raw, E, p.pool_kernel / 2, do_pool, is_max}, row, E, k, sh, idx);
+  select_unit(sk, sk, row, E, k, sh, idx);
 }
 
 }  // namespace
