@@ -546,14 +546,18 @@ def run_ours(args, rank, world, local_rank):
     mufu_peak = MUFU_EX2_PER_CLK_SM * n_sms * mhz * 1e6 / 1e9
     mufu_achieved = score_exp2(wl) / (score_ms / 1e3) / 1e9
     traffic = None
+    traffic_single = None  # the one-sweep form (window normalisers supplied)
     tf = os.path.join(ROOT, "profiles", "score_traffic.json")
     if os.path.exists(tf):
         try:
             t = json.load(open(tf))
             if t.get("workload") == wl.name and t.get("kernel_src_hash") == kernel_hash():
                 traffic = t["bytes_per_launch"]
+                traffic_single = t.get("single_sweep", {}).get("bytes_per_launch")
         except (OSError, ValueError, KeyError):
             pass
+    if args.lse_supplied:
+        traffic = traffic_single
 
     # ---- end to end through the C ABI with host buffers ----
     e2e = None
@@ -610,7 +614,7 @@ def run_ours(args, rank, world, local_rank):
             "kernel_ms": kms_l,
             "roofline": {"kernel": "score_kernel (one sweep)", "bound": "hbm", "achieved": ach_l,
                          "peak": hbm_peak, "unit": "GB/s", "frac": None if ach_l is None else ach_l / hbm_peak,
-                         "traffic": None},
+                         "traffic": traffic_single},
             "clocks": clk_l,
             "how": "kvev_evict_prefill_lse: the window rows' log-sum-exp supplied (as a caller's prefill "
                    "attention returns it; computed once, untimed), the score kernel makes one sweep"}
