@@ -363,7 +363,8 @@ def time_prefill(plan, wl, K, V, Q, lens, bufs, stream, steps, barrier, kvev, ls
         barrier()
     last = kvev.kvev_plan_last_timings(plan.handle)
     per_kernel = {k: (v if v >= 0 else None) for k, v in last.items()}
-    launched = sum(1 for v in last.values() if v >= 0) * steps
+    # the supplied normalisers' fill kernel runs inside the prologue's event pair
+    launched = (sum(1 for v in last.values() if v >= 0) + (1 if lse is not None else 0)) * steps
     return ev0.elapsed_time(ev1) / steps, per_kernel, clk.summary(), launched
 
 
@@ -655,7 +656,9 @@ def run_ours(args, rank, world, local_rank):
                                          "frac": perf / (score_ms / 1e3) / 1e12 / tc_peak,
                                          "work": "row pass + key pass, 256 x 256 tiles"}},
             "clocks": clocks,
-            "gpu_launches": args.steps * 6,  # prologue, window scores, row pass, key pass, select, gather
+            # prologue, window scores, row pass (or, with --lse-supplied, the two normaliser fills
+            # instead), key pass, select, gather
+            "gpu_launches": args.steps * (7 if args.lse_supplied else 6),
             "e2e": None, "cpu_baseline": None,
         }
         print(json.dumps(out), flush=True)
