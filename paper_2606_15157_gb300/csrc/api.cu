@@ -570,18 +570,18 @@ int evict_prefill_impl(kvev_plan* plan, const void* const* K, const void* const*
   int rc = check_prefill_args(P, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
                               out_count);
   if (rc != KVEV_OK) return rc;
-  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return KVEV_EINVAL;
-  if (workspace_bytes < ws_layout(P, B, S_cap).total) return KVEV_ENOMEM;
-  rc = ensure_device(plan);
-  if (rc != KVEV_OK) return rc;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  P.last_stream = s;
   if (lse_win) {  // every scored layer needs its rows' log-sum-exp
     for (int l = 0; l < P.L; ++l)
       if (is_scoring(P.route_pre[l]) &&
           (!lse_win[l] || (reinterpret_cast<uintptr_t>(lse_win[l]) & 3u)))
         return KVEV_EINVAL;
   }
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return KVEV_EINVAL;
+  if (workspace_bytes < ws_layout(P, B, S_cap).total) return KVEV_ENOMEM;
+  rc = ensure_device(plan);
+  if (rc != KVEV_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  P.last_stream = s;
   return evict_impl(P, P.ctx, K, V, Q_win, scores, lens_dev, B, S_cap, out_K, out_V, out_idx,
                     out_count, h2o_state, workspace, s, lse_win);
 }

@@ -178,6 +178,15 @@ def test_evict_argument_errors_before_device_work(kv):
     assert kv.kvev_evict_prefill_scored(**dict(sargs, Q_ptrs=[None, fake], score_ptrs=[fake + 2, None])) == kv.EINVAL
     assert kv.kvev_evict_prefill_scored(**dict(sargs, Q_ptrs=[None, fake], score_ptrs=[fake, None],
                                                 workspace_bytes=64)) == kv.ENOMEM  # past the checks
+    # caller-supplied normalisers: required for the scoring layer (layer 0), 4-byte aligned;
+    # the StreamingLLM layer's entry is ignored
+    largs = dict(args, lse_ptrs=[fake, None])
+    assert kv.kvev_evict_prefill_lse(**dict(largs, lse_ptrs=None)) == kv.EINVAL
+    assert kv.kvev_evict_prefill_lse(**dict(largs, lse_ptrs=[None, fake])) == kv.EINVAL
+    assert kv.kvev_evict_prefill_lse(**dict(largs, lse_ptrs=[fake + 2, None])) == kv.EINVAL
+    assert kv.kvev_evict_prefill_lse(**dict(largs, Q_ptrs=[None, fake])) == kv.EINVAL  # Q_win still read
+    assert kv.kvev_evict_prefill_lse(**dict(largs, workspace_bytes=64)) == kv.ENOMEM   # past the checks
+    assert kv.kvev_evict_prefill_lse(**dict(largs, B=0)) == kv.OK
     kv.kvev_plan_destroy(h)
 
 
