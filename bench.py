@@ -751,7 +751,8 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
     Q_win of the SnapKV / H2O layers) are copied to the device on four copy
     streams, and the tensors that are only gathered row by row (V of every
     layer, K of the StreamingLLM layers) stay in pinned host memory, read in
-    place over the host link by the gather kernel; the kept indices and counts
+    place over the host link by the gather kernel (by the selection kernel for
+    the StreamingLLM layers); the kept indices and counts
     are read back.  Steps alternate between two device copies of the streamed
     inputs, so a step's uploads overlap the previous step's eviction (each step
     still uploads its own inputs and reads back its own result).  The bytes
@@ -831,7 +832,7 @@ def run_e2e(args, wl, plan, dev, lens_dev, stream, tot_bytes, barrier, max_over_
     for _ in range(args.warmup):
         step()
     stream.synchronize()
-    # rows the gather reads in place from host memory: every kept row of V, and
+    # rows read in place from host memory: every kept row of V, and
     # of K for the layers whose K stays on the host (FULL layers keep nothing)
     row = wl.d * 2
     counts = cnt_h.numpy().reshape(wl.L, -1)

@@ -652,8 +652,6 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
                float* h2o_state, void* workspace, cudaStream_t s, const float* const* lse_win) {
   auto supplied = [&](int l) { return scores != nullptr && scores[l] != nullptr; };
   if (static_cast<int64_t>(B) * P.H_kv * S_cap > (1LL << 31) - 1) return KVEV_ENOTSUP;
-  int64_t total_rows = 0;
-  for (int l = 0; l < P.L; ++l) total_rows += rows_per_layer(P, B, l);
   const WsLayout ws = ws_layout(P, B, S_cap);
   uint8_t* wsb = static_cast<uint8_t*>(workspace);
   int* lens_ok = reinterpret_cast<int*>(wsb + ws.lens);
@@ -856,7 +854,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   std::memset(&sel, 0, sizeof(sel));
   GatherParams ga;
   std::memset(&ga, 0, sizeof(ga));
-  int64_t off = 0;
+  int64_t off = 0, goff = 0;
   for (int l = 0; l < P.L; ++l) {
     LayerDesc ld;
     ld.method = P.route_pre[l];
@@ -870,12 +868,18 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
       ld.scores = supplied(l) ? scores[l]
                               : reinterpret_cast<const float*>(wsb + ws.raw) +
                                     static_cast<size_t>(ld.score_slot) * B * P.H_kv * S_cap;
+    ga.grow_off[l] = goff;
+    if (is_scoring(ld.method)) goff += rows_per_layer(P, B, l);  // StreamingLLM rows: selection launch
     off += rows_per_layer(P, B, l);
     sel.layer[l] = ld;
     ga.layer[l] = ld;
-    ga.K[l] = K[l];
-    ga.V[l] = V[l];
+    ga.K[l] = sel.K[l] = K[l];
+    ga.V[l] = sel.V[l] = V[l];
   }
+  for (int l = 0; l < P.L; ++l)  // selection dispatch: scoring layers first
+    if (is_scoring(P.route_pre[l])) sel.order[sel.L_first++] = l;
+  for (int l = 0, j = sel.L_first; l < P.L; ++l)
+    if (!is_scoring(P.route_pre[l])) sel.order[j++] = l;
   sel.L = P.L;
   sel.B = B;
   sel.H_kv = P.H_kv;
@@ -884,6 +888,9 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   sel.pool_kernel = P.pool_kernel;
   sel.pool_type = P.pool_type;
   sel.sink = P.sink;
+  sel.d = P.d;
+  sel.out_K = out_K;
+  sel.out_V = out_V;
   sel.lens = lens_ok;
   sel.out_idx = out_idx;
   sel.out_count = out_count;
@@ -899,7 +906,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   ga.H_kv = P.H_kv;
   ga.S_cap = S_cap;
   ga.d = P.d;
-  ga.total_rows = total_rows;
+  ga.total_rows = goff;
   ga.out_idx = out_idx;
   ga.out_K = out_K;
   ga.out_V = out_V;
@@ -907,7 +914,7 @@ int evict_impl(kvev_plan& P, DevCtx& D, const void* const* K, const void* const*
   ga.status = D.status;
   mark(KVEV_K_GATHER, 0);
   if (launch_gather(ga, s, D.num_sms) != cudaSuccess) return KVEV_ECUDA;
-  if (total_rows > 0) mark(KVEV_K_GATHER, 1);
+  if (goff > 0) mark(KVEV_K_GATHER, 1);
   return KVEV_OK;
 }
 

@@ -1,5 +1,7 @@
-// gather.cu -- gather-compaction of the kept K/V rows of every non-FULL layer
-// into the packed output cache, in one grid-stride launch.
+// gather.cu -- gather-compaction of the kept K/V rows of every SnapKV and H2O
+// layer into the packed output cache, in one grid-stride launch (the
+// StreamingLLM layers' rows, whose positions need no scores, are copied by the
+// selection launch).
 //
 // Output row (layer l, unit (s, h), slot j) = K[l][s][h][out_idx[row]] and the
 // same for V; slots past the kept count (out_idx = -1) are zero-filled.  For
@@ -17,14 +19,15 @@ namespace {
 
 constexpr int kGatherThreads = 256;
 
-// Layer owning packed row `row`: the last layer whose first row is <= row.  A
-// FULL layer owns no rows and shares its row_off with the next layer, so the
-// search (which takes the highest such index) never lands on it.
-__device__ __forceinline__ int find_layer(const GatherParams& p, long long row) {
+// Layer owning gathered row `g`: the last layer whose first gathered row is
+// <= g.  FULL and StreamingLLM layers own no gathered rows and share their
+// grow_off with the next layer, so the search (which takes the highest such
+// index) never lands on them.
+__device__ __forceinline__ int find_layer(const GatherParams& p, long long g) {
   int lo = 0, hi = p.L - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (p.layer[mid].row_off <= row) lo = mid;
+    if (p.grow_off[mid] <= g) lo = mid;
     else hi = mid - 1;
   }
   return lo;
@@ -35,11 +38,12 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const __grid_con
   const int rows_per_block = kGatherThreads / tpr;
   const int sub = threadIdx.x % tpr;
   const long long step = static_cast<long long>(gridDim.x) * rows_per_block;
-  for (long long row = static_cast<long long>(blockIdx.x) * rows_per_block + threadIdx.x / tpr;
-       row < p.total_rows; row += step) {
-    const int l = find_layer(p, row);
+  for (long long g = static_cast<long long>(blockIdx.x) * rows_per_block + threadIdx.x / tpr;
+       g < p.total_rows; g += step) {
+    const int l = find_layer(p, g);
     const LayerDesc& ld = p.layer[l];
-    const long long local = row - ld.row_off;
+    const long long local = g - p.grow_off[l];
+    const long long row = ld.row_off + local;  // packed output row
     const int rem = static_cast<int>(local / ld.slots);
     int pos = p.out_idx[row];
     if (pos >= p.S_cap) {  // never produced by the selection; guard the loads anyway

@@ -131,12 +131,19 @@ struct LseParams {
 
 struct SelectParams {
   LayerDesc layer[kMaxLayers];
-  int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink;
+  int order[kMaxLayers];  // layers in dispatch order: the L_first scoring layers, then the rest
+  int L_first;
+  int L, B, H_kv, S_cap, W, pool_kernel, pool_type, sink, d;
   const int* lens;
   int* out_idx;
   int* out_count;     // [L][B][H_kv]
   uint32_t* keys;     // workspace: [scoring unit][key_stride] selection keys
   int key_stride;     // S_cap rounded up to a multiple of 128 (whole transposed key blocks)
+  // StreamingLLM layers: their kept rows are copied by the selection launch
+  const void* K[kMaxLayers];
+  const void* V[kMaxLayers];
+  void* out_K;
+  void* out_V;
 };
 
 // Per-layer description of the decode arena.
@@ -186,8 +193,9 @@ struct GatherParams {
   LayerDesc layer[kMaxLayers];
   const void* K[kMaxLayers];
   const void* V[kMaxLayers];
+  long long grow_off[kMaxLayers];  // first gathered row of the layer (SnapKV / H2O layers own rows)
   int L, B, H_kv, S_cap, d;
-  long long total_rows;
+  long long total_rows;  // gathered rows: the packed rows of the SnapKV and H2O layers
   const int* out_idx;
   void* out_K;
   void* out_V;

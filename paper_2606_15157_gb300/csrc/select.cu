@@ -9,10 +9,18 @@
 //              positions plus the window [E, n).
 //   H2O      : E = n - r (r = protected recent window); keys = raw window
 //              scores; keep the top (b - r) of [0, E) plus [E, n).
-//   Streaming: keep [0, sink) plus the last `recent` positions (closed form).
+//   Streaming: keep [0, sink) plus the last `recent` positions (closed form);
+//              this launch also copies those K/V rows into the packed cache
+//              (they need no scores, and the selection leaves HBM mostly
+//              idle), so the gather launch skips these layers.
 //   b >= n   : keep every position.
 // Top-k order: larger score first, equal scores keep the lower position.
 // Output indices are ascending; unused slots hold -1.
+//
+// CTAs take the SnapKV / H2O units longest sequence first (the units of the
+// longest sequence, then of the next one ...), so the long selections start
+// early; the StreamingLLM and FULL units are spread evenly between them, so
+// that the copies' HBM traffic overlaps the latency-bound selections.
 //
 // A unit takes a CTA of 256 threads, so that several units share an SM and
 // one unit's barriers and round trips overlap another's passes.  Keys are an
@@ -684,12 +692,84 @@ __device__ void select_unit(const Gen& gen, const Scalar4& sk, uint32_t* row, in
   write_kept(row, E, k, T, need, sh, out);
 }
 
+// The sequence of rank r in order of decreasing length (equal lengths: lower
+// index first), by warp 0 (B <= 32; larger batches keep the index order).
+__device__ int seq_of_rank(const SelectParams& p, int r, SelShared& sh) {
+  if (p.B > 32) return r;
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    const int n = lane < p.B ? p.lens[lane] : -1;
+    int rank = 0;
+    for (int j = 0; j < p.B; ++j) {
+      const int nj = __shfl_sync(0xffffffffu, n, j);
+      rank += nj > n || (nj == n && j < lane);
+    }
+    const uint32_t m = __ballot_sync(0xffffffffu, lane < p.B && rank == r);
+    if (lane == 0) sh.bcast[0] = __ffs(m) - 1;
+  }
+  __syncthreads();
+  return sh.bcast[0];
+}
+
+// A StreamingLLM unit's kept rows (positions pos_j of slots j < count) into its
+// packed output rows, K and V as 16-byte vectors, four of each in flight per
+// thread; slots past the count are zero-filled.
+__device__ void copy_streaming_rows(const SelectParams& p, int l, int rem, int n, int count, bool identity) {
+  const LayerDesc& ld = p.layer[l];
+  const int vec = p.d / 8, total = ld.slots * vec;
+  const size_t src0 = static_cast<size_t>(rem) * p.S_cap * vec;
+  const size_t dst0 = (static_cast<size_t>(ld.row_off) + static_cast<size_t>(rem) * ld.slots) * vec;
+  const uint4* Ks = static_cast<const uint4*>(p.K[l]) + src0;
+  const uint4* Vs = static_cast<const uint4*>(p.V[l]) + src0;
+  uint4* Kd = static_cast<uint4*>(p.out_K) + dst0;
+  uint4* Vd = static_cast<uint4*>(p.out_V) + dst0;
+  constexpr int kU = 4;
+  for (int i0 = threadIdx.x; i0 < total; i0 += kU * kSelectThreads) {
+    uint4 kv[kU], vv[kU];
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int i = i0 + q * kSelectThreads;
+      kv[q] = make_uint4(0, 0, 0, 0);
+      vv[q] = make_uint4(0, 0, 0, 0);
+      const int j = i / vec;
+      if (i < total && j < count) {
+        const int pos = identity || j < p.sink ? j : n - ld.recent + (j - p.sink);
+        const size_t e = static_cast<size_t>(pos) * vec + (i - j * vec);
+        kv[q] = __ldg(Ks + e);
+        vv[q] = __ldg(Vs + e);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int i = i0 + q * kSelectThreads;
+      if (i < total) {
+        __stcs(Kd + i, kv[q]);
+        __stcs(Vd + i, vv[q]);
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kernel(const __grid_constant__ SelectParams p) {
   __shared__ SelShared sh;
   const int per_layer = p.B * p.H_kv;
-  const int l = blockIdx.x / per_layer;
-  const int rem = blockIdx.x - l * per_layer;
-  const int s = rem / p.H_kv;
+  // dispatch order: two lists, each in (sequence rank, layer, head) order --
+  // the first L_first layers of p.order (the scoring layers) and the rest --
+  // merged evenly: CTA b takes the c-th unit of the second list when
+  // c = floor(b n2 / N) steps up at b, else the (b - c)-th of the first
+  const long long N = static_cast<long long>(p.L) * per_layer;
+  const long long n2 = static_cast<long long>(p.L - p.L_first) * per_layer;
+  const int c = static_cast<int>(blockIdx.x * n2 / N);
+  const bool second = (blockIdx.x + 1) * n2 / N > c;
+  int b = second ? c : static_cast<int>(blockIdx.x) - c;
+  const int first = second ? p.L_first : 0;
+  const int nl = second ? p.L - p.L_first : p.L_first;
+  const int r = b / (nl * p.H_kv);
+  const int t = b - r * nl * p.H_kv;
+  const int l = p.order[first + t / p.H_kv];
+  const int h = t - (t / p.H_kv) * p.H_kv;
+  const int s = seq_of_rank(p, r, sh);
+  const int rem = s * p.H_kv + h;
   const LayerDesc ld = p.layer[l];
   const int n = p.lens[s];
   int* cnt = p.out_count + static_cast<size_t>(l) * per_layer + rem;
@@ -697,8 +777,8 @@ __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kerne
     if (threadIdx.x == 0) *cnt = n;
     return;
   }
-  const int b = ld.slots;
-  int* idx = p.out_idx + ld.row_off + static_cast<long long>(rem) * b;
+  const int b_l = ld.slots;
+  int* idx = p.out_idx + ld.row_off + static_cast<long long>(rem) * b_l;
 
   int count, E = n, k = 0;  // select top-k of [0, E), then keep [E, n)
   bool identity = false;
@@ -710,18 +790,19 @@ __global__ void __launch_bounds__(kSelectThreads, kSelectCtasPerSm) select_kerne
       for (int j = threadIdx.x; j < count; j += blockDim.x)
         idx[j] = j < p.sink ? j : n - ld.recent + (j - p.sink);
     }
+    copy_streaming_rows(p, l, rem, n, count, identity);
   } else {
-    identity = n <= b;
-    count = identity ? n : b;
+    identity = n <= b_l;
+    count = identity ? n : b_l;
     if (!identity) {
       const int protect = ld.method == KVEV_SNAPKV ? p.W : ld.h2o_recent;
       E = n - protect;
-      k = b - protect;
+      k = b_l - protect;
     }
   }
   if (identity)
     for (int j = threadIdx.x; j < n; j += blockDim.x) idx[j] = j;
-  for (int j = count + threadIdx.x; j < b; j += blockDim.x) idx[j] = -1;
+  for (int j = count + threadIdx.x; j < b_l; j += blockDim.x) idx[j] = -1;
   if (threadIdx.x == 0) *cnt = count;
   if (identity || ld.method == KVEV_STREAMING) return;
 
