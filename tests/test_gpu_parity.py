@@ -247,6 +247,27 @@ def test_edge_lengths(torch, orc, d):
     parity.check_workload(wl, dev, wl.lens)
 
 
+def test_selection_dispatch_orders(torch, orc):
+    # The selection launch takes the SnapKV / H2O units longest sequence first
+    # (sequences ranked by warp 0, up to 32 of them; larger batches keep the
+    # index order), with the StreamingLLM units (which also copy their kept
+    # rows) and FULL units spread between them.  Cases: 40 ragged sequences (the
+    # index order), equal lengths (rank ties), a route with no scoring layer
+    # and one with no StreamingLLM or FULL layer.
+    rng = np.random.default_rng(11)
+    lens40 = rng.integers(150, 600, size=40)
+    lens40[[3, 17, 31]] = 600  # ties across the first 32 and past them
+    cases = [
+        ([gen.STREAMING, gen.SNAPKV, gen.FULL, gen.H2O], [40, 64, 0, 90], lens40),
+        ([gen.SNAPKV, gen.STREAMING, gen.H2O], [48, 40, 70], [500, 500, 320, 500, 320]),
+        ([gen.STREAMING, gen.FULL, gen.STREAMING], [40, 0, 24], [700, 30, 455]),
+        ([gen.SNAPKV, gen.H2O], [64, 100], [900, 300, 1200]),
+    ]
+    for routes, budgets, lens in cases:
+        wl = _custom(routes, budgets, lens, H_q=4, H_kv=2, d=64)
+        parity.check_workload(wl, device_workload(wl), wl.lens)
+
+
 def test_edge_window_and_groups(torch, orc):
     # Different GQA group sizes and windows: R = G*W = 16, 48 (a 16-column tail), 128, 192, 256.
     for (H_q, H_kv, W) in [(4, 2, 8), (12, 4, 16), (8, 2, 32), (12, 2, 32), (32, 8, 64)]:
