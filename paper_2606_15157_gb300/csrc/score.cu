@@ -711,39 +711,50 @@ __global__ void __launch_bounds__(kScoreThreads, 1) score_kernel(const __grid_co
 
 // ---------------------------------------------------------------------------
 // Prologue: per-unit chunk counts, prefix sums, item -> unit map, flag reset.
+// Each CTA takes a contiguous slice of the units: it scans the chunk counts
+// of every unit up to the end of its slice (a few block-wide scans; the
+// counts are cheap to recompute) and writes its units' start offsets, work
+// items and cleared merge-tree counters, so that the writes are spread over
+// the grid instead of queued behind one SM.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ PrologueParams p) {
   __shared__ int warp_sums[32];
   __shared__ int carry;
   const int tid = threadIdx.x;
-  if (tid == 0) {
-    carry = 0;
-    *p.abort_flag = 0;
-  }
-  for (int i = tid; i < p.n_node_cnt; i += blockDim.x) p.node_cnt[i] = 0;
-  for (int s = tid; s < p.B; s += blockDim.x) {
-    int n = p.lens_in[s];
-    if (n < 0 || n > p.S_cap) {
-      atomicOr(p.status, kStatusDevice);
-      n = 0;
+  const int slice = (p.n_units + gridDim.x - 1) / gridDim.x;
+  const int u0 = min(static_cast<int>(blockIdx.x) * slice, p.n_units);
+  const int u1 = min(u0 + slice, p.n_units);
+  if (tid == 0) carry = 0;
+  if (blockIdx.x == 0) {
+    if (tid == 0) *p.abort_flag = 0;
+    for (int s = tid; s < p.B; s += blockDim.x) {
+      int n = p.lens_in[s];
+      if (n < 0 || n > p.S_cap) {
+        atomicOr(p.status, kStatusDevice);
+        n = 0;
+      }
+      p.lens[s] = n;
     }
-    p.lens[s] = n;
   }
   __syncthreads();
+  if (u0 == u1) {  // an empty slice (or no scoring units at all)
+    if (p.n_units == 0 && blockIdx.x == 0 && tid == 0) p.chunk_start[0] = 0;
+    return;
+  }
   const int per_layer = p.B * p.H_kv;
-  for (int base = 0; base < p.n_units; base += blockDim.x) {
+  for (int base = 0; base < u1; base += blockDim.x) {
     const int u = base + tid;
-    int c = 0;
+    int c = 0, n = 0;
     if (u < p.n_units) {
       const int ls = u / per_layer;
       const int s = (u - ls * per_layer) / p.H_kv;
-      const int n = p.lens[s];
+      n = p.lens_in[s];
+      if (n < 0 || n > p.S_cap) n = 0;  // flagged by CTA 0
       const bool h2o = p.slayer_method[ls] == KVEV_H2O;
       // H2O layers scored over the whole prompt have their own kernels
       const bool need =
           n > 0 && !p.slayer_ext[ls] && (h2o ? p.mode != kScoreNoH2O : n > p.slayer_budget[ls]);
       c = need ? (n + p.chunk_keys - 1) / p.chunk_keys : 0;
-      p.ready[u] = 0;
     }
     // block-wide exclusive scan of c
     int x = c;
@@ -766,21 +777,27 @@ __global__ void __launch_bounds__(1024) prologue_kernel(const __grid_constant__ 
     }
     __syncthreads();
     const int excl = carry + (w > 0 ? warp_sums[w - 1] : 0) + x - c;
-    if (u < p.n_units) {
+    if (u >= u0 && u < u1) {
       p.chunk_start[u] = excl;
-      const int n = p.lens[(u % per_layer) / p.H_kv];
+      p.ready[u] = 0;
+      if ((excl + c) * kTreeLevels > p.n_node_cnt) {  // never for a workspace of ws_layout's size
+        atomicOr(p.status, kStatusDevice);
+        c = 0;
+      }
       for (int q = 0; q < c; ++q) {
         const int key0 = q * p.chunk_keys;
         const int nk = min(p.chunk_keys, n - key0);
         const int ntiles = (nk + kTileKeys - 1) / kTileKeys;
         p.item[excl + q] = make_int4(u, n, key0, ntiles | (c << 16));
+#pragma unroll
+        for (int lv = 0; lv < kTreeLevels; ++lv) p.node_cnt[(excl + q) * kTreeLevels + lv] = 0;
       }
     }
     __syncthreads();
     if (tid == blockDim.x - 1) carry = excl + c;
     __syncthreads();
   }
-  if (tid == 0) p.chunk_start[p.n_units] = carry;
+  if (u1 == p.n_units && tid == 0) p.chunk_start[p.n_units] = carry;
 }
 
 // ---------------------------------------------------------------------------
@@ -841,7 +858,10 @@ cudaError_t score_set_smem(int d, size_t smem) {
 }
 
 cudaError_t launch_prologue(const PrologueParams& p, cudaStream_t s) {
-  prologue_kernel<<<1, 1024, 0, s>>>(p);
+  // about 128 units per CTA
+  const int want = (p.n_units + 127) / 128;
+  const int grid = want < 1 ? 1 : want > 256 ? 256 : want;
+  prologue_kernel<<<grid, 1024, 0, s>>>(p);
   return cudaGetLastError();
 }
 
